@@ -1,0 +1,60 @@
+"""Pure-Python brute force of one CLEAR-MoE FFN token (test infrastructure; tiny shapes only).
+
+Per token and per output element, with Python floats and math.erf, in the factorised order
+y_i = sum_k U[i][k] S[k] (sum_j Vh[k][j] z_j) + sum_j R_a[i][j] z_j: it never forms W_shared,
+never sorts or permutes, and shares no code with `oracle.clearmoe`, so the two pin each other.
+"""
+from __future__ import annotations
+
+import math
+
+
+def _gelu(u: float) -> float:
+    return u * 0.5 * (1.0 + math.erf(u / math.sqrt(2.0)))
+
+
+def token_expert(x_t, Wg, bg) -> int:
+    best_e, best = 0, None
+    for e in range(len(Wg)):
+        s = float(bg[e])
+        for k in range(len(x_t)):
+            s += float(Wg[e][k]) * float(x_t[k])
+        if best is None or s > best:  # strict: an equal later logit never wins
+            best_e, best = e, s
+    return best_e
+
+
+def token_forward(x_t, W1, b1, U, S, Vh, residuals, e: int):
+    H, d, r = len(W1), len(x_t), len(S)
+    z = []
+    for j in range(H):
+        u = float(b1[j])
+        for k in range(d):
+            u += float(W1[j][k]) * float(x_t[k])
+        z.append(_gelu(u))
+    proj = []
+    for k in range(r):
+        s = 0.0
+        for j in range(H):
+            s += float(Vh[k][j]) * z[j]
+        proj.append(float(S[k]) * s)
+    R = residuals[e]
+    y = []
+    for i in range(len(U)):
+        acc = 0.0
+        for k in range(r):
+            acc += float(U[i][k]) * proj[k]
+        for j in range(H):
+            acc += float(R[i][j]) * z[j]
+        y.append(acc)
+    return y
+
+
+def layer(x, W1, b1, U, S, Vh, residuals, Wg, bg):
+    """Returns (expert per token, output rows) for every token of x."""
+    a, y = [], []
+    for x_t in x:
+        e = token_expert(x_t, Wg, bg)
+        a.append(e)
+        y.append(token_forward(x_t, W1, b1, U, S, Vh, residuals, e))
+    return a, y

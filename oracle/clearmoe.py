@@ -1,0 +1,157 @@
+"""Float64 oracle of one CLEAR-MoE FFN layer (test infrastructure; see the package docstring).
+
+Notation follows the paper: tokens x [T x d], fc1 W1 [H x d] + b1 [H], z = GELU(fc1(x)) [T x H],
+fc2 W2 [d x H], truncated SVD W_shared = U_r Sigma_r V_r^T with U_r [d x r], Sigma_r = diag(S_r),
+V_r^T = Vh_r [r x H], residual experts W_e^res [d x H], linear router W_g [E x d], b_g [E].
+
+Every step is taken in the order of Algorithm 3:
+  1. z <- GELU(fc1(x))                      (shared, all tokens)
+  2. h_sh <- z W_shared^T                    (W_shared materialised, as the paper does)
+  3. a <- argmax(g(x))                       (top-1 expert assignment)
+  4. sort z by a; sub-batch boundaries       (stable sort; counts and offsets)
+  5. h_res[e] <- z_e (W_e^res)^T             (one product per expert sub-batch)
+  6. unshuffle h_res; y <- h_sh + h_res
+"""
+from __future__ import annotations
+
+import numpy as np
+from scipy.special import erf
+
+NEAR_TIE_REL = 1e-5  # router-logit top-2 gap below which a token's expert is not compared
+LN_EPS = 1e-6
+
+
+def f64(a) -> np.ndarray:
+    return np.asarray(a, dtype=np.float64)
+
+
+# ---------------------------------------------------------------- quantisation point (bf16)
+def to_bf16(v) -> np.ndarray:
+    """Round float64 values to the nearest bf16 (8 significant bits), ties to even.
+
+    v = m * 2**e with 0.5 <= |m| < 1 (frexp); bf16 keeps 8 bits of m, so the result is
+    rint(m * 2**8) * 2**(e - 8), and numpy's rint rounds halves to even."""
+    m, e = np.frexp(f64(v))
+    return np.ldexp(np.rint(np.ldexp(m, 8)), e - 8)
+
+
+# ---------------------------------------------------------------- Phase 4 router + Alg. 3 step 3
+def router_logits(x, Wg, bg, precision=np.float64) -> np.ndarray:
+    """Linear router g(x) = W_g x + b_g (Section "Phase 4: Router Fitting", Linear router with
+    d x E weights and a bias per expert)."""
+    x, Wg, bg = (np.asarray(a, dtype=precision) for a in (x, Wg, bg))
+    return x @ Wg.T + bg
+
+
+def argmax_lowest(logits) -> np.ndarray:
+    """a_t = min{e : logit_{t,e} = max_e logit_{t,e}} (Algorithm 3, "a <- argmax g(x)"; the
+    paper leaves ties open, the lowest index wins here)."""
+    return np.argmax(logits, axis=1).astype(np.int64)  # numpy returns the first maximum
+
+
+def near_ties(x, Wg, bg, rel=NEAR_TIE_REL) -> np.ndarray:
+    """Tokens whose top-2 router logits (float64) differ by less than rel * max(|l1|, |l2|)."""
+    lg = router_logits(x, Wg, bg)
+    if lg.shape[1] < 2:
+        return np.zeros(lg.shape[0], dtype=bool)
+    top = np.sort(lg, axis=1)[:, -2:]
+    gap = top[:, 1] - top[:, 0]
+    scale = np.maximum(np.abs(top[:, 0]), np.abs(top[:, 1]))
+    return gap <= rel * scale
+
+
+def route(x, Wg, bg) -> dict:
+    """Algorithm 3 steps 3-4: expert index per token, then "sort z by a" with sub-batch
+    boundaries. The decision is taken on float32 logits (the precision the router is run in);
+    the sort is stable (ascending token id within an expert)."""
+    E = np.asarray(Wg).shape[0]
+    a = argmax_lowest(router_logits(x, Wg, bg, precision=np.float32))
+    return sort_by_expert(a, E) | dict(near_tie=near_ties(x, Wg, bg))
+
+
+def sort_by_expert(a, E: int) -> dict:
+    """counts_e = |{t : a_t = e}|, offsets = exclusive prefix sum (E + 1 entries),
+    perm[slot] = token, tokens of expert e in slots [offsets_e, offsets_{e+1}) in id order."""
+    a = np.asarray(a, dtype=np.int64)
+    counts = np.bincount(a, minlength=E).astype(np.int64)
+    offsets = np.concatenate([[0], np.cumsum(counts)]).astype(np.int64)
+    perm = np.argsort(a, kind="stable").astype(np.int64)
+    return dict(a=a, counts=counts, offsets=offsets, perm=perm)
+
+
+# ---------------------------------------------------------------- Eq. 2 pieces
+def gelu(u) -> np.ndarray:
+    """GELU(u) = u * Phi(u), Phi the standard normal CDF = (1 + erf(u / sqrt 2)) / 2."""
+    u = f64(u)
+    return u * 0.5 * (1.0 + erf(u / np.sqrt(2.0)))
+
+
+def fc1_gelu(x, W1, b1, z_bf16: bool = False) -> np.ndarray:
+    """z = GELU(fc1(x)) = GELU(x W1^T + b1) (Eq. 2; Algorithm 3 step 1). With z_bf16 the
+    hidden state is stored in bf16, as the bf16 layer stores it."""
+    z = gelu(f64(x) @ f64(W1).T + f64(b1))
+    return to_bf16(z) if z_bf16 else z
+
+
+def shared_weight(U, S, Vh) -> np.ndarray:
+    """W_shared = U_r Sigma_r V_r^T, materialised as a dense d x H matrix (Eq. 2 and the
+    Phase 3 text: materialised before inference, no factorised compute)."""
+    return f64(U) @ np.diag(f64(S)) @ f64(Vh)
+
+
+def experts_forward(z, W_sh, residuals, a) -> np.ndarray:
+    """Algorithm 3 steps 2 and 4-6 on hidden states z [T x H] with assignment a [T]."""
+    z = f64(z)
+    T = z.shape[0]
+    E = len(residuals)
+    h_sh = z @ f64(W_sh).T                                   # step 2
+    srt = sort_by_expert(a, E)                               # step 4
+    z_sorted = z[srt["perm"]]
+    h_res_sorted = np.zeros((T, f64(W_sh).shape[0]))
+    for e in range(E):                                       # step 5
+        lo, hi = srt["offsets"][e], srt["offsets"][e + 1]
+        if hi > lo:
+            h_res_sorted[lo:hi] = z_sorted[lo:hi] @ f64(residuals[e]).T
+    h_res = np.empty_like(h_res_sorted)
+    h_res[srt["perm"]] = h_res_sorted                        # step 6: unshuffle
+    return h_sh + h_res
+
+
+def ffn_forward(x, W1, b1, U, S, Vh, residuals, Wg=None, bg=None, a=None,
+                z_bf16: bool = False) -> np.ndarray:
+    """y = W_shared z + W_{a}^res z, z = GELU(fc1(x)) (Eq. 2 / Algorithm 3). `a` overrides the
+    router's assignment (random routing, or the near-tie substitution of the parity tests)."""
+    if a is None:
+        a = route(x, Wg, bg)["a"]
+    z = fc1_gelu(x, W1, b1, z_bf16)
+    return experts_forward(z, shared_weight(U, S, Vh), residuals, a)
+
+
+def dense_ffn(x, W1, b1, W2, z_bf16: bool = False) -> np.ndarray:
+    """The unconverted layer: y = W2 GELU(W1 x + b1) (the dense FFN, D0)."""
+    return fc1_gelu(x, W1, b1, z_bf16) @ f64(W2).T
+
+
+# ---------------------------------------------------------------- the 12-sublayer stack
+def layer_norm(y, eps: float = LN_EPS) -> np.ndarray:
+    """Per-token LayerNorm without affine: (y - mean) / sqrt(biased variance + eps)."""
+    y = f64(y)
+    mu = y.mean(axis=1, keepdims=True)
+    var = ((y - mu) ** 2).mean(axis=1, keepdims=True)
+    return (y - mu) / np.sqrt(var + eps)
+
+
+def stack_layer(x, L: dict, a=None, bf16: bool = True) -> np.ndarray:
+    """One sublayer of the stack: CLEAR-MoE FFN or dense FFN, output stored in bf16."""
+    if L["moe"]:
+        y = ffn_forward(x, L["W1"], L["b1"], L["U"], L["S"], L["Vh"], L["residuals"],
+                        L["Wg"], L["bg"], a=a, z_bf16=bf16)
+    else:
+        y = dense_ffn(x, L["W1"], L["b1"], L["W2"], z_bf16=bf16)
+    return to_bf16(y) if bf16 else y
+
+
+def stack_next_input(y, bf16: bool = True) -> np.ndarray:
+    """x_{l+1} = LN(y_l), stored in bf16."""
+    x = layer_norm(y)
+    return to_bf16(x) if bf16 else x
