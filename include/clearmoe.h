@@ -1,0 +1,141 @@
+/*
+ * clearmoe.h -- C ABI of the GB300 (sm_103a) CLEAR-MoE FFN layer.
+ *
+ * CLEAR-MoE (arxiv 2606.28516) converts a frozen ViT FFN into a shared fc1, a shared truncated-SVD
+ * fc2 basis and per-cluster residual fc2 experts chosen by a top-1 router (Eq. 2, Algorithms 2-3):
+ *
+ *     z = GELU(W1 x + b1)                       (fc1 shared by every expert, exact-erf GELU)
+ *     a = argmax_e (W_g x + b_g)_e              (linear router, lowest index on ties)
+ *     y = U_r diag(S_r) Vh_r z + W_a^res z      (shared SVD basis + residual expert of token a)
+ *
+ * Shapes (row-major, element type "D" = the layer's dtype unless stated):
+ *   x [T x d], W1 [H x d], b1 [H], U_r [d x r], S_r [r] (always float32), Vh_r = V_r^T [r x H],
+ *   residual_e[e] [d x H] for e < E, W_g [E x d], b_g [E], W2 [d x H], out [T x d].
+ *
+ * Conventions for every call below:
+ *   - Every pointer named as a tensor is a DEVICE pointer owned by the caller, 16-byte aligned,
+ *     to a dense row-major array of the stated shape. The library never frees caller memory.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream). Calls only enqueue work and
+ *     return; they never synchronise, except clearmoe_layer_status and clearmoe_layer_destroy.
+ *   - One handle may be used by one stream at a time: its workspace holds the hidden states and
+ *     routing of the last forward.
+ *   - Arguments are validated on the host first; on any error nothing is enqueued and the
+ *     outputs are untouched. Return values are clearmoe_status codes.
+ *   - Device-side waits are bounded. A wait that runs out writes CLEARMOE_ETIMEOUT into the
+ *     handle's device status word (read by clearmoe_layer_status); the outputs of that call are
+ *     then undefined, and the handle stays usable.
+ */
+#ifndef CLEARMOE_H
+#define CLEARMOE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    CLEARMOE_OK = 0,
+    CLEARMOE_EINVAL = -1,       /* bad argument: null pointer, size out of range, misalignment */
+    CLEARMOE_EUNSUPPORTED = -2, /* valid but not tiled by this build (see clearmoe_layer_create) */
+    CLEARMOE_ECUDA = -3,        /* a CUDA runtime/driver call failed */
+    CLEARMOE_ENOMEM = -4,       /* workspace allocation failed */
+    CLEARMOE_ETIMEOUT = -5      /* a bounded device-side wait ran out */
+} clearmoe_status;
+
+typedef enum { CLEARMOE_F32 = 0, CLEARMOE_BF16 = 1 } clearmoe_dtype;
+
+/* Capacity of a layer handle. d and hidden are fixed per handle; T, E and r are per call and
+ * bounded by max_tokens, max_E and max_r. dtype selects the arithmetic:
+ *   CLEARMOE_BF16: bf16 storage, fp32 accumulation on the tcgen05 tensor cores; z, the shared-
+ *                  basis coefficients t = diag(S_r) Vh_r z and out are stored in bf16.
+ *   CLEARMOE_F32:  fp32 storage and fp32 FMA on the CUDA cores (exact-fp32 path).
+ * Tiling limits (else CLEARMOE_EUNSUPPORTED): bf16 needs d % 64 == 0, hidden % 64 == 0 and
+ * r % 16 == 0 per call; fp32 needs d % 4 == 0 and hidden % 4 == 0. max_E <= 16, max_r <= 256. */
+typedef struct {
+    int64_t max_tokens;
+    int32_t d;
+    int32_t hidden;
+    int32_t max_E;
+    int32_t max_r;
+    int32_t dtype; /* clearmoe_dtype */
+} clearmoe_layer_desc;
+
+/* Linear router (Phase 4, "Linear": d x E weights and a bias per expert): W [E x d], b [E],
+ * both device pointers in the layer's dtype. */
+typedef struct {
+    const void* W;
+    const void* b;
+} clearmoe_router;
+
+typedef struct clearmoe_layer clearmoe_layer;
+
+/* Allocates the handle and its device workspace on the current device (hidden states
+ * [max_tokens x hidden], basis coefficients [max_tokens x max_r], routing arrays, status word).
+ * Returns EINVAL for a null/invalid desc, EUNSUPPORTED per the tiling limits above, ENOMEM or
+ * ECUDA if allocation fails (nothing is leaked). */
+int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out);
+
+/* Synchronises the device, frees the workspace and the handle. NULL is accepted. */
+int clearmoe_layer_destroy(clearmoe_layer* layer);
+
+/* Routing only (Algorithm 3, steps 3-4): for every token t, a_t = the lowest e maximising
+ * the fp32 logit W_g x_t + b_g; counts_e, offsets = exclusive prefix sum of counts (E + 1
+ * entries), and perm[slot] = token with the tokens of expert e in slots
+ * [offsets_e, offsets_{e+1}) in increasing id order (a stable sort by expert). One fused
+ * kernel; results stay in the handle (read them with clearmoe_get_routing).
+ * 1 <= T <= max_tokens, 1 <= E <= max_E. */
+int clearmoe_route(clearmoe_layer* layer, const void* x, int64_t T, const clearmoe_router* router,
+                   int32_t E, void* stream);
+
+/* The CLEAR-MoE FFN forward (Eq. 2 with Algorithm 3): routes (as clearmoe_route), computes
+ * z = GELU(W1 x + b1) for every token in expert-sorted order (the gather by perm is folded into
+ * the fc1 operand loads), the shared basis through its factors, t = diag(S_r) Vh_r z, and then,
+ * per expert sub-batch, out[perm[slot]] = U_r t + residual_e[e] z (the scatter and the sum of
+ * the shared and residual terms are folded into the epilogue; each row is written once).
+ * residual_e is a HOST array of E device pointers, each to a [d x H] matrix.
+ * 1 <= T <= max_tokens, 1 <= E <= max_E, 1 <= r <= min(max_r, d, H). out [T x d] must not
+ * alias any input. */
+int clearmoe_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                         const void* b1, const void* U_r, const float* S_r, const void* Vh_r,
+                         const void* const* residual_e, const clearmoe_router* router,
+                         int32_t E, int32_t r, void* out, void* stream);
+
+/* The dense FFN the layer was converted from, on the same device: out = W2 GELU(W1 x + b1)
+ * (the comparison path; no bias on fc2, as in Eq. 2). 1 <= T <= max_tokens. */
+int clearmoe_dense_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                               const void* b1, const void* W2, void* out, void* stream);
+
+/* Per-token LayerNorm without affine between stacked sublayers: x_out = (y - mean(y)) /
+ * sqrt(var(y) + 1e-6), biased variance, fp32 statistics; y and x_out [T x d] in the layer's
+ * dtype (they may alias). 1 <= T <= max_tokens. */
+int clearmoe_layer_norm(clearmoe_layer* layer, const void* y, int64_t T, void* x_out,
+                        void* stream);
+
+/* Copies (device to device, on `stream`) the routing of the last clearmoe_route /
+ * clearmoe_ffn_forward on this handle: idx [T], counts [E], offsets [E + 1], perm [T], all
+ * int32 device pointers; any may be NULL to skip it. EINVAL if no forward has run yet. */
+int clearmoe_get_routing(clearmoe_layer* layer, int32_t* idx, int32_t* counts, int32_t* offsets,
+                         int32_t* perm, void* stream);
+
+/* Synchronises the device, returns the handle's device status word (CLEARMOE_OK or the first
+ * device-side error since the last call, e.g. CLEARMOE_ETIMEOUT) and clears it. */
+int clearmoe_layer_status(clearmoe_layer* layer);
+
+/* Fault injection for tests of the bounded waits: the grid-wide wait of the routing kernel
+ * gives up after wait_limit_ns nanoseconds (default 1e9) and, when phantom_arrivals > 0, waits
+ * for that many arrivals more than can ever come, so the wait runs out and the call reports
+ * CLEARMOE_ETIMEOUT through clearmoe_layer_status. phantom_arrivals = 0 restores normal use. */
+int clearmoe_debug_set_wait(clearmoe_layer* layer, int64_t wait_limit_ns, int32_t phantom_arrivals);
+
+/* Static string for a status code. */
+const char* clearmoe_strerror(int status);
+
+/* Library version as MAJOR * 10000 + MINOR * 100 + PATCH. */
+int clearmoe_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CLEARMOE_H */

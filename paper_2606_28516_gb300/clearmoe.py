@@ -1,0 +1,155 @@
+"""ctypes binding of libclearmoe.so, one Python function per C entry point (same names).
+
+Argument marshalling only: tensors become device pointers, torch's current stream becomes the
+cudaStream_t, non-zero status codes become ClearMoEError. Every step of the layer runs in the
+library's CUDA kernels; there is no Python or CPU fallback. The C declarations, with argument
+meaning, layout, ownership and errors, are in include/clearmoe.h.
+"""
+from __future__ import annotations
+
+import ctypes
+import pathlib
+
+_LIB_PATH = pathlib.Path(__file__).resolve().parent / "libclearmoe.so"
+_lib = None
+
+OK, EINVAL, EUNSUPPORTED, ECUDA, ENOMEM, ETIMEOUT = 0, -1, -2, -3, -4, -5
+F32, BF16 = 0, 1
+
+
+class ClearMoEError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        super().__init__(f"{where}: {clearmoe_strerror(code)} ({code})")
+        self.code = code
+
+
+class clearmoe_layer_desc(ctypes.Structure):
+    _fields_ = [("max_tokens", ctypes.c_int64), ("d", ctypes.c_int32), ("hidden", ctypes.c_int32),
+                ("max_E", ctypes.c_int32), ("max_r", ctypes.c_int32), ("dtype", ctypes.c_int32)]
+
+
+class clearmoe_router(ctypes.Structure):
+    _fields_ = [("W", ctypes.c_void_p), ("b", ctypes.c_void_p)]
+
+
+_P, _I64, _I32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+_SIGS = {
+    "clearmoe_layer_create": [ctypes.POINTER(clearmoe_layer_desc), ctypes.POINTER(ctypes.c_void_p)],
+    "clearmoe_layer_destroy": [_P],
+    "clearmoe_route": [_P, _P, _I64, ctypes.POINTER(clearmoe_router), _I32, _P],
+    "clearmoe_ffn_forward": [_P, _P, _I64, _P, _P, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
+                             ctypes.POINTER(clearmoe_router), _I32, _I32, _P, _P],
+    "clearmoe_dense_ffn_forward": [_P, _P, _I64, _P, _P, _P, _P, _P],
+    "clearmoe_layer_norm": [_P, _P, _I64, _P, _P],
+    "clearmoe_get_routing": [_P, _P, _P, _P, _P, _P],
+    "clearmoe_layer_status": [_P],
+    "clearmoe_debug_set_wait": [_P, _I64, _I32],
+    "clearmoe_strerror": [ctypes.c_int],
+    "clearmoe_version": [],
+}
+
+
+def lib() -> ctypes.CDLL:
+    """Loads libclearmoe.so (built in-tree). Raises if it is missing: there is no fallback."""
+    global _lib
+    if _lib is None:
+        if not _LIB_PATH.exists():
+            raise RuntimeError(f"{_LIB_PATH} is not built; run paper_2606_28516_gb300.build.build()")
+        try:
+            import torch  # noqa: F401  (loads the CUDA runtime the library links against)
+        except ImportError:
+            pass
+        L = ctypes.CDLL(str(_LIB_PATH))
+        for name, args in _SIGS.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = ctypes.c_char_p if name == "clearmoe_strerror" else ctypes.c_int
+        _lib = L
+    return _lib
+
+
+def _check(code: int, where: str) -> None:
+    if code != OK:
+        raise ClearMoEError(code, where)
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError("tensors passed to libclearmoe must be contiguous CUDA tensors")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def clearmoe_strerror(code: int) -> str:
+    return lib().clearmoe_strerror(code).decode()
+
+
+def clearmoe_version() -> int:
+    return lib().clearmoe_version()
+
+
+def clearmoe_layer_create(max_tokens: int, d: int, hidden: int, max_E: int, max_r: int,
+                          dtype: int) -> int:
+    desc = clearmoe_layer_desc(max_tokens, d, hidden, max_E, max_r, dtype)
+    h = ctypes.c_void_p()
+    _check(lib().clearmoe_layer_create(ctypes.byref(desc), ctypes.byref(h)), "clearmoe_layer_create")
+    return h.value
+
+
+def clearmoe_layer_destroy(layer: int) -> None:
+    _check(lib().clearmoe_layer_destroy(layer), "clearmoe_layer_destroy")
+
+
+def _router(Wg, bg) -> clearmoe_router:
+    return clearmoe_router(_ptr(Wg), _ptr(bg))
+
+
+def clearmoe_route(layer: int, x, Wg, bg, stream=None) -> None:
+    r = _router(Wg, bg)
+    _check(lib().clearmoe_route(layer, _ptr(x), x.shape[0], ctypes.byref(r), Wg.shape[0],
+                                _stream(stream)), "clearmoe_route")
+
+
+def clearmoe_ffn_forward(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, bg, out,
+                         stream=None) -> None:
+    """residual_e: a sequence of E [d x H] tensors, or one [E x d x H] tensor."""
+    E = Wg.shape[0]
+    res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
+    r = _router(Wg, bg)
+    _check(lib().clearmoe_ffn_forward(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), _ptr(U_r),
+                                      _ptr(S_r), _ptr(Vh_r), res, ctypes.byref(r), E,
+                                      S_r.shape[0], _ptr(out), _stream(stream)),
+           "clearmoe_ffn_forward")
+
+
+def clearmoe_dense_ffn_forward(layer: int, x, W1, b1, W2, out, stream=None) -> None:
+    _check(lib().clearmoe_dense_ffn_forward(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
+                                            _ptr(W2), _ptr(out), _stream(stream)),
+           "clearmoe_dense_ffn_forward")
+
+
+def clearmoe_layer_norm(layer: int, y, x_out, stream=None) -> None:
+    _check(lib().clearmoe_layer_norm(layer, _ptr(y), y.shape[0], _ptr(x_out), _stream(stream)),
+           "clearmoe_layer_norm")
+
+
+def clearmoe_get_routing(layer: int, idx=None, counts=None, offsets=None, perm=None,
+                         stream=None) -> None:
+    _check(lib().clearmoe_get_routing(layer, _ptr(idx), _ptr(counts), _ptr(offsets), _ptr(perm),
+                                      _stream(stream)), "clearmoe_get_routing")
+
+
+def clearmoe_layer_status(layer: int) -> int:
+    return lib().clearmoe_layer_status(layer)
+
+
+def clearmoe_debug_set_wait(layer: int, wait_limit_ns: int, phantom_arrivals: int) -> None:
+    _check(lib().clearmoe_debug_set_wait(layer, wait_limit_ns, phantom_arrivals),
+           "clearmoe_debug_set_wait")

@@ -1,0 +1,425 @@
+// C ABI of the CLEAR-MoE FFN layer (include/clearmoe.h): handle, workspace, argument checks, and
+// the launch sequence of each call. No compute happens here; every step runs in a kernel.
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "common.cuh"
+#include "internal.h"
+
+struct clearmoe_layer {
+    clearmoe_layer_desc desc;
+    int device;
+    int num_sms;
+    size_t esz;
+    // workspace (device)
+    void* z;            // [max_tokens x hidden]  hidden states, expert-sorted order
+    void* t;            // [max_tokens x max_r]   shared-basis coefficients
+    int32_t* idx;       // [max_tokens]
+    int32_t* perm;      // [max_tokens]
+    int32_t* counts;    // [CM_MAX_E]
+    int32_t* offsets;   // [CM_MAX_E + 1]
+    int32_t* cta_counts;  // [route_max_ctas x CM_MAX_E]
+    unsigned long long* barrier;
+    int32_t* status;
+    unsigned long long barrier_total;
+    int64_t wait_limit_ns;
+    int32_t phantom;
+    int64_t last_T;
+    int32_t last_E;
+};
+
+namespace {
+
+using cm::encode_tmap_bf16;
+
+inline bool misaligned(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
+
+int cuda_fail(cudaError_t e) {
+    if (e == cudaSuccess) return CLEARMOE_OK;
+    (void)cudaGetLastError();
+    return CLEARMOE_ECUDA;
+}
+
+void free_ws(clearmoe_layer* L) {
+    void* ptrs[] = {L->z, L->t, L->idx, L->perm, L->counts, L->offsets, L->cta_counts, L->barrier, L->status};
+    for (void* p : ptrs)
+        if (p) cudaFree(p);
+}
+
+int check_common(const clearmoe_layer* L, const void* x, int64_t T) {
+    if (!L || !x) return CLEARMOE_EINVAL;
+    if (T < 1 || T > L->desc.max_tokens) return CLEARMOE_EINVAL;
+    if (misaligned(x)) return CLEARMOE_EINVAL;
+    return CLEARMOE_OK;
+}
+
+int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router, int E,
+             cudaStream_t s) {
+    int grid = 0, chunk = 0;
+    if (cm::route_grid(T, L->desc.d, E, L->desc.dtype, L->num_sms, &grid, &chunk) != 0)
+        return CLEARMOE_ECUDA;
+    if (grid > cm::route_max_ctas(L->num_sms, L->desc.dtype, L->desc.d, E)) return CLEARMOE_EUNSUPPORTED;
+    cm::RouteArgs a;
+    a.x = x;
+    a.T = T;
+    a.d = L->desc.d;
+    a.E = E;
+    a.dtype = L->desc.dtype;
+    a.Wg = router->W;
+    a.bg = router->b;
+    a.idx = L->idx;
+    a.perm = L->perm;
+    a.counts = L->counts;
+    a.offsets = L->offsets;
+    a.cta_counts = L->cta_counts;
+    a.barrier = L->barrier;
+    a.target = L->barrier_total + (unsigned long long)grid + (unsigned long long)L->phantom;
+    a.wait_limit_ns = L->wait_limit_ns;
+    a.status = L->status;
+    const int rc = cuda_fail(cm::launch_route(a, grid, chunk, s));
+    if (rc == CLEARMOE_OK) {
+        L->barrier_total += (unsigned long long)grid;
+        L->last_T = T;
+        L->last_E = E;
+    }
+    return rc;
+}
+
+int check_router(const clearmoe_layer* L, const clearmoe_router* router, int E) {
+    if (!router || !router->W || !router->b) return CLEARMOE_EINVAL;
+    if (misaligned(router->W)) return CLEARMOE_EINVAL;
+    if (E < 1 || E > L->desc.max_E) return CLEARMOE_EINVAL;
+    return CLEARMOE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* clearmoe_strerror(int status) {
+    switch (status) {
+        case CLEARMOE_OK: return "ok";
+        case CLEARMOE_EINVAL: return "invalid argument";
+        case CLEARMOE_EUNSUPPORTED: return "shape not supported by this build";
+        case CLEARMOE_ECUDA: return "CUDA error";
+        case CLEARMOE_ENOMEM: return "out of device memory";
+        case CLEARMOE_ETIMEOUT: return "a bounded device-side wait timed out";
+        default: return "unknown status";
+    }
+}
+
+int clearmoe_version(void) { return 100; }
+
+int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out) {
+    if (!desc || !out) return CLEARMOE_EINVAL;
+    *out = nullptr;
+    const clearmoe_layer_desc& D = *desc;
+    if (D.max_tokens < 1 || D.d < 1 || D.hidden < 1 || D.max_E < 1 || D.max_r < 1) return CLEARMOE_EINVAL;
+    if (D.dtype != CLEARMOE_F32 && D.dtype != CLEARMOE_BF16) return CLEARMOE_EINVAL;
+    if (D.max_E > CM_MAX_E || D.max_r > CM_MAX_R) return CLEARMOE_EUNSUPPORTED;
+    if (D.max_tokens > (int64_t)1 << 30) return CLEARMOE_EUNSUPPORTED;
+    if (D.dtype == CLEARMOE_BF16) {
+        if (D.d % 64 || D.hidden % 64 || D.d > 1024) return CLEARMOE_EUNSUPPORTED;
+    } else {
+        if (D.d % 4 || D.hidden % 4 || D.d > 512) return CLEARMOE_EUNSUPPORTED;
+    }
+    clearmoe_layer* L = new (std::nothrow) clearmoe_layer();
+    if (!L) return CLEARMOE_ENOMEM;
+    std::memset(L, 0, sizeof(*L));
+    L->desc = D;
+    L->esz = D.dtype == CLEARMOE_BF16 ? 2 : 4;
+    L->wait_limit_ns = 1000000000LL;
+    if (cudaGetDevice(&L->device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device) != cudaSuccess) {
+        delete L;
+        (void)cudaGetLastError();
+        return CLEARMOE_ECUDA;
+    }
+    const size_t T = (size_t)D.max_tokens;
+    const size_t ncta = (size_t)cm::route_max_ctas(L->num_sms, D.dtype, D.d, D.max_E);
+    bool ok = cudaMalloc(&L->z, T * D.hidden * L->esz) == cudaSuccess &&
+              cudaMalloc(&L->t, T * D.max_r * L->esz) == cudaSuccess &&
+              cudaMalloc((void**)&L->idx, T * 4) == cudaSuccess &&
+              cudaMalloc((void**)&L->perm, T * 4) == cudaSuccess &&
+              cudaMalloc((void**)&L->counts, CM_MAX_E * 4) == cudaSuccess &&
+              cudaMalloc((void**)&L->offsets, (CM_MAX_E + 1) * 4) == cudaSuccess &&
+              cudaMalloc((void**)&L->cta_counts, ncta * CM_MAX_E * 4) == cudaSuccess &&
+              cudaMalloc((void**)&L->barrier, 8) == cudaSuccess &&
+              cudaMalloc((void**)&L->status, 4) == cudaSuccess;
+    if (ok) {
+        ok = cudaMemset(L->barrier, 0, 8) == cudaSuccess && cudaMemset(L->status, 0, 4) == cudaSuccess &&
+             cudaDeviceSynchronize() == cudaSuccess;
+    }
+    if (!ok) {
+        const cudaError_t e = cudaGetLastError();
+        free_ws(L);
+        delete L;
+        return e == cudaErrorMemoryAllocation ? CLEARMOE_ENOMEM : CLEARMOE_ECUDA;
+    }
+    *out = L;
+    return CLEARMOE_OK;
+}
+
+int clearmoe_layer_destroy(clearmoe_layer* L) {
+    if (!L) return CLEARMOE_OK;
+    const cudaError_t e = cudaDeviceSynchronize();
+    free_ws(L);
+    delete L;
+    return cuda_fail(e);
+}
+
+int clearmoe_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router, int32_t E,
+                   void* stream) {
+    int rc = check_common(L, x, T);
+    if (rc) return rc;
+    if ((rc = check_router(L, router, E))) return rc;
+    return do_route(L, x, T, router, E, static_cast<cudaStream_t>(stream));
+}
+
+int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                         const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
+                         const clearmoe_router* router, int32_t E, int32_t r, void* out, void* stream) {
+    int rc = check_common(L, x, T);
+    if (rc) return rc;
+    if ((rc = check_router(L, router, E))) return rc;
+    if (!W1 || !b1 || !U_r || !S_r || !Vh_r || !residual_e || !out) return CLEARMOE_EINVAL;
+    const int d = L->desc.d, H = L->desc.hidden;
+    if (r < 1 || r > L->desc.max_r || r > d || r > H) return CLEARMOE_EINVAL;
+    for (int e = 0; e < E; ++e)
+        if (!residual_e[e] || misaligned(residual_e[e])) return CLEARMOE_EINVAL;
+    if (misaligned(W1) || misaligned(b1) || misaligned(U_r) || misaligned(S_r) || misaligned(Vh_r) ||
+        misaligned(out))
+        return CLEARMOE_EINVAL;
+    const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
+    if (bf16 && r % 16) return CLEARMOE_EUNSUPPORTED;
+    if (!bf16 && r % 4) return CLEARMOE_EUNSUPPORTED;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+    if ((rc = do_route(L, x, T, router, E, s))) return rc;
+
+    if (!bf16) {
+        cm::SimtGemmArgs g;
+        std::memset(&g, 0, sizeof(g));
+        // fc1 + bias + GELU on tokens gathered in expert order
+        g.A0 = static_cast<const float*>(x);
+        g.lda0 = d;
+        g.K0 = d;
+        g.B0 = static_cast<const float*>(W1);
+        g.a_rows = L->perm;
+        g.M = T;
+        g.N = H;
+        g.bias = static_cast<const float*>(b1);
+        g.gelu = 1;
+        g.C = static_cast<float*>(L->z);
+        g.ldc = H;
+        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        // t = diag(S_r) Vh_r z
+        std::memset(&g, 0, sizeof(g));
+        g.A0 = static_cast<const float*>(L->z);
+        g.lda0 = H;
+        g.K0 = H;
+        g.B0 = static_cast<const float*>(Vh_r);
+        g.M = T;
+        g.N = r;
+        g.scale = S_r;
+        g.C = static_cast<float*>(L->t);
+        g.ldc = r;
+        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        // out[perm[slot]] = U_r t + W_e^res z per expert sub-batch
+        std::memset(&g, 0, sizeof(g));
+        g.A0 = static_cast<const float*>(L->t);
+        g.lda0 = r;
+        g.K0 = r;
+        g.B0 = static_cast<const float*>(U_r);
+        g.A1 = static_cast<const float*>(L->z);
+        g.lda1 = H;
+        g.K1 = H;
+        for (int e = 0; e < E; ++e) g.B1[e] = static_cast<const float*>(residual_e[e]);
+        g.M = T;
+        g.N = d;
+        g.C = static_cast<float*>(out);
+        g.ldc = d;
+        g.c_rows = L->perm;
+        g.offsets = L->offsets;
+        g.E = E;
+        return cuda_fail(cm::launch_simt_gemm(g, s));
+    }
+
+    // ---- bf16: tcgen05 GEMMs
+    const int bn1 = cm::tc_pick_bn(cm::TC_GATHER, H);
+    const int bn2 = cm::tc_pick_bn(cm::TC_DENSE, r);
+    const int bn3 = cm::tc_pick_bn(cm::TC_GROUPED, d);
+    if (!bn1 || !bn2 || !bn3) return CLEARMOE_EUNSUPPORTED;
+    cm::TcGemmArgs g;
+    std::memset(&g, 0, sizeof(g));
+    g.status = L->status;
+    g.wait_limit_ns = L->wait_limit_ns;
+    // fc1 + b1 + GELU, A rows gathered by perm
+    if (encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
+    g.mode = cm::TC_GATHER;
+    g.epi = cm::TC_EPI_BIAS_GELU;
+    g.M = T;
+    g.N = H;
+    g.K0 = d;
+    g.gather_src = x;
+    g.gather_ld = d;
+    g.rows = L->perm;
+    g.bias = b1;
+    g.C = L->z;
+    g.ldc = H;
+    if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
+    // t = diag(S_r) Vh_r z
+    cm::TcGemmArgs g2;
+    std::memset(&g2, 0, sizeof(g2));
+    g2.status = L->status;
+    g2.wait_limit_ns = L->wait_limit_ns;
+    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, Vh_r, r, H, bn2))
+        return CLEARMOE_ECUDA;
+    g2.mode = cm::TC_DENSE;
+    g2.epi = cm::TC_EPI_SCALE;
+    g2.M = T;
+    g2.N = r;
+    g2.K0 = H;
+    g2.scale = S_r;
+    g2.C = L->t;
+    g2.ldc = r;
+    if ((rc = cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s)))) return rc;
+    // out[perm[slot]] = [t | z] [U_r | W_e^res]^T per expert sub-batch
+    cm::TcGemmArgs g3;
+    std::memset(&g3, 0, sizeof(g3));
+    g3.status = L->status;
+    g3.wait_limit_ns = L->wait_limit_ns;
+    if (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, bn3) ||
+        encode_tmap_bf16(&g3.tmA1, L->z, T, H, 128))
+        return CLEARMOE_ECUDA;
+    for (int e = 0; e < E; ++e)
+        if (encode_tmap_bf16(&g3.tmB1[e], residual_e[e], d, H, bn3)) return CLEARMOE_ECUDA;
+    g3.mode = cm::TC_GROUPED;
+    g3.epi = cm::TC_EPI_SCATTER;
+    g3.M = T;
+    g3.N = d;
+    g3.K0 = r;
+    g3.K1 = H;
+    g3.offsets = L->offsets;
+    g3.E = E;
+    g3.rows = L->perm;
+    g3.C = out;
+    g3.ldc = d;
+    return cuda_fail(cm::launch_tc_gemm(g3, L->num_sms, s));
+}
+
+int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                               const void* W2, void* out, void* stream) {
+    int rc = check_common(L, x, T);
+    if (rc) return rc;
+    if (!W1 || !b1 || !W2 || !out) return CLEARMOE_EINVAL;
+    if (misaligned(W1) || misaligned(b1) || misaligned(W2) || misaligned(out)) return CLEARMOE_EINVAL;
+    const int d = L->desc.d, H = L->desc.hidden;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (L->desc.dtype == CLEARMOE_F32) {
+        cm::SimtGemmArgs g;
+        std::memset(&g, 0, sizeof(g));
+        g.A0 = static_cast<const float*>(x);
+        g.lda0 = d;
+        g.K0 = d;
+        g.B0 = static_cast<const float*>(W1);
+        g.M = T;
+        g.N = H;
+        g.bias = static_cast<const float*>(b1);
+        g.gelu = 1;
+        g.C = static_cast<float*>(L->z);
+        g.ldc = H;
+        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        std::memset(&g, 0, sizeof(g));
+        g.A0 = static_cast<const float*>(L->z);
+        g.lda0 = H;
+        g.K0 = H;
+        g.B0 = static_cast<const float*>(W2);
+        g.M = T;
+        g.N = d;
+        g.C = static_cast<float*>(out);
+        g.ldc = d;
+        return cuda_fail(cm::launch_simt_gemm(g, s));
+    }
+    const int bn1 = cm::tc_pick_bn(cm::TC_DENSE, H);
+    const int bn2 = cm::tc_pick_bn(cm::TC_DENSE, d);
+    cm::TcGemmArgs g;
+    std::memset(&g, 0, sizeof(g));
+    g.status = L->status;
+    g.wait_limit_ns = L->wait_limit_ns;
+    if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
+    g.mode = cm::TC_DENSE;
+    g.epi = cm::TC_EPI_BIAS_GELU;
+    g.M = T;
+    g.N = H;
+    g.K0 = d;
+    g.bias = b1;
+    g.C = L->z;
+    g.ldc = H;
+    if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
+    cm::TcGemmArgs g2;
+    std::memset(&g2, 0, sizeof(g2));
+    g2.status = L->status;
+    g2.wait_limit_ns = L->wait_limit_ns;
+    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, W2, d, H, bn2))
+        return CLEARMOE_ECUDA;
+    g2.mode = cm::TC_DENSE;
+    g2.epi = cm::TC_EPI_STORE;
+    g2.M = T;
+    g2.N = d;
+    g2.K0 = H;
+    g2.C = out;
+    g2.ldc = d;
+    return cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s));
+}
+
+int clearmoe_layer_norm(clearmoe_layer* L, const void* y, int64_t T, void* x_out, void* stream) {
+    int rc = check_common(L, y, T);
+    if (rc) return rc;
+    if (!x_out || misaligned(x_out)) return CLEARMOE_EINVAL;
+    return cuda_fail(cm::launch_layer_norm(y, x_out, T, L->desc.d, L->desc.dtype, static_cast<cudaStream_t>(stream)));
+}
+
+int clearmoe_get_routing(clearmoe_layer* L, int32_t* idx, int32_t* counts, int32_t* offsets, int32_t* perm,
+                         void* stream) {
+    if (!L) return CLEARMOE_EINVAL;
+    if (L->last_T < 1) return CLEARMOE_EINVAL;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t T = (size_t)L->last_T, E = (size_t)L->last_E;
+    cudaError_t e = cudaSuccess;
+    if (idx && e == cudaSuccess) e = cudaMemcpyAsync(idx, L->idx, T * 4, cudaMemcpyDeviceToDevice, s);
+    if (counts && e == cudaSuccess) e = cudaMemcpyAsync(counts, L->counts, E * 4, cudaMemcpyDeviceToDevice, s);
+    if (offsets && e == cudaSuccess) e = cudaMemcpyAsync(offsets, L->offsets, (E + 1) * 4, cudaMemcpyDeviceToDevice, s);
+    if (perm && e == cudaSuccess) e = cudaMemcpyAsync(perm, L->perm, T * 4, cudaMemcpyDeviceToDevice, s);
+    return cuda_fail(e);
+}
+
+int clearmoe_layer_status(clearmoe_layer* L) {
+    if (!L) return CLEARMOE_EINVAL;
+    if (cudaDeviceSynchronize() != cudaSuccess) {
+        (void)cudaGetLastError();
+        return CLEARMOE_ECUDA;
+    }
+    int32_t st = 0;
+    if (cudaMemcpy(&st, L->status, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return CLEARMOE_ECUDA;
+    if (st != 0) {
+        if (cudaMemset(L->status, 0, 4) != cudaSuccess) return CLEARMOE_ECUDA;
+        if (st == CLEARMOE_ETIMEOUT) {
+            // arrivals of a launch that gave up no longer match the host's count: start afresh
+            if (cudaMemset(L->barrier, 0, 8) != cudaSuccess) return CLEARMOE_ECUDA;
+            L->barrier_total = 0;
+        }
+        if (cudaDeviceSynchronize() != cudaSuccess) return CLEARMOE_ECUDA;
+    }
+    return st;
+}
+
+int clearmoe_debug_set_wait(clearmoe_layer* L, int64_t wait_limit_ns, int32_t phantom_arrivals) {
+    if (!L || wait_limit_ns < 1000 || phantom_arrivals < 0) return CLEARMOE_EINVAL;
+    L->wait_limit_ns = wait_limit_ns;
+    L->phantom = phantom_arrivals;
+    return CLEARMOE_OK;
+}
+
+}  // extern "C"

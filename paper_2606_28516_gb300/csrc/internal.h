@@ -1,0 +1,93 @@
+// Host-side launchers shared between the translation units of the library (not part of the ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace cm {
+
+struct RouteArgs {
+    const void* x;
+    int64_t T;
+    int d;
+    int E;
+    int dtype;  // clearmoe_dtype
+    const void* Wg;
+    const void* bg;
+    int32_t* idx;
+    int32_t* perm;
+    int32_t* counts;
+    int32_t* offsets;
+    int32_t* cta_counts;           // [max_route_ctas x CM_MAX_E] scratch
+    unsigned long long* barrier;   // monotone arrival counter
+    unsigned long long target;     // counter value that releases this launch
+    int64_t wait_limit_ns;
+    int32_t* status;
+};
+
+// Grid of the routing kernel for T tokens (co-resident CTAs); chunk = rows per CTA.
+int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* chunk);
+int route_max_ctas(int num_sms, int dtype, int d, int E);
+cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s);
+
+// ---- exact-fp32 SIMT GEMMs (fp32 layer) ----
+struct SimtGemmArgs {
+    // C[m, n] = epi(sum_k A0[rowA(m), k] B0[n, k] + sum_k A1[m, k] B1_e[n, k])
+    const float* A0;
+    int64_t lda0;
+    int K0;
+    const float* B0;
+    const int32_t* a_rows;  // gather rows of A0 (nullable)
+    const float* A1;
+    int64_t lda1;
+    int K1;
+    const float* B1[16];     // grouped: per-expert B of the second segment; else B1[0]
+    int64_t M;
+    int N;
+    const float* bias;   // + bias[n]
+    int gelu;            // GELU after bias
+    const float* scale;  // * scale[n]
+    float* C;
+    int64_t ldc;
+    const int32_t* c_rows;   // scatter rows of C (nullable)
+    const int32_t* offsets;  // grouped: expert boundaries [E + 1] (nullable = not grouped)
+    int E;
+};
+cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s);
+
+cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s);
+
+// ---- tcgen05 bf16 GEMMs ----
+enum TcEpi { TC_EPI_BIAS_GELU = 0, TC_EPI_SCALE = 1, TC_EPI_STORE = 2, TC_EPI_SCATTER = 3 };
+enum TcMode { TC_DENSE = 0, TC_GATHER = 1, TC_GROUPED = 2 };
+
+struct TcGemmArgs {
+    int mode;  // TcMode
+    int epi;   // TcEpi
+    int64_t M;
+    int N;
+    int K0;
+    int K1;  // second K segment (grouped only)
+    CUtensorMap tmA0, tmA1, tmB0;
+    CUtensorMap tmB1[16];
+    const void* gather_src;    // gather: rows of A0 read directly (bf16 [.. x K0])
+    int64_t gather_ld;         // elements
+    const int32_t* rows;       // gather: A row of output row m; scatter: output row of slot m
+    const int32_t* offsets;    // grouped: [E + 1]
+    int E;
+    const void* bias;          // bf16 [N]
+    const float* scale;        // fp32 [N]
+    void* C;                   // bf16
+    int64_t ldc;
+    int32_t* status;
+    int64_t wait_limit_ns;
+};
+int tc_pick_bn(int mode, int N);
+cudaError_t launch_tc_gemm(const TcGemmArgs& a, int num_sms, cudaStream_t s);
+
+// Encode a 2-D bf16 row-major [rows x cols] tensor map, box {64, box_rows}, 128-byte swizzle.
+int encode_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols,
+                     int box_rows);
+
+}  // namespace cm

@@ -1,0 +1,343 @@
+// Fused routing kernel of the CLEAR-MoE FFN (Algorithm 3, steps 3-4):
+//   logits = W_g x + b_g (linear router), a = argmax (lowest index on ties),
+//   per-expert histogram, exclusive prefix sum, and the stable permutation perm[slot] = token.
+//
+// One cooperative launch of co-resident CTAs; CTA b owns a contiguous range of `chunk` tokens.
+//   phase 1: stream x once from HBM, router logits and argmax per token, local histogram;
+//   grid-wide wait (bounded, on a monotone arrival counter);
+//   phase 2: each CTA sums the histograms of the CTAs before it and writes its tokens' slots in
+//            token order (ranks from warp match masks), which makes the sort stable.
+// bf16 tokens: the d x E contraction runs on the legacy warp MMA (m16n8k16, fp32 accumulate)
+// straight from registers: the 16-byte loads of x are coalesced, and the K order of each
+// fragment is permuted identically for x and W_g, which leaves every dot product unchanged.
+// fp32 tokens: fp32 FMA on the CUDA cores (an fp32 router decision needs fp32 products).
+#include "common.cuh"
+#include "internal.h"
+
+namespace cm {
+
+constexpr int RT_THREADS = 256;
+constexpr int RT_WARPS = RT_THREADS / 32;
+
+__device__ __forceinline__ uint4 ldg_nc_v4(const uint4* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1,
+                                               uint32_t a2, uint32_t a3, uint32_t b0,
+                                               uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+        "{%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// better (value, index) with the lower index winning exact ties
+__device__ __forceinline__ void arg_better(float& bv, int& be, float v, int e) {
+    if (v > bv || (v == bv && e < be)) {
+        bv = v;
+        be = e;
+    }
+}
+
+__host__ __device__ inline size_t frag_bytes(int dtype, int d, int E) {
+    if (dtype == CLEARMOE_BF16) return (size_t)((E + 7) / 8) * (d / 32) * 32 * 16;
+    return (size_t)E * d * 4;
+}
+static size_t route_smem(int dtype, int d, int E, int chunk) {
+    return ((frag_bytes(dtype, d, E) + 15) & ~(size_t)15) + (size_t)((chunk + 15) & ~15);
+}
+
+template <bool BF16>
+__global__ void __launch_bounds__(RT_THREADS) route_kernel(const RouteArgs a, const int chunk) {
+    extern __shared__ __align__(16) unsigned char smem[];
+    __shared__ int s_count[CM_MAX_E];
+    __shared__ int s_base[CM_MAX_E];
+    __shared__ int s_tot[CM_MAX_E];
+    __shared__ int s_run[CM_MAX_E];
+    __shared__ int s_wc[RT_WARPS][CM_MAX_E];
+    __shared__ int s_abort;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int E = a.E, d = a.d;
+    const int64_t row0 = (int64_t)blockIdx.x * chunk;
+    const int nrows = (int)max((int64_t)0, min((int64_t)chunk, a.T - row0));
+    const int nchunk = d / 32;
+    const int NT = (E + 7) / 8;
+    uint8_t* sidx = smem + ((frag_bytes(BF16 ? CLEARMOE_BF16 : CLEARMOE_F32, d, E) + 15) & ~15);
+
+    if (tid < CM_MAX_E) s_count[tid] = 0;
+    if (tid == 0) s_abort = 0;
+
+    // ---------------- phase 1: router logits + argmax for this CTA's rows
+    if constexpr (BF16) {
+        // B fragments of W_g: [n-tile][32-column chunk][lane] -> 8 consecutive bf16 of row
+        // nt*8 + lane/4, columns chunk*32 + (lane%4)*8.
+        uint4* bfrag = reinterpret_cast<uint4*>(smem);
+        const uint16_t* W = static_cast<const uint16_t*>(a.Wg);
+        for (int i = tid; i < NT * nchunk * 32; i += RT_THREADS) {
+            const int l = i & 31, c = (i >> 5) % nchunk, nt = (i >> 5) / nchunk;
+            const int e = nt * 8 + (l >> 2);
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (e < E) v = *reinterpret_cast<const uint4*>(W + (size_t)e * d + c * 32 + (l & 3) * 8);
+            bfrag[i] = v;
+        }
+        __syncthreads();
+        const uint16_t* bgp = static_cast<const uint16_t*>(a.bg);
+        const int g = lane >> 2, tig = lane & 3;
+        const int ngroups = (nrows + 15) / 16;
+        const uint4 zero = make_uint4(0, 0, 0, 0);
+        for (int grp = warp; grp < ngroups; grp += RT_WARPS) {
+            const int iA = grp * 16 + g, iB = iA + 8;
+            const bool vA = iA < nrows, vB = iB < nrows;
+            const uint4* pA = reinterpret_cast<const uint4*>(
+                                  static_cast<const uint16_t*>(a.x) + (row0 + (vA ? iA : 0)) * d) + tig;
+            const uint4* pB = reinterpret_cast<const uint4*>(
+                                  static_cast<const uint16_t*>(a.x) + (row0 + (vB ? iB : 0)) * d) + tig;
+            float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+            for (int c0 = 0; c0 < nchunk; c0 += 8) {
+                uint4 xa[8], xb[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int c = c0 + i;
+                    xa[i] = (vA && c < nchunk) ? ldg_nc_v4(pA + 4 * c) : zero;
+                    xb[i] = (vB && c < nchunk) ? ldg_nc_v4(pB + 4 * c) : zero;
+                }
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int c = c0 + i;
+                    if (c < nchunk) {
+#pragma unroll
+                        for (int nt = 0; nt < 2; ++nt) {
+                            if (nt < NT) {
+                                const uint4 w = bfrag[(nt * nchunk + c) * 32 + lane];
+                                mma_bf16_16816(acc[nt], xa[i].x, xb[i].x, xa[i].y, xb[i].y, w.x, w.y);
+                                mma_bf16_16816(acc[nt], xa[i].z, xb[i].z, xa[i].w, xb[i].w, w.z, w.w);
+                            }
+                        }
+                    }
+                }
+            }
+            // D fragment: acc[nt][0..1] = row g, experts nt*8 + 2*tig + {0,1}; [2..3] = row g+8
+            float bA = -INFINITY, bB = -INFINITY;
+            int eA = 0x7fffffff, eB = 0x7fffffff;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+#pragma unroll
+                for (int j = 0; j < 2; ++j) {
+                    const int e = nt * 8 + 2 * tig + j;
+                    if (nt < NT && e < E) {
+                        const uint16_t bb = bgp[e];
+                        const float bias = __uint_as_float((uint32_t)bb << 16);
+                        arg_better(bA, eA, acc[nt][j] + bias, e);
+                        arg_better(bB, eB, acc[nt][2 + j] + bias, e);
+                    }
+                }
+            }
+#pragma unroll
+            for (int off = 1; off <= 2; off <<= 1) {
+                const float ovA = __shfl_xor_sync(0xffffffffu, bA, off);
+                const int oeA = __shfl_xor_sync(0xffffffffu, eA, off);
+                const float ovB = __shfl_xor_sync(0xffffffffu, bB, off);
+                const int oeB = __shfl_xor_sync(0xffffffffu, eB, off);
+                arg_better(bA, eA, ovA, oeA);
+                arg_better(bB, eB, ovB, oeB);
+            }
+            if (eA > E - 1) eA = 0;  // only reachable with non-finite logits
+            if (eB > E - 1) eB = 0;
+            if (tig == 0) {
+                if (vA) {
+                    a.idx[row0 + iA] = eA;
+                    sidx[iA] = (uint8_t)eA;
+                }
+                if (vB) {
+                    a.idx[row0 + iB] = eB;
+                    sidx[iB] = (uint8_t)eB;
+                }
+            }
+        }
+    } else {
+        float* Wf = reinterpret_cast<float*>(smem);
+        const float* W = static_cast<const float*>(a.Wg);
+        for (int i = tid; i < E * d; i += RT_THREADS) Wf[i] = W[i];
+        __syncthreads();
+        const float* bgp = static_cast<const float*>(a.bg);
+        const float* X = static_cast<const float*>(a.x);
+        for (int i = warp; i < nrows; i += RT_WARPS) {
+            const float* xr = X + (row0 + i) * d;
+            float acc[CM_MAX_E];
+#pragma unroll
+            for (int e = 0; e < CM_MAX_E; ++e) acc[e] = 0.f;
+            for (int k = lane; k < d; k += 32) {
+                const float xv = xr[k];
+#pragma unroll
+                for (int e = 0; e < CM_MAX_E; ++e)
+                    if (e < E) acc[e] = fmaf(xv, Wf[e * d + k], acc[e]);
+            }
+            float bv = -INFINITY;
+            int be = 0x7fffffff;
+#pragma unroll
+            for (int e = 0; e < CM_MAX_E; ++e) {
+                if (e < E) {
+                    float v = acc[e];
+#pragma unroll
+                    for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+                    arg_better(bv, be, v + bgp[e], e);
+                }
+            }
+            if (be > E - 1) be = 0;
+            if (lane == 0) {
+                a.idx[row0 + i] = be;
+                sidx[i] = (uint8_t)be;
+            }
+        }
+    }
+    __syncthreads();
+
+    // ---------------- local histogram, published for the other CTAs
+    for (int i = tid; i < nrows; i += RT_THREADS) atomicAdd(&s_count[sidx[i]], 1);
+    __syncthreads();
+    if (tid < E) a.cta_counts[(size_t)blockIdx.x * CM_MAX_E + tid] = s_count[tid];
+    __threadfence();
+    __syncthreads();
+
+    // ---------------- grid-wide wait (bounded)
+    if (tid == 0) {
+        atomicAdd(a.barrier, 1ULL);
+        const uint64_t t0 = globaltimer();
+        while (ld_acquire_u64(a.barrier) < a.target) {
+            if (globaltimer() - t0 > (uint64_t)a.wait_limit_ns) {
+                s_abort = 1;
+                set_status(a.status, CLEARMOE_ETIMEOUT);
+                break;
+            }
+            __nanosleep(64);
+        }
+    }
+    __syncthreads();
+    if (s_abort) return;
+
+    // ---------------- phase 2: global offsets, then this CTA's slots in token order
+    for (int e = warp; e < E; e += RT_WARPS) {
+        int before = 0, total = 0;
+        for (int b = lane; b < (int)gridDim.x; b += 32) {
+            const int c = __ldcg(&a.cta_counts[(size_t)b * CM_MAX_E + e]);
+            total += c;
+            if (b < (int)blockIdx.x) before += c;
+        }
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) {
+            before += __shfl_xor_sync(0xffffffffu, before, off);
+            total += __shfl_xor_sync(0xffffffffu, total, off);
+        }
+        if (lane == 0) {
+            s_base[e] = before;
+            s_tot[e] = total;
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        int run = 0;
+        for (int e = 0; e < E; ++e) {
+            const int t = s_tot[e];
+            s_base[e] += run;
+            if (blockIdx.x == 0) {
+                a.counts[e] = t;
+                a.offsets[e] = run;
+            }
+            run += t;
+            s_run[e] = 0;
+        }
+        if (blockIdx.x == 0) a.offsets[E] = run;
+    }
+    const unsigned lt = (1u << lane) - 1u;
+    for (int i0 = 0; i0 < nrows; i0 += RT_THREADS) {
+        if (tid < RT_WARPS * CM_MAX_E) (&s_wc[0][0])[tid] = 0;
+        __syncthreads();
+        const int i = i0 + tid;
+        const bool valid = i < nrows;
+        const int e = valid ? (int)sidx[i] : CM_MAX_E + 1;
+        const unsigned same = __match_any_sync(0xffffffffu, e);
+        const int rank = __popc(same & lt);
+        if (valid && rank == 0) s_wc[warp][e] = __popc(same);
+        __syncthreads();
+        if (tid < E) {
+            int run = s_run[tid];
+            for (int w = 0; w < RT_WARPS; ++w) {
+                const int c = s_wc[w][tid];
+                s_wc[w][tid] = run;
+                run += c;
+            }
+            s_run[tid] = run;
+        }
+        __syncthreads();
+        if (valid) a.perm[s_base[e] + s_wc[warp][e] + rank] = (int32_t)(row0 + i);
+        __syncthreads();
+    }
+}
+
+int route_max_ctas(int num_sms, int, int, int) { return num_sms * 8; }
+
+int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* chunk) {
+    const bool bf16 = dtype == CLEARMOE_BF16;
+    int occ = 0;
+    int64_t want = (int64_t)num_sms * 2;
+    int64_t ch = ((T + want - 1) / want + 15) / 16 * 16;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaFuncSetAttribute((const void*)route_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+        cudaFuncSetAttribute((const void*)route_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+        attr_set = true;
+    }
+    for (int iter = 0; iter < 4; ++iter) {
+        const size_t smem = route_smem(dtype, d, E, (int)ch);
+        cudaError_t err = cudaOccupancyMaxActiveBlocksPerMultiprocessorWithFlags(
+            &occ, bf16 ? (const void*)route_kernel<true> : (const void*)route_kernel<false>,
+            RT_THREADS, smem, cudaOccupancyDefault);
+        if (err != cudaSuccess) return -1;
+        if (occ <= 0) return -2;
+        const int64_t maxg = (int64_t)occ * num_sms;
+        if (want <= maxg) break;
+        want = maxg;
+        ch = ((T + want - 1) / want + 15) / 16 * 16;
+    }
+    if (ch < 16) ch = 16;
+    *chunk = (int)ch;
+    *grid = (int)((T + ch - 1) / ch);
+    return 0;
+}
+
+cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s) {
+    const bool bf16 = a.dtype == CLEARMOE_BF16;
+    const size_t smem = route_smem(a.dtype, a.d, a.E, chunk);
+    const void* fn = bf16 ? (const void*)route_kernel<true> : (const void*)route_kernel<false>;
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(RT_THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (bf16) return cudaLaunchKernelEx(&cfg, route_kernel<true>, a, chunk);
+    return cudaLaunchKernelEx(&cfg, route_kernel<false>, a, chunk);
+}
+
+}  // namespace cm

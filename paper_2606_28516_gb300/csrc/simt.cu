@@ -1,0 +1,204 @@
+// Exact-fp32 path of the CLEAR-MoE FFN (fp32 layers) and the LayerNorm between stacked sublayers.
+//
+// fp32 layers keep fp32 products: TF32 tensor cores round each operand to 10 mantissa bits
+// (relative error ~5e-4 per product), more than the fp32 path's 1e-4 budget, so these GEMMs run
+// on the CUDA cores. One tiled kernel covers every product of the layer:
+//   C[m, n] = epi( sum_k A0[rowA(m), k] B0[n, k]  +  sum_k A1[m, k] B1_e[n, k] )
+// with an optional row gather of A0 (fc1 on tokens in expert order), an optional second K
+// segment with a per-expert B (the grouped residual GEMM, Algorithm 3 step 5), an epilogue of
+// bias, GELU and per-column scale, and an optional row scatter of C (the unshuffle, step 6).
+#include "common.cuh"
+#include "internal.h"
+
+namespace cm {
+
+constexpr int SG_M = 64, SG_N = 64, SG_K = 16;
+
+__global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, const int n_tiles_n) {
+    __shared__ float As[SG_K][SG_M + 4];
+    __shared__ float Bs[SG_K][SG_N + 4];
+    const int tid = threadIdx.x;
+    const int nt = blockIdx.x % n_tiles_n;
+    const int mt = blockIdx.x / n_tiles_n;
+    int64_t m_lo, m_hi;
+    int e = 0;
+    if (a.offsets) {
+        int acc = 0;
+        bool found = false;
+        for (e = 0; e < a.E; ++e) {
+            const int lo = a.offsets[e], hi = a.offsets[e + 1];
+            const int tiles = (hi - lo + SG_M - 1) / SG_M;
+            if (mt < acc + tiles) {
+                m_lo = lo + (int64_t)(mt - acc) * SG_M;
+                m_hi = min((int64_t)hi, m_lo + SG_M);
+                found = true;
+                break;
+            }
+            acc += tiles;
+        }
+        if (!found) return;
+    } else {
+        m_lo = (int64_t)mt * SG_M;
+        if (m_lo >= a.M) return;
+        m_hi = min(a.M, m_lo + SG_M);
+    }
+    const int n0 = nt * SG_N;
+    const float* B1 = a.B1[a.offsets ? e : 0];
+    const int tx = tid & 15, ty = tid >> 4;
+    float acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+
+    for (int seg = 0; seg < 2; ++seg) {
+        const float* A = seg == 0 ? a.A0 : a.A1;
+        const float* B = seg == 0 ? a.B0 : B1;
+        const int K = seg == 0 ? a.K0 : a.K1;
+        const int64_t lda = seg == 0 ? a.lda0 : a.lda1;
+        if (A == nullptr || K == 0) continue;
+        for (int k0 = 0; k0 < K; k0 += SG_K) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int idx = tid + i * 256;
+                const int r = idx >> 4, kk = idx & 15;
+                const int64_t m = m_lo + r;
+                float v = 0.f;
+                if (m < m_hi && k0 + kk < K) {
+                    const int64_t ar = (seg == 0 && a.a_rows) ? (int64_t)a.a_rows[m] : m;
+                    v = A[ar * lda + k0 + kk];
+                }
+                As[kk][r] = v;
+                const int n = n0 + r;
+                float w = 0.f;
+                if (n < a.N && k0 + kk < K) w = B[(int64_t)n * K + k0 + kk];
+                Bs[kk][r] = w;
+            }
+            __syncthreads();
+#pragma unroll
+            for (int kk = 0; kk < SG_K; ++kk) {
+                float av[4], bv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) av[i] = As[kk][ty * 4 + i];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) bv[j] = Bs[kk][tx * 4 + j];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+            }
+            __syncthreads();
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int64_t m = m_lo + ty * 4 + i;
+        if (m >= m_hi) continue;
+        const int64_t orow = a.c_rows ? (int64_t)a.c_rows[m] : m;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int n = n0 + tx * 4 + j;
+            if (n >= a.N) continue;
+            float v = acc[i][j];
+            if (a.bias) v += a.bias[n];
+            if (a.gelu) v = gelu_erf(v);
+            if (a.scale) v *= a.scale[n];
+            a.C[orow * a.ldc + n] = v;
+        }
+    }
+}
+
+cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
+    const int n_tiles_n = (a.N + SG_N - 1) / SG_N;
+    int64_t m_tiles = (a.M + SG_M - 1) / SG_M;
+    if (a.offsets) m_tiles += a.E;  // each expert adds at most one ragged tile
+    const int64_t blocks = m_tiles * n_tiles_n;
+    if (blocks <= 0) return cudaSuccess;
+    simt_gemm_kernel<<<(unsigned)blocks, 256, 0, s>>>(a, n_tiles_n);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ LayerNorm (no affine)
+// One warp per token row; fp32 statistics in two passes over registers (mean, then the biased
+// variance of the centred values); x = (y - mean) / sqrt(var + 1e-6).
+template <bool BF16>
+__global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x, int64_t T, int d) {
+    const int lane = threadIdx.x & 31;
+    const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (row >= T) return;
+    constexpr int VEC = BF16 ? 8 : 4;  // elements per 16-byte chunk
+    constexpr int MAXC = 4;            // chunks per lane: d <= 32 * MAXC * VEC
+    float v[MAXC][VEC];
+    const int nch = d / VEC;
+    float sum = 0.f;
+#pragma unroll
+    for (int c = 0; c < MAXC; ++c) {
+        const int ch = lane + 32 * c;
+        if (ch < nch) {
+            const uint4 u = reinterpret_cast<const uint4*>(
+                static_cast<const unsigned char*>(y) + (row * d + (int64_t)ch * VEC) * (BF16 ? 2 : 4))[0];
+            if constexpr (BF16) {
+                const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    v[c][2 * j] = bf16_lo(w[j]);
+                    v[c][2 * j + 1] = bf16_hi(w[j]);
+                }
+            } else {
+                v[c][0] = __uint_as_float(u.x);
+                v[c][1] = __uint_as_float(u.y);
+                v[c][2] = __uint_as_float(u.z);
+                v[c][3] = __uint_as_float(u.w);
+            }
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) sum += v[c][j];
+        }
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    const float mean = sum / (float)d;
+    float sq = 0.f;
+#pragma unroll
+    for (int c = 0; c < MAXC; ++c) {
+        if (lane + 32 * c < nch) {
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) {
+                const float t = v[c][j] - mean;
+                sq += t * t;
+            }
+        }
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+    const float inv = 1.0f / sqrtf(sq / (float)d + 1e-6f);
+#pragma unroll
+    for (int c = 0; c < MAXC; ++c) {
+        const int ch = lane + 32 * c;
+        if (ch < nch) {
+            uint4 u;
+            if constexpr (BF16) {
+                uint32_t w[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    w[j] = pack_bf16((v[c][2 * j] - mean) * inv, (v[c][2 * j + 1] - mean) * inv);
+                u = make_uint4(w[0], w[1], w[2], w[3]);
+            } else {
+                u = make_uint4(__float_as_uint((v[c][0] - mean) * inv), __float_as_uint((v[c][1] - mean) * inv),
+                               __float_as_uint((v[c][2] - mean) * inv), __float_as_uint((v[c][3] - mean) * inv));
+            }
+            reinterpret_cast<uint4*>(static_cast<unsigned char*>(x) +
+                                     (row * d + (int64_t)ch * VEC) * (BF16 ? 2 : 4))[0] = u;
+        }
+    }
+}
+
+cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s) {
+    const unsigned blocks = (unsigned)((T + 7) / 8);
+    if (dtype == CLEARMOE_BF16)
+        layer_norm_kernel<true><<<blocks, 256, 0, s>>>(y, x, T, d);
+    else
+        layer_norm_kernel<false><<<blocks, 256, 0, s>>>(y, x, T, d);
+    return cudaGetLastError();
+}
+
+}  // namespace cm

@@ -1,0 +1,416 @@
+// bf16 GEMMs of the CLEAR-MoE FFN on the 5th-generation tensor cores (tcgen05, sm_103a).
+//
+//   C[m, n] = epilogue( sum_k A[m, k] B[n, k] ),  A and B K-major bf16, fp32 accumulate in TMEM.
+//
+// One persistent, warp-specialised kernel per (N tile width, operand mode):
+//   warps 0-3  epilogue: tcgen05.ld of the accumulator (one TMEM lane quarter each), bias+GELU /
+//              column scale / plain, round to bf16, stage through shared memory, coalesced
+//              16-byte stores; rows may be scattered (out[perm[slot]], Algorithm 3 step 6);
+//   warp 4     TMEM allocation and the single thread that issues tcgen05.mma (M=128, N=BN,
+//              K=16 per instruction) and tcgen05.commit;
+//   warp 5     TMA producer (dense / grouped modes): 128-byte-swizzled A and B tiles;
+//   warps 6-9  gather producers (gather mode): the A rows of fc1 are tokens picked by the routing
+//              permutation, so they are copied row by row with 16-byte cp.async straight into the
+//              swizzled layout (chunk j of row r at r*128 + (j ^ (r & 7))*16), while B comes by TMA.
+// Stages of a shared-memory ring are handed over by mbarriers (full: TMA bytes / cp.async
+// arrivals; empty: tcgen05.commit). Two TMEM accumulators let the epilogue of one tile overlap the
+// MMAs of the next. The grouped mode walks tiles (expert, m-tile, n-tile) from the device-resident
+// expert offsets and chains two K segments into one accumulator: [t | z] x [U_r | W_e^res].
+// Every wait is bounded; on time-out the CTA records CLEARMOE_ETIMEOUT, drains its in-flight
+// copies and MMAs, frees TMEM and returns.
+#include "common.cuh"
+#include "internal.h"
+
+namespace cm {
+
+constexpr int TC_BM = 128;
+constexpr int TC_BK = 64;
+constexpr int TC_NUM_EPI = 4;
+constexpr int TC_WARP_MMA = 4;
+constexpr int TC_WARP_TMA = 5;
+constexpr int TC_WARP_GATHER = 6;
+constexpr int TC_GATHER_THREADS = 128;
+
+template <int BN>
+struct TcCfg {
+    static constexpr int A_BYTES = TC_BM * TC_BK * 2;
+    static constexpr int B_BYTES = BN * TC_BK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int STAGES_RAW = (200 * 1024) / STAGE_BYTES;
+    static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
+    static constexpr int CW = BN < 32 ? BN : 32;      // epilogue columns per TMEM load
+    static constexpr int STG_ROW = CW * 2 + 16;       // staging row pitch (bytes)
+    static constexpr int STG_BYTES = TC_NUM_EPI * 32 * STG_ROW;
+    static constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128
+                                     : (2 * BN <= 256) ? 256 : 512;
+    static constexpr int NBARS = 2 * STAGES + 5;
+    static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + NBARS * 8 + 16 + 4 * 20;
+};
+
+struct TileInfo {
+    int64_t m0;
+    int rows;
+    int n0;
+    int e;
+};
+
+__device__ __forceinline__ TileInfo decode_tile(const TcGemmArgs& a, int tile, int n_tiles,
+                                                const int* s_prefix, int BN) {
+    TileInfo t;
+    const int mt = tile / n_tiles;
+    t.n0 = (tile % n_tiles) * BN;
+    if (a.mode == TC_GROUPED) {
+        int e = 0;
+        while (e + 1 < a.E && s_prefix[e + 1] <= mt) ++e;
+        const int64_t lo = a.offsets[e], hi = a.offsets[e + 1];
+        t.m0 = lo + (int64_t)(mt - s_prefix[e]) * TC_BM;
+        t.rows = (int)min((int64_t)TC_BM, hi - t.m0);
+        t.e = e;
+    } else {
+        t.m0 = (int64_t)mt * TC_BM;
+        t.rows = (int)min((int64_t)TC_BM, a.M - t.m0);
+        t.e = 0;
+    }
+    return t;
+}
+
+template <int BN, int MODE>
+__global__ void __launch_bounds__(MODE == TC_GATHER ? 320 : 192, 1)
+    tc_gemm_kernel(const __grid_constant__ TcGemmArgs a) {
+    using C = TcCfg<BN>;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    unsigned char* sm = smem_raw + ((1024 - (raw_addr & 1023)) & 1023);
+    unsigned char* stg = sm + C::STAGES * C::STAGE_BYTES;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(stg + C::STG_BYTES);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::NBARS);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    int* s_prefix = reinterpret_cast<int*>(tmem_slot + 4);  // [CM_MAX_E + 1]
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (C::STAGES + s); };
+    auto tfull_bar = [&](int i) { return bar0 + 8u * (2 * C::STAGES + i); };
+    auto tempty_bar = [&](int i) { return bar0 + 8u * (2 * C::STAGES + 2 + i); };
+    const uint32_t drain_bar = bar0 + 8u * (2 * C::STAGES + 4);
+    const uint64_t lim = (uint64_t)a.wait_limit_ns;
+
+    const int n_tiles = a.N / BN;
+    const int nk0 = (a.K0 + TC_BK - 1) / TC_BK;
+    const int nk1 = MODE == TC_GROUPED ? (a.K1 + TC_BK - 1) / TC_BK : 0;
+    const int nkb = nk0 + nk1;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::STAGES; ++s) {
+            mbar_init(full_bar(s), MODE == TC_GATHER ? TC_GATHER_THREADS + 1 : 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(tfull_bar(i), 1);
+            mbar_init(tempty_bar(i), TC_NUM_EPI);
+        }
+        mbar_init(drain_bar, 1);
+        *abort_flag = 0;
+        if (MODE == TC_GROUPED) {
+            int acc = 0;
+            for (int e = 0; e < a.E; ++e) {
+                s_prefix[e] = acc;
+                acc += (a.offsets[e + 1] - a.offsets[e] + TC_BM - 1) / TC_BM;
+            }
+            s_prefix[a.E] = acc;
+        }
+        mbar_fence_init();
+    }
+    if (warp == TC_WARP_MMA) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    int m_tiles;
+    if (MODE == TC_GROUPED)
+        m_tiles = s_prefix[a.E];
+    else
+        m_tiles = (int)((a.M + TC_BM - 1) / TC_BM);
+    const int num_tiles = m_tiles * n_tiles;
+
+    if (MODE != TC_GATHER && warp == TC_WARP_TMA) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t ph = 0;
+            uint32_t issued = 0;  // bit s: stage s has a load in flight or done
+            uint32_t par = 0;     // bit s: parity of stage s's last load
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+                const TileInfo t = decode_tile(a, tile, n_tiles, s_prefix, BN);
+                for (int kb = 0; kb < nkb; ++kb) {
+                    if (!mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sA = smem_u32(sm + stage * C::STAGE_BYTES);
+                    const uint32_t sB = sA + C::A_BYTES;
+                    mbar_arrive_expect_tx(full_bar(stage), C::STAGE_BYTES);
+                    if (kb < nk0) {
+                        tma_load_2d(sA, &a.tmA0, kb * TC_BK, (int)t.m0, full_bar(stage));
+                        tma_load_2d(sB, &a.tmB0, kb * TC_BK, t.n0, full_bar(stage));
+                    } else {
+                        const int kk = (kb - nk0) * TC_BK;
+                        tma_load_2d(sA, &a.tmA1, kk, (int)t.m0, full_bar(stage));
+                        tma_load_2d(sB, &a.tmB1[t.e], kk, t.n0, full_bar(stage));
+                    }
+                    issued |= 1u << stage;
+                    par = (par & ~(1u << stage)) | (ph << stage);
+                    if (++stage == C::STAGES) {
+                        stage = 0;
+                        ph ^= 1;
+                    }
+                }
+            }
+            if (!ok) {  // let every copy in flight land before the CTA retires
+                for (int s = 0; s < C::STAGES; ++s)
+                    if (issued & (1u << s)) mbar_wait(full_bar(s), (par >> s) & 1, nullptr, a.status, 10000000ull);
+            }
+        }
+    } else if (MODE == TC_GATHER && warp >= TC_WARP_GATHER) {
+        // ------------------------------------------------ gather producers (fc1 in expert order)
+        const int pt = threadIdx.x - TC_WARP_GATHER * 32;
+        const int cch = pt & 7;   // 16-byte chunk of the 128-byte row segment
+        const int rsub = pt >> 3; // rows rsub + 16 i
+        const uint16_t* X = static_cast<const uint16_t*>(a.gather_src);
+        int stage = 0;
+        uint32_t ph = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+            const TileInfo t = decode_tile(a, tile, n_tiles, s_prefix, BN);
+            int64_t src[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int r = rsub + 16 * i;
+                src[i] = (r < t.rows) ? (int64_t)a.rows[t.m0 + r] : -1;
+            }
+            for (int kb = 0; kb < nkb; ++kb) {
+                if (!mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t sA = smem_u32(sm + stage * C::STAGE_BYTES);
+                const uint32_t sB = sA + C::A_BYTES;
+                if (pt == 0) {
+                    mbar_arrive_expect_tx(full_bar(stage), C::B_BYTES);
+                    tma_load_2d(sB, &a.tmB0, kb * TC_BK, t.n0, full_bar(stage));
+                }
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int r = rsub + 16 * i;
+                    if (src[i] >= 0)
+                        cp_async_16(sA + r * 128 + ((cch ^ (r & 7)) << 4),
+                                    X + src[i] * a.gather_ld + kb * TC_BK + cch * 8);
+                }
+                asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(full_bar(stage))
+                             : "memory");
+                if (++stage == C::STAGES) {
+                    stage = 0;
+                    ph ^= 1;
+                }
+            }
+        }
+        cp_async_wait<0>();
+    } else if (warp == TC_WARP_MMA) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(TC_BM, BN);
+            int stage = 0;
+            uint32_t ph = 0;
+            int acc = 0;
+            uint32_t aph = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+                if (!mbar_wait(tempty_bar(acc), aph ^ 1, abort_flag, a.status, lim)) break;
+                tc_fence_after();
+                const uint32_t dtm = tmem_base + acc * BN;
+                for (int kb = 0; kb < nkb; ++kb) {
+                    if (!mbar_wait(full_bar(stage), ph, abort_flag, a.status, lim)) {
+                        ok = false;
+                        break;
+                    }
+                    if (MODE == TC_GATHER) fence_proxy_async_smem();
+                    tc_fence_after();
+                    const uint32_t sA = smem_u32(sm + stage * C::STAGE_BYTES);
+                    const uint32_t sB = sA + C::A_BYTES;
+                    const int kvalid = kb < nk0 ? min(TC_BK, a.K0 - kb * TC_BK)
+                                                : min(TC_BK, a.K1 - (kb - nk0) * TC_BK);
+                    const int steps = kvalid >> 4;
+                    for (int k = 0; k < steps; ++k)
+                        umma_bf16(dtm, sdesc_kmajor_sw128(sA + k * 32), sdesc_kmajor_sw128(sB + k * 32),
+                                  idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                    umma_commit(empty_bar(stage));
+                    if (++stage == C::STAGES) {
+                        stage = 0;
+                        ph ^= 1;
+                    }
+                }
+                if (!ok) break;
+                umma_commit(tfull_bar(acc));
+                acc ^= 1;
+                if (acc == 0) aph ^= 1;
+            }
+            umma_commit(drain_bar);  // every MMA issued above has completed once this fires
+            mbar_wait(drain_bar, 0, nullptr, a.status, 10000000ull);
+        }
+        __syncwarp();
+    } else if (warp < TC_NUM_EPI) {
+        // ------------------------------------------------ epilogue
+        const int q = warp;
+        unsigned char* wstg = stg + warp * 32 * C::STG_ROW;
+        constexpr int LPR = C::CW / 8;  // lanes per staged row (16 bytes each)
+        constexpr int RPP = 32 / LPR;   // rows per store pass
+        int acc = 0;
+        uint32_t aph = 0;
+        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+            const TileInfo t = decode_tile(a, tile, n_tiles, s_prefix, BN);
+            if (!mbar_wait(tfull_bar(acc), aph, abort_flag, a.status, lim)) break;
+            tc_fence_after();
+            const int r = q * 32 + lane;
+            int64_t orow = -1;
+            if (r < t.rows) orow = (a.epi == TC_EPI_SCATTER) ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
+            for (int c = 0; c < BN; c += C::CW) {
+                uint32_t v[C::CW];
+                const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
+                CM_TMEM_LD_X16(taddr, v);
+                if constexpr (C::CW == 32) CM_TMEM_LD_X16(taddr + 16, (v + 16));
+                tmem_wait_ld();
+                float f[C::CW];
+#pragma unroll
+                for (int j = 0; j < C::CW; ++j) f[j] = __uint_as_float(v[j]);
+                const int nb = t.n0 + c;
+                if (a.epi == TC_EPI_BIAS_GELU) {
+                    const uint4* bp = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.bias) + nb);
+#pragma unroll
+                    for (int j8 = 0; j8 < C::CW / 8; ++j8) {
+                        const uint4 b = __ldg(bp + j8);
+                        const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+                        for (int h = 0; h < 4; ++h) {
+                            f[j8 * 8 + 2 * h] = gelu_erf(f[j8 * 8 + 2 * h] + bf16_lo(bw[h]));
+                            f[j8 * 8 + 2 * h + 1] = gelu_erf(f[j8 * 8 + 2 * h + 1] + bf16_hi(bw[h]));
+                        }
+                    }
+                } else if (a.epi == TC_EPI_SCALE) {
+#pragma unroll
+                    for (int j4 = 0; j4 < C::CW / 4; ++j4) {
+                        const float4 s4 = __ldg(reinterpret_cast<const float4*>(a.scale + nb) + j4);
+                        f[4 * j4] *= s4.x;
+                        f[4 * j4 + 1] *= s4.y;
+                        f[4 * j4 + 2] *= s4.z;
+                        f[4 * j4 + 3] *= s4.w;
+                    }
+                }
+                uint4* dst = reinterpret_cast<uint4*>(wstg + lane * C::STG_ROW);
+#pragma unroll
+                for (int j8 = 0; j8 < C::CW / 8; ++j8)
+                    dst[j8] = make_uint4(pack_bf16(f[8 * j8], f[8 * j8 + 1]), pack_bf16(f[8 * j8 + 2], f[8 * j8 + 3]),
+                                         pack_bf16(f[8 * j8 + 4], f[8 * j8 + 5]), pack_bf16(f[8 * j8 + 6], f[8 * j8 + 7]));
+                __syncwarp();
+#pragma unroll
+                for (int p = 0; p < LPR; ++p) {
+                    const int rr = p * RPP + lane / LPR;
+                    const int64_t o = __shfl_sync(0xffffffffu, orow, rr);
+                    const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * C::STG_ROW + (lane % LPR) * 16);
+                    if (o >= 0)
+                        *reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.C) + o * a.ldc + nb + (lane % LPR) * 8) = val;
+                }
+                __syncwarp();
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty_bar(acc));
+            acc ^= 1;
+            if (acc == 0) aph ^= 1;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == TC_WARP_MMA) tmem_dealloc(tmem_base, C::TMEM_COLS);
+}
+
+// ------------------------------------------------------------------ host side
+int tc_pick_bn(int mode, int N) {
+    (void)mode;
+    const int cands[5] = {256, 128, 64, 32, 16};
+    for (int c : cands)
+        if (N % c == 0) return c;
+    return 0;
+}
+
+template <int BN, int MODE>
+static cudaError_t launch_one(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
+    using C = TcCfg<BN>;
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<BN, MODE>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    const int n_tiles = a.N / BN;
+    int64_t m_tiles = (a.M + TC_BM - 1) / TC_BM;
+    if (MODE == TC_GROUPED) m_tiles += a.E;
+    int64_t tiles = m_tiles * n_tiles;
+    const int grid = (int)(tiles < num_sms ? tiles : num_sms);
+    if (grid <= 0) return cudaSuccess;
+    tc_gemm_kernel<BN, MODE><<<grid, MODE == TC_GATHER ? 320 : 192, C::SMEM, s>>>(a);
+    return cudaGetLastError();
+}
+
+template <int MODE>
+static cudaError_t launch_mode(const TcGemmArgs& a, int bn, int num_sms, cudaStream_t s) {
+    switch (bn) {
+        case 256: return launch_one<256, MODE>(a, num_sms, s);
+        case 128: return launch_one<128, MODE>(a, num_sms, s);
+        case 64: return launch_one<64, MODE>(a, num_sms, s);
+        case 32: return launch_one<32, MODE>(a, num_sms, s);
+        case 16: return launch_one<16, MODE>(a, num_sms, s);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_tc_gemm(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
+    const int bn = tc_pick_bn(a.mode, a.N);
+    if (bn == 0) return cudaErrorInvalidValue;
+    if (a.mode == TC_GATHER) return launch_mode<TC_GATHER>(a, bn, num_sms, s);
+    if (a.mode == TC_GROUPED) return launch_mode<TC_GROUPED>(a, bn, num_sms, s);
+    return launch_mode<TC_DENSE>(a, bn, num_sms, s);
+}
+
+typedef CUresult (*PFN_encodeTiled_t)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                      const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                      const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                      CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+int encode_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
+    static PFN_encodeTiled_t fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess || !p)
+            return -1;
+        fn = reinterpret_cast<PFN_encodeTiled_t>(p);
+    }
+    const cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    const cuuint64_t gstride[1] = {(cuuint64_t)cols * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)TC_BK, (cuuint32_t)box_rows};
+    const cuuint32_t es[2] = {1, 1};
+    const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride, box, es,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? 0 : -2;
+}
+
+}  // namespace cm

@@ -291,3 +291,19 @@ def make_stack(shape: StackShape = VIT_BASE_STACK12, T: int | None = None) -> di
         layers.append(L)
         x_cal = layer_norm(_hidden(xc, W1, b1) @ W2.T.astype(np.float32))
     return dict(shape=shape, dtype="bf16", x=round_bf16(x), layers=layers, T=T)
+
+
+def to_torch(layer: dict, device="cuda") -> dict:
+    """Device copies of a layer's arrays in its dtype (bf16 values convert exactly); S_r and
+    the integer metadata keep their types."""
+    import torch
+
+    tdt = torch.bfloat16 if layer.get("dtype", "bf16") == "bf16" else torch.float32
+    out = {}
+    for k in ("x", "W1", "b1", "W2", "U", "Vh", "residuals", "Wg", "bg"):
+        if k in layer:
+            out[k] = torch.from_numpy(np.ascontiguousarray(layer[k], dtype=np.float32)).to(
+                device=device, dtype=tdt).contiguous()
+    if "S" in layer:
+        out["S"] = torch.from_numpy(np.ascontiguousarray(layer["S"], dtype=np.float32)).to(device)
+    return out
