@@ -1,0 +1,390 @@
+#!/usr/bin/env python
+"""Throughput of the CLEAR-MoE FFN layer on GB300; prints one JSON line.
+
+A step is one CLEAR-MoE FFN forward (routing, fc1 + GELU, shared-basis factor, grouped residual
+experts with the scatter) over one batch of synthetic ViT tokens, through the library's C ABI.
+The default workload is the DeiT-B / ViT-B-shaped layer (T = 256 images x 197 tokens = 50,432,
+d = 768, H = 3,072, E = 8, r = 128, bf16), the shape the GEMM target is quoted on.
+
+  value  tokens/s over K timed steps (inputs resident in HBM), CUDA events on the launch stream,
+         L2 flushed (a 256 MB write) before every step, outside the timed events
+  e2e    the same call with x copied from pinned host memory and out copied back inside each step
+  roofline  the dominant kernel's algorithmic FLOPs (or bytes) per launch / its event-timed duration
+  cpu_baseline  the float64 CPU oracle on a bounded sample of the same workload (rank 0, N = 1)
+
+--impl reference times the CPU oracle itself (the method has no other reference code).
+Multi-GPU (torchrun): every rank runs an independent replica on its own tokens (weak scaling;
+the layer needs no exchange between token shards); value = all tokens / max rank time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import pathlib
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = pathlib.Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+METRIC = ("CLEAR-MoE FFN tokens/sec/layer (1×GB300) + % HBM peak (dispatch), "
+          "% tensor peak (GEMMs)")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+STAGES = ("route", "fc1_gelu", "basis", "grouped")
+KERNEL_OF_STAGE = {"route": "route_kernel", "fc1_gelu": "tc_gemm_kernel<256, gather>",
+                   "basis": "tc_gemm_kernel<128, dense>", "grouped": "tc_gemm_kernel<256, grouped>"}
+# DRAM traffic per launch from the committed ncu capture (profiles/), with the hash of the kernel
+# source it was taken on; a different hash means the kernel changed and the figure is void.
+TRAFFIC = {}
+
+
+def workloads():
+    import synth
+    return {"deit_base_bf16": synth.DEIT_BASE_BF16, "deit_small_bf16": synth.DEIT_SMALL_BF16,
+            "deit_tiny_fp32": synth.DEIT_TINY_FP32}
+
+
+def peaks():
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        d = json.loads(p.read_text())
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def stage_work(s):
+    """Algorithmic work per launch of each kernel (per-token figures x T)."""
+    esz = 2 if s.dtype == "bf16" else 4
+    T, d, H, E, r = s.T, s.d, s.H, s.E, s.r
+    return {
+        "route": {"bytes": T * d * esz + (E * d + E) * esz + 8 * T + 8 * E, "flops": 2 * T * d * E},
+        "fc1_gelu": {"flops": 2 * T * d * H},
+        "basis": {"flops": 2 * T * H * r},
+        "grouped": {"flops": 2 * T * d * r + 2 * T * d * H},
+    }
+
+
+def layer_roofline_s(s, pk):
+    esz = 2 if s.dtype == "bf16" else 4
+    T, d, H, E, r = s.T, s.d, s.H, s.E, s.r
+    flops = T * (2 * d * H + 2 * r * (H + d) + 2 * d * H + 2 * d * E)
+    weights = (H * d + H + d * r + r + r * H + E * d * H + E * d + E) * esz
+    bytes_ = 2 * T * d * esz + weights
+    return max(flops / (pk["bf16_tflops_sustained"] * 1e12), bytes_ / (pk["hbm_gbs"] * 1e9))
+
+
+def source_hash():
+    h = hashlib.sha256()
+    for f in sorted((ROOT / "paper_2606_28516_gb300" / "csrc").glob("*")):
+        h.update(f.read_bytes())
+    return h.hexdigest()[:16]
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 100 ms during the timed region."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        self.rows = []
+        if self.proc is None:
+            return
+        time.sleep(0.2)
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) == 7:
+                self.rows.append(f)
+
+    def summary(self):
+        if not getattr(self, "rows", None):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[3 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(self.rows)}
+
+
+def oracle_rate(L, budget_s=12.0, chunk=1024, max_tokens=None):
+    """Oracle tokens/s on row chunks of the workload until budget_s of CPU time is spent."""
+    import numpy as np
+    from oracle import clearmoe as O
+    s = L["shape"]
+    rt = O.route(L["x"][: min(s.T, 8192)], L["Wg"], L["bg"])  # warm the BLAS threads
+    del rt
+    done, t0 = 0, time.perf_counter()
+    limit = max_tokens or s.T
+    while done < limit:
+        n = min(chunk, limit - done)
+        rows = slice(done, done + n)
+        a = O.route(L["x"][rows], L["Wg"], L["bg"])["a"]
+        O.ffn_forward(L["x"][rows], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], L["residuals"],
+                      a=a, z_bf16=s.dtype == "bf16")
+        done += n
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    el = time.perf_counter() - t0
+    return done / el, done, el
+
+
+def blas_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return len(os.sched_getaffinity(0))
+
+
+def run_reference(args):
+    import numpy as np  # noqa: F401
+    import synth
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    shape = workloads()[args.workload]
+    L = synth.make_layer(shape)
+    # per-step sample sized so that warmup + steps take about a minute of CPU time in total
+    probe, _, _ = oracle_rate(L, budget_s=2.0, chunk=256, max_tokens=512)
+    per_step = max(16, min(4096, int(probe * 60.0 / max(1, args.steps + args.warmup))))
+    for _ in range(args.warmup):
+        oracle_rate(L, budget_s=1e9, chunk=per_step, max_tokens=per_step)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_rate(L, budget_s=1e9, chunk=per_step, max_tokens=per_step)
+    el = time.perf_counter() - t0
+    value = per_step * args.steps / el
+    cores = blas_threads()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": el * 1e3 / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": shape.name, "T": shape.T, "d": shape.d, "H": shape.H,
+                   "E": shape.E, "r": shape.r, "sample_tokens_per_step": per_step},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{per_step} tokens of the workload per step (float64 numpy "
+                                   f"oracle, Algorithm 3 order, W_shared materialised per call)"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="deit_base_bf16", choices=sorted(workloads()))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=100)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import numpy as np
+    import torch
+
+    import synth
+    import __graft_entry__
+    from paper_2606_28516_gb300 import clearmoe as cm
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    if rank == 0:
+        __graft_entry__.build()
+    if dist:
+        dist.barrier()
+    cm.lib()
+
+    shape = workloads()[args.workload].with_(seed=rank)
+    L = synth.make_layer(shape)
+    D = synth.to_torch(L)
+    s = shape
+    dt = cm.BF16 if s.dtype == "bf16" else cm.F32
+    h = cm.clearmoe_layer_create(s.T, s.d, s.H, s.E, s.r, dt)
+    out = torch.empty(s.T, s.d, device="cuda", dtype=D["x"].dtype)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.int32, device="cuda")  # 256 MB > L2
+    stream = torch.cuda.current_stream()
+
+    def forward(x=None):
+        cm.clearmoe_ffn_forward(h, D["x"] if x is None else x, D["W1"], D["b1"], D["U"], D["S"],
+                                D["Vh"], D["residuals"], D["Wg"], D["bg"], out)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        forward()
+    torch.cuda.synchronize()
+    assert cm.clearmoe_layer_status(h) == 0
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        wall0 = time.perf_counter()
+        for k in range(K):
+            flush.zero_()
+            cm.clearmoe_set_profile_events(h, ev[k])
+            forward()
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+    cm.clearmoe_set_profile_events(h, [])
+    if dist:
+        dist.barrier()
+    assert cm.clearmoe_layer_status(h) == 0
+    stage_ms = {st: [ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)]
+                for i, st in enumerate(STAGES)}
+    step_ms = [ev[k][0].elapsed_time(ev[k][4]) for k in range(K)]
+    total_ms = float(sum(step_ms))
+    if dist:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    value = world * s.T * K / (total_ms / 1e3)
+
+    # same-GPU dense FFN, same timing rules
+    dense_ms = []
+    dout = torch.empty_like(out)
+    dev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(min(K, 200))]
+    for k in range(len(dev) + args.warmup):
+        flush.zero_()
+        if k >= args.warmup:
+            cm.clearmoe_set_profile_events(h, dev[k - args.warmup])
+        cm.clearmoe_dense_ffn_forward(h, D["x"], D["W1"], D["b1"], D["W2"], dout)
+    torch.cuda.synchronize()
+    cm.clearmoe_set_profile_events(h, [])
+    dense_ms = [e[0].elapsed_time(e[2]) for e in dev]
+    dense_value = s.T / (statistics.mean(dense_ms) / 1e3)
+
+    # end to end through the C ABI with host buffers: H2D of x and D2H of out inside each step
+    x_host = D["x"].cpu().pin_memory()
+    out_host = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    x_dev = torch.empty_like(D["x"])
+    Ke = max(1, min(args.e2e_steps, K))
+    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(Ke)]
+    for k in range(Ke + args.warmup):
+        flush.zero_()
+        if k >= args.warmup:
+            e2e_ev[k - args.warmup][0].record(stream)
+        x_dev.copy_(x_host, non_blocking=True)
+        forward(x_dev)
+        out_host.copy_(out, non_blocking=True)
+        if k >= args.warmup:
+            e2e_ev[k - args.warmup][1].record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_ev)
+    if dist:
+        t = torch.tensor([e2e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = world * s.T * Ke / (e2e_ms / 1e3)
+    assert cm.clearmoe_layer_status(h) == 0
+    cm.clearmoe_layer_destroy(h)
+
+    pk, pk_src = peaks()
+    work = stage_work(s)
+    avg = {st: statistics.mean(v) for st, v in stage_ms.items()}
+    dom = max(avg, key=avg.get)
+    dur_s = avg[dom] / 1e3
+    if dom == "route":
+        ach = work[dom]["bytes"] / dur_s / 1e9
+        roof = {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s"}
+    else:
+        ach = work[dom]["flops"] / dur_s / 1e12
+        roof = {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops_sustained"],
+                "unit": "TFLOP/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    tr = TRAFFIC.get(dom)
+    roof["traffic"] = tr["bytes"] if tr and tr["src"] == source_hash() else None
+    roof["kernel"] = KERNEL_OF_STAGE[dom]
+    roof["peak_source"] = f"{pk_src} ({'sustained bf16' if roof['bound'] == 'tensor' else 'HBM copy'})"
+
+    per_stage = {}
+    for st in STAGES:
+        d_s = avg[st] / 1e3
+        if "bytes" in work[st]:
+            g = work[st]["bytes"] / d_s / 1e9
+            per_stage[st] = {"us": avg[st] * 1e3, "GB_s": g, "hbm_frac": g / pk["hbm_gbs"]}
+        else:
+            tf = work[st]["flops"] / d_s / 1e12
+            per_stage[st] = {"us": avg[st] * 1e3, "TFLOP_s": tf,
+                             "tensor_frac": tf / pk["bf16_tflops_sustained"]}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, n, el = oracle_rate(L, budget_s=12.0)
+        cpu = {"value": rate, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle",
+               "sample": f"first {n} tokens of the workload in 1,024-token chunks ({el:.1f} s; "
+                         f"float64 numpy oracle, routing + Algorithm 3)"}
+
+    mean_step = total_ms / K
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": mean_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": s.dtype, "data": "synthetic",
+        "config": {"workload": s.name, "T": s.T, "d": s.d, "H": s.H, "E": s.E, "r": s.r,
+                   "tokens": "Gaussian-mixture ViT tokens, layer-normalised; weights N(0, 0.02^2) "
+                             "converted by truncated SVD + k-means (seeded)",
+                   "l2": "flushed before every step (256 MB write, outside the timed events)",
+                   "parallelism": f"replicas{world}"},
+        "e2e": {"value": e2e_value, "unit": "tokens/s",
+                "h2d_bytes_per_step": int(D["x"].numel() * D["x"].element_size()),
+                "d2h_bytes_per_step": int(out.numel() * out.element_size())},
+        "gpu_launches": 4 * K,
+        "roofline": roof,
+        "cpu_baseline": cpu,
+        "clocks": clk.summary(),
+        "stages": per_stage,
+        "layer_roofline_frac": layer_roofline_s(s, pk) / (mean_step / 1e3),
+        "dense_ffn": {"value": dense_value, "unit": "tokens/s",
+                      "ms_per_step": statistics.mean(dense_ms)},
+        "wall_s_timed": wall,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -128,6 +128,13 @@ int clearmoe_layer_status(clearmoe_layer* layer);
  * CLEARMOE_ETIMEOUT through clearmoe_layer_status. phantom_arrivals = 0 restores normal use. */
 int clearmoe_debug_set_wait(clearmoe_layer* layer, int64_t wait_limit_ns, int32_t phantom_arrivals);
 
+/* Per-stage timing: when n >= 5, clearmoe_ffn_forward records events[0] before its first kernel
+ * and events[i] after its i-th kernel (1 routing, 2 fc1 + GELU, 3 shared-basis factor, 4 grouped
+ * residual GEMM); clearmoe_dense_ffn_forward records events[0..2] around its two kernels. The
+ * events are cudaEvent_t handles owned by the caller, recorded on the call's stream; n = 0 (or
+ * events = NULL) turns recording off. The library never waits on them. */
+int clearmoe_set_profile_events(clearmoe_layer* layer, void* const* events, int32_t n);
+
 /* Static string for a status code. */
 const char* clearmoe_strerror(int status);
 

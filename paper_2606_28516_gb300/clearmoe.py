@@ -44,6 +44,7 @@ _SIGS = {
     "clearmoe_get_routing": [_P, _P, _P, _P, _P, _P],
     "clearmoe_layer_status": [_P],
     "clearmoe_debug_set_wait": [_P, _I64, _I32],
+    "clearmoe_set_profile_events": [_P, ctypes.POINTER(ctypes.c_void_p), _I32],
     "clearmoe_strerror": [ctypes.c_int],
     "clearmoe_version": [],
 }
@@ -153,3 +154,16 @@ def clearmoe_layer_status(layer: int) -> int:
 def clearmoe_debug_set_wait(layer: int, wait_limit_ns: int, phantom_arrivals: int) -> None:
     _check(lib().clearmoe_debug_set_wait(layer, wait_limit_ns, phantom_arrivals),
            "clearmoe_debug_set_wait")
+
+
+def clearmoe_set_profile_events(layer: int, events) -> None:
+    """events: torch.cuda.Event(enable_timing=True) objects (or none to stop recording). torch
+    creates an event's CUDA handle on its first record, so each is recorded once here first; the
+    library then re-records it on the forward's stream."""
+    for e in events:
+        if not e.cuda_event:
+            e.record()
+    handles = [e.cuda_event for e in events]
+    arr = (ctypes.c_void_p * max(1, len(handles)))(*handles)
+    _check(lib().clearmoe_set_profile_events(layer, arr, len(handles)),
+           "clearmoe_set_profile_events")

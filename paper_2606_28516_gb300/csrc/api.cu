@@ -27,6 +27,8 @@ struct clearmoe_layer {
     int32_t phantom;
     int64_t last_T;
     int32_t last_E;
+    cudaEvent_t prof[8];
+    int32_t prof_n;
 };
 
 namespace {
@@ -84,6 +86,10 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
         L->last_E = E;
     }
     return rc;
+}
+
+inline void mark(const clearmoe_layer* L, int i, cudaStream_t s) {
+    if (i < L->prof_n && L->prof[i]) cudaEventRecord(L->prof[i], s);
 }
 
 int check_router(const clearmoe_layer* L, const clearmoe_router* router, int E) {
@@ -196,7 +202,9 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     if (!bf16 && r % 4) return CLEARMOE_EUNSUPPORTED;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
 
+    mark(L, 0, s);
     if ((rc = do_route(L, x, T, router, E, s))) return rc;
+    mark(L, 1, s);
 
     if (!bf16) {
         cm::SimtGemmArgs g;
@@ -214,6 +222,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
         g.C = static_cast<float*>(L->z);
         g.ldc = H;
         if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        mark(L, 2, s);
         // t = diag(S_r) Vh_r z
         std::memset(&g, 0, sizeof(g));
         g.A0 = static_cast<const float*>(L->z);
@@ -226,6 +235,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
         g.C = static_cast<float*>(L->t);
         g.ldc = r;
         if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        mark(L, 3, s);
         // out[perm[slot]] = U_r t + W_e^res z per expert sub-batch
         std::memset(&g, 0, sizeof(g));
         g.A0 = static_cast<const float*>(L->t);
@@ -243,7 +253,9 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
         g.c_rows = L->perm;
         g.offsets = L->offsets;
         g.E = E;
-        return cuda_fail(cm::launch_simt_gemm(g, s));
+        rc = cuda_fail(cm::launch_simt_gemm(g, s));
+        mark(L, 4, s);
+        return rc;
     }
 
     // ---- bf16: tcgen05 GEMMs
@@ -269,6 +281,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g.C = L->z;
     g.ldc = H;
     if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
+    mark(L, 2, s);
     // t = diag(S_r) Vh_r z
     cm::TcGemmArgs g2;
     std::memset(&g2, 0, sizeof(g2));
@@ -285,6 +298,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g2.C = L->t;
     g2.ldc = r;
     if ((rc = cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s)))) return rc;
+    mark(L, 3, s);
     // out[perm[slot]] = [t | z] [U_r | W_e^res]^T per expert sub-batch
     cm::TcGemmArgs g3;
     std::memset(&g3, 0, sizeof(g3));
@@ -306,7 +320,9 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g3.rows = L->perm;
     g3.C = out;
     g3.ldc = d;
-    return cuda_fail(cm::launch_tc_gemm(g3, L->num_sms, s));
+    rc = cuda_fail(cm::launch_tc_gemm(g3, L->num_sms, s));
+    mark(L, 4, s);
+    return rc;
 }
 
 int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
@@ -317,6 +333,7 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     if (misaligned(W1) || misaligned(b1) || misaligned(W2) || misaligned(out)) return CLEARMOE_EINVAL;
     const int d = L->desc.d, H = L->desc.hidden;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    mark(L, 0, s);
     if (L->desc.dtype == CLEARMOE_F32) {
         cm::SimtGemmArgs g;
         std::memset(&g, 0, sizeof(g));
@@ -331,6 +348,7 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
         g.C = static_cast<float*>(L->z);
         g.ldc = H;
         if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        mark(L, 1, s);
         std::memset(&g, 0, sizeof(g));
         g.A0 = static_cast<const float*>(L->z);
         g.lda0 = H;
@@ -340,7 +358,9 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
         g.N = d;
         g.C = static_cast<float*>(out);
         g.ldc = d;
-        return cuda_fail(cm::launch_simt_gemm(g, s));
+        rc = cuda_fail(cm::launch_simt_gemm(g, s));
+        mark(L, 2, s);
+        return rc;
     }
     const int bn1 = cm::tc_pick_bn(cm::TC_DENSE, H);
     const int bn2 = cm::tc_pick_bn(cm::TC_DENSE, d);
@@ -358,6 +378,7 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     g.C = L->z;
     g.ldc = H;
     if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
+    mark(L, 1, s);
     cm::TcGemmArgs g2;
     std::memset(&g2, 0, sizeof(g2));
     g2.status = L->status;
@@ -371,7 +392,9 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     g2.K0 = H;
     g2.C = out;
     g2.ldc = d;
-    return cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s));
+    rc = cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s));
+    mark(L, 2, s);
+    return rc;
 }
 
 int clearmoe_layer_norm(clearmoe_layer* L, const void* y, int64_t T, void* x_out, void* stream) {
@@ -413,6 +436,13 @@ int clearmoe_layer_status(clearmoe_layer* L) {
         if (cudaDeviceSynchronize() != cudaSuccess) return CLEARMOE_ECUDA;
     }
     return st;
+}
+
+int clearmoe_set_profile_events(clearmoe_layer* L, void* const* events, int32_t n) {
+    if (!L || n < 0 || n > 8 || (n > 0 && !events)) return CLEARMOE_EINVAL;
+    for (int i = 0; i < 8; ++i) L->prof[i] = (i < n) ? static_cast<cudaEvent_t>(events[i]) : nullptr;
+    L->prof_n = n;
+    return CLEARMOE_OK;
 }
 
 int clearmoe_debug_set_wait(clearmoe_layer* L, int64_t wait_limit_ns, int32_t phantom_arrivals) {
