@@ -135,6 +135,32 @@ int clearmoe_debug_set_wait(clearmoe_layer* layer, int64_t wait_limit_ns, int32_
  * events = NULL) turns recording off. The library never waits on them. */
 int clearmoe_set_profile_events(clearmoe_layer* layer, void* const* events, int32_t n);
 
+/* Routing without a handle, for callers that cannot allocate device memory (engines that own
+ * every device byte and forbid allocation in their enqueue path, processes held to a fixed
+ * memory budget, loops that cannot afford cudaMalloc's implicit device synchronisation). The
+ * paper has no counterpart: this is a deployment variant of clearmoe_route, with the same results
+ * (idx [T], counts [E], offsets [E + 1], perm [T]: caller-owned int32 device outputs) for tokens
+ * x [T x d] of dtype `dtype` and the router W [E x d], b [E] in that dtype.
+ *   - It calls no cudaMalloc, cudaFree or other allocating routine. Its scratch (per-CTA expert
+ *     histograms, the arrival counter of the grid-wide wait, a spare status word) is one static
+ *     device array of 65,600 bytes that every GPU loading the library holds until exit; it serves
+ *     up to 1,024 routing CTAs (two per SM on GPUs with up to 512 SMs). A launch that would need
+ *     more returns CLEARMOE_EUNSUPPORTED and enqueues nothing.
+ *   - The first call on a device looks up the array's device address (once per device, with that
+ *     device current); make that first call before any stream capture.
+ *   - Every call shares the array and it keeps the last call's contents; each call clears what
+ *     must start at zero. Calls whose work overlaps on the GPU (other streams, other host
+ *     threads) race on the array: serialise them.
+ *   - status (optional int32 device pointer, else NULL) is set to 0 at the start of the call and
+ *     receives CLEARMOE_ETIMEOUT if the bounded grid-wide wait (1 s) runs out, in which case the
+ *     outputs are undefined.
+ * Limits: 1 <= T <= 2^30, 1 <= E <= 16; bf16: d % 64 == 0, d <= 1024; fp32: d % 4 == 0, d <= 512;
+ * x and W 16-byte aligned. Host-side errors return EINVAL / EUNSUPPORTED / ECUDA with nothing
+ * enqueued. */
+int clearmoe_route_noalloc(const void* x, int64_t T, int32_t d, int32_t dtype,
+                           const clearmoe_router* router, int32_t E, int32_t* idx, int32_t* counts,
+                           int32_t* offsets, int32_t* perm, int32_t* status, void* stream);
+
 /* Static string for a status code. */
 const char* clearmoe_strerror(int status);
 

@@ -45,6 +45,8 @@ _SIGS = {
     "clearmoe_layer_status": [_P],
     "clearmoe_debug_set_wait": [_P, _I64, _I32],
     "clearmoe_set_profile_events": [_P, ctypes.POINTER(ctypes.c_void_p), _I32],
+    "clearmoe_route_noalloc": [_P, _I64, _I32, _I32, ctypes.POINTER(clearmoe_router), _I32, _P, _P,
+                               _P, _P, _P, _P],
     "clearmoe_strerror": [ctypes.c_int],
     "clearmoe_version": [],
 }
@@ -167,3 +169,17 @@ def clearmoe_set_profile_events(layer: int, events) -> None:
     arr = (ctypes.c_void_p * max(1, len(handles)))(*handles)
     _check(lib().clearmoe_set_profile_events(layer, arr, len(handles)),
            "clearmoe_set_profile_events")
+
+
+def clearmoe_route_noalloc(x, Wg, bg, idx, counts, offsets, perm, status=None,
+                           stream=None) -> None:
+    """Routing without a handle or any device allocation (see include/clearmoe.h): the outputs
+    idx [T], counts [E], offsets [E + 1], perm [T] (int32) and the optional status word are
+    caller-owned CUDA tensors."""
+    import torch
+    dtype = BF16 if x.dtype == torch.bfloat16 else F32
+    r = _router(Wg, bg)
+    _check(lib().clearmoe_route_noalloc(_ptr(x), x.shape[0], x.shape[1], dtype, ctypes.byref(r),
+                                        Wg.shape[0], _ptr(idx), _ptr(counts), _ptr(offsets),
+                                        _ptr(perm), _ptr(status), _stream(stream)),
+           "clearmoe_route_noalloc")
