@@ -39,6 +39,46 @@ __device__ __forceinline__ float gelu_erf(float u) {
     return 0.5f * u * (1.0f + erff(u * 0.70710678118654752440f));
 }
 
+// GELU of a pair for the bf16 layer, whose hidden state is stored in bf16. erf is evaluated by
+// the rational approximation of Abramowitz & Stegun, Handbook of Mathematical Functions, 7.1.28
+// (C. Hastings): erf(x) = 1 - (1 + a1 x + ... + a6 x^6)^-16 for x >= 0, |error| <= 3e-7, with
+// x = |u| / sqrt(2) folded into the coefficients. Then GELU(u) = u - u y / 2 for u >= 0 and
+// u y / 2 for u < 0, y = P^-16. Evaluated with packed fp32x2 FMAs; the absolute error of the
+// result is below 7.1e-7 for every u (checked against float64 on a 2M-point grid), far below
+// the bf16 spacing of z. The fp32 layer keeps gelu_erf (CUDA's erff).
+struct GeluAS {
+    static constexpr double S = 0.70710678118654752440;  // 1 / sqrt(2)
+    static constexpr float B1 = (float)(0.0705230784 * S);
+    static constexpr float B2 = (float)(0.0422820123 * S * S);
+    static constexpr float B3 = (float)(0.0092705272 * S * S * S);
+    static constexpr float B4 = (float)(0.0001520143 * S * S * S * S);
+    static constexpr float B5 = (float)(0.0002765672 * S * S * S * S * S);
+    static constexpr float B6 = (float)(0.0000430638 * S * S * S * S * S * S);
+};
+
+__device__ __forceinline__ float rcp_approx(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ float2 gelu_pair_as(float2 u) {
+    const float2 au = make_float2(fabsf(u.x), fabsf(u.y));
+    float2 p = __ffma2_rn(make_float2(GeluAS::B6, GeluAS::B6), au, make_float2(GeluAS::B5, GeluAS::B5));
+    p = __ffma2_rn(p, au, make_float2(GeluAS::B4, GeluAS::B4));
+    p = __ffma2_rn(p, au, make_float2(GeluAS::B3, GeluAS::B3));
+    p = __ffma2_rn(p, au, make_float2(GeluAS::B2, GeluAS::B2));
+    p = __ffma2_rn(p, au, make_float2(GeluAS::B1, GeluAS::B1));
+    p = __ffma2_rn(p, au, make_float2(1.0f, 1.0f));
+    p = __fmul2_rn(p, p);
+    p = __fmul2_rn(p, p);
+    p = __fmul2_rn(p, p);
+    p = __fmul2_rn(p, p);  // P^16 (overflows to +inf for |u| > ~10, where y = 0 is exact in fp32)
+    const float2 y = make_float2(rcp_approx(p.x), rcp_approx(p.y));
+    const float2 h = __fmul2_rn(__fmul2_rn(make_float2(0.5f, 0.5f), u), y);
+    return make_float2(u.x >= 0.f ? u.x - h.x : h.x, u.y >= 0.f ? u.y - h.y : h.y);
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -157,6 +197,12 @@ __device__ __forceinline__ void tmem_wait_ld() {
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),             \
           "=r"(r[13]), "=r"(r[14]), "=r"(r[15])                                                  \
         : "r"(taddr))
+
+#define CM_TMEM_LD_X8(taddr, r)                                                                  \
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"         \
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),        \
+                   "=r"(r[6]), "=r"(r[7])                                                         \
+                 : "r"(taddr))
 
 // Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with 128-byte swizzle:
 // rows of 128 bytes (64 elements of K), 8-row swizzle atoms 1024 bytes apart (SBO), descriptor

@@ -3,13 +3,14 @@
 //   C[m, n] = epilogue( sum_k A[m, k] B[n, k] ),  A and B K-major bf16, fp32 accumulate in TMEM.
 //
 // One persistent, warp-specialised kernel per (N tile width, operand mode):
-//   warps 0-3  epilogue: tcgen05.ld of the accumulator (one TMEM lane quarter each), bias+GELU /
-//              column scale / plain, round to bf16, stage through shared memory, coalesced
-//              16-byte stores; rows may be scattered (out[perm[slot]], Algorithm 3 step 6);
-//   warp 4     TMEM allocation and the single thread that issues tcgen05.mma (M=128, N=BN,
+//   warps 0-7  epilogue: tcgen05.ld of the accumulator (warp w reads TMEM lane quarter w % 4 and
+//              column half w / 4), bias+GELU / column scale / plain, round to bf16, stage through
+//              shared memory, coalesced 16-byte stores; rows may be scattered (out[perm[slot]],
+//              Algorithm 3 step 6);
+//   warp 8     TMEM allocation and the single thread that issues tcgen05.mma (M=128, N=BN,
 //              K=16 per instruction) and tcgen05.commit;
-//   warp 5     TMA producer (dense / grouped modes): 128-byte-swizzled A and B tiles;
-//   warps 6-9  gather producers (gather mode): the A rows of fc1 are tokens picked by the routing
+//   warp 9     TMA producer (dense / grouped modes): 128-byte-swizzled A and B tiles;
+//   warps 10-13 gather producers (gather mode): the A rows of fc1 are tokens picked by the routing
 //              permutation, so they are copied row by row with 16-byte cp.async straight into the
 //              swizzled layout (chunk j of row r at r*128 + (j ^ (r & 7))*16), while B comes by TMA.
 // Stages of a shared-memory ring are handed over by mbarriers (full: TMA bytes / cp.async
@@ -25,20 +26,23 @@ namespace cm {
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;
-constexpr int TC_NUM_EPI = 4;
-constexpr int TC_WARP_MMA = 4;
-constexpr int TC_WARP_TMA = 5;
-constexpr int TC_WARP_GATHER = 6;
+constexpr int TC_NUM_EPI = 8;  // two warps per TMEM lane quarter, each on half the columns
+constexpr int TC_WARP_MMA = 8;
+constexpr int TC_WARP_TMA = 9;
+constexpr int TC_WARP_GATHER = 10;
 constexpr int TC_GATHER_THREADS = 128;
+constexpr int TC_THREADS_TMA = 32 * (TC_WARP_TMA + 1);
+constexpr int TC_THREADS_GATHER = 32 * TC_WARP_GATHER + TC_GATHER_THREADS;
 
 template <int BN>
 struct TcCfg {
     static constexpr int A_BYTES = TC_BM * TC_BK * 2;
     static constexpr int B_BYTES = BN * TC_BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES_RAW = (200 * 1024) / STAGE_BYTES;
+    static constexpr int STAGES_RAW = (196 * 1024) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
-    static constexpr int CW = BN < 32 ? BN : 32;      // epilogue columns per TMEM load
+    static constexpr int HALF = BN / 2;               // columns per epilogue warp
+    static constexpr int CW = HALF < 32 ? HALF : 32;  // epilogue columns per TMEM load
     static constexpr int STG_ROW = CW * 2 + 16;       // staging row pitch (bytes)
     static constexpr int STG_BYTES = TC_NUM_EPI * 32 * STG_ROW;
     static constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128
@@ -75,7 +79,7 @@ __device__ __forceinline__ TileInfo decode_tile(const TcGemmArgs& a, int tile, i
 }
 
 template <int BN, int MODE>
-__global__ void __launch_bounds__(MODE == TC_GATHER ? 320 : 192, 1)
+__global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THREADS_TMA, 1)
     tc_gemm_kernel(const __grid_constant__ TcGemmArgs a) {
     using C = TcCfg<BN>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -263,7 +267,8 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? 320 : 192, 1)
         __syncwarp();
     } else if (warp < TC_NUM_EPI) {
         // ------------------------------------------------ epilogue
-        const int q = warp;
+        const int q = warp & 3;
+        const int c_lo = (warp >> 2) * C::HALF;
         unsigned char* wstg = stg + warp * 32 * C::STG_ROW;
         constexpr int LPR = C::CW / 8;  // lanes per staged row (16 bytes each)
         constexpr int RPP = 32 / LPR;   // rows per store pass
@@ -276,11 +281,15 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? 320 : 192, 1)
             const int r = q * 32 + lane;
             int64_t orow = -1;
             if (r < t.rows) orow = (a.epi == TC_EPI_SCATTER) ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
-            for (int c = 0; c < BN; c += C::CW) {
-                uint32_t v[C::CW];
+            for (int c = c_lo; c < c_lo + C::HALF; c += C::CW) {
+                uint32_t v[32];
                 const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
-                CM_TMEM_LD_X16(taddr, v);
-                if constexpr (C::CW == 32) CM_TMEM_LD_X16(taddr + 16, (v + 16));
+                if constexpr (C::CW == 8) {
+                    CM_TMEM_LD_X8(taddr, v);
+                } else {
+                    CM_TMEM_LD_X16(taddr, v);
+                    if constexpr (C::CW == 32) CM_TMEM_LD_X16(taddr + 16, (v + 16));
+                }
                 tmem_wait_ld();
                 float f[C::CW];
 #pragma unroll
@@ -294,8 +303,11 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? 320 : 192, 1)
                         const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
                         for (int h = 0; h < 4; ++h) {
-                            f[j8 * 8 + 2 * h] = gelu_erf(f[j8 * 8 + 2 * h] + bf16_lo(bw[h]));
-                            f[j8 * 8 + 2 * h + 1] = gelu_erf(f[j8 * 8 + 2 * h + 1] + bf16_hi(bw[h]));
+                            const float2 g = gelu_pair_as(
+                                __fadd2_rn(make_float2(f[j8 * 8 + 2 * h], f[j8 * 8 + 2 * h + 1]),
+                                           make_float2(bf16_lo(bw[h]), bf16_hi(bw[h]))));
+                            f[j8 * 8 + 2 * h] = g.x;
+                            f[j8 * 8 + 2 * h + 1] = g.y;
                         }
                     }
                 } else if (a.epi == TC_EPI_SCALE) {
@@ -363,7 +375,7 @@ static cudaError_t launch_one(const TcGemmArgs& a, int num_sms, cudaStream_t s) 
     int64_t tiles = m_tiles * n_tiles;
     const int grid = (int)(tiles < num_sms ? tiles : num_sms);
     if (grid <= 0) return cudaSuccess;
-    tc_gemm_kernel<BN, MODE><<<grid, MODE == TC_GATHER ? 320 : 192, C::SMEM, s>>>(a);
+    tc_gemm_kernel<BN, MODE><<<grid, MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THREADS_TMA, C::SMEM, s>>>(a);
     return cudaGetLastError();
 }
 
