@@ -1,0 +1,85 @@
+"""GPU parity of the 12-sublayer ViT-B stack (100,864 tokens, d = 768, H = 3,072, odd sublayers
+CLEAR-MoE with E = 8, r = 128, even sublayers dense, x_{l+1} = LN(y_l), bf16), through the C ABI.
+
+Every sublayer is checked against the oracle on the GPU's own input to that sublayer, so errors do
+not compound across layers: routing on all tokens (bit-exact outside near ties), the sublayer's
+output on sampled rows (plus the whole smallest expert), and the LayerNorm on sampled rows."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import clearmoe as O
+from paper_2606_28516_gb300 import clearmoe as cm
+
+from gpu_util import check_routing, out_error, sample_rows, tol
+
+pytestmark = pytest.mark.gpu
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to("cuda", torch.bfloat16)
+
+
+def test_vit_base_stack12(workload):
+    import __graft_entry__
+    __graft_entry__.build()
+    S = workload(synth.VIT_BASE_STACK12)
+    sh = S["shape"]
+    T = S["T"]
+    h = cm.clearmoe_layer_create(T, sh.d, sh.H, sh.E, sh.r, cm.BF16)
+    try:
+        x = _dev(S["x"])
+        rng = np.random.default_rng(1)
+        for l, L in enumerate(S["layers"]):
+            W1, b1 = _dev(L["W1"]), _dev(L["b1"])
+            y = torch.empty(T, sh.d, device="cuda", dtype=torch.bfloat16)
+            if L["moe"]:
+                U, Vh, res = _dev(L["U"]), _dev(L["Vh"]), _dev(L["residuals"])
+                Wg, bg = _dev(L["Wg"]), _dev(L["bg"])
+                Sr = torch.from_numpy(L["S"].astype(np.float32)).cuda()
+                cm.clearmoe_ffn_forward(h, x, W1, b1, U, Sr, Vh, res, Wg, bg, y)
+                idx = torch.empty(T, dtype=torch.int32, device="cuda")
+                perm = torch.empty_like(idx)
+                counts = torch.empty(sh.E, dtype=torch.int32, device="cuda")
+                offsets = torch.empty(sh.E + 1, dtype=torch.int32, device="cuda")
+                cm.clearmoe_get_routing(h, idx, counts, offsets, perm)
+            else:
+                cm.clearmoe_dense_ffn_forward(h, x, W1, b1, _dev(L["W2"]), y)
+            x_next = torch.empty_like(y)
+            cm.clearmoe_layer_norm(h, y, x_next)
+            torch.cuda.synchronize()
+            assert cm.clearmoe_layer_status(h) == 0
+            x_in = x.float().cpu().numpy()
+            if L["moe"]:
+                gr = dict(a=idx.cpu().numpy().astype(np.int64), counts=counts.cpu().numpy().astype(np.int64),
+                          offsets=offsets.cpu().numpy().astype(np.int64),
+                          perm=perm.cpu().numpy().astype(np.int64))
+                check_routing(gr, x_in, L["Wg"], L["bg"])
+                rows = sample_rows(gr, T, n=1024, seed=l)
+                want = O.ffn_forward(x_in[rows], L["W1"], L["b1"], L["U"], L["S"], L["Vh"],
+                                     L["residuals"], a=gr["a"][rows], z_bf16=True)
+            else:
+                rows = np.sort(rng.choice(T, 1024, replace=False))
+                want = O.dense_ffn(x_in[rows], L["W1"], L["b1"], L["W2"], z_bf16=True)
+            ridx = torch.from_numpy(rows).cuda()
+            err = out_error(y[ridx], want, "bf16")
+            assert err <= tol("bf16"), f"sublayer {l}: output error {err:.3e}"
+            # x_{l+1} is stored in bf16: compare with the oracle's LayerNorm rounded to bf16,
+            # allowing one bf16 step plus 1e-5 absolute (the GPU's fp32 mean differs from the
+            # float64 one by ~1e-9, which is many ulps of an output that is itself ~1e-7)
+            ln_want = O.stack_next_input(y[ridx].float().cpu().numpy())
+            ln_got = x_next[ridx].float().cpu().numpy().astype(np.float64)
+            _, ex = np.frexp(np.abs(ln_want))
+            ulp = np.ldexp(1.0, ex - 8)
+            bad = np.abs(ln_got - ln_want) > ulp + 1e-5
+            if bad.any():
+                i, j = np.argwhere(bad)[0]
+                yr = y[ridx].float().cpu().numpy().astype(np.float64)[i]
+                raise AssertionError(
+                    f"sublayer {l}: LayerNorm off by > 1 ulp at {bad.sum()} of {bad.size} elements; "
+                    f"first: got {ln_got[i, j]!r} want {ln_want[i, j]!r}; row mean {yr.mean():.6g} "
+                    f"std {yr.std():.6g} max|y| {np.abs(yr).max():.6g}")
+            x = x_next
+    finally:
+        cm.clearmoe_layer_destroy(h)
