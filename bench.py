@@ -130,13 +130,12 @@ class ClockSampler:
                 "samples": len(self.rows)}
 
 
-def oracle_rate(L, budget_s=12.0, chunk=1024, max_tokens=None):
+def oracle_rate(L, budget_s=12.0, chunk=1024, max_tokens=None, warm=True):
     """Oracle tokens/s on row chunks of the workload until budget_s of CPU time is spent."""
-    import numpy as np
     from oracle import clearmoe as O
     s = L["shape"]
-    rt = O.route(L["x"][: min(s.T, 8192)], L["Wg"], L["bg"])  # warm the BLAS threads
-    del rt
+    if warm:  # start the BLAS threads outside the timed part
+        O.route(L["x"][: min(s.T, 8192)], L["Wg"], L["bg"])
     done, t0 = 0, time.perf_counter()
     limit = max_tokens or s.T
     while done < limit:
@@ -175,10 +174,10 @@ def run_reference(args):
     probe, _, _ = oracle_rate(L, budget_s=2.0, chunk=256, max_tokens=512)
     per_step = max(16, min(4096, int(probe * 60.0 / max(1, args.steps + args.warmup))))
     for _ in range(args.warmup):
-        oracle_rate(L, budget_s=1e9, chunk=per_step, max_tokens=per_step)
+        oracle_rate(L, budget_s=1e9, chunk=per_step, max_tokens=per_step, warm=False)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle_rate(L, budget_s=1e9, chunk=per_step, max_tokens=per_step)
+        oracle_rate(L, budget_s=1e9, chunk=per_step, max_tokens=per_step, warm=False)
     el = time.perf_counter() - t0
     value = per_step * args.steps / el
     cores = blas_threads()
@@ -207,7 +206,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="deit_base_bf16", choices=sorted(workloads()))
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--e2e-steps", type=int, default=200)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
@@ -295,24 +294,54 @@ def main():
     dense_ms = [e[0].elapsed_time(e[2]) for e in dev]
     dense_value = s.T / (statistics.mean(dense_ms) / 1e3)
 
-    # end to end through the C ABI with host buffers: H2D of x and D2H of out inside each step
-    x_host = D["x"].cpu().pin_memory()
-    out_host = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    x_dev = torch.empty_like(D["x"])
+    # End to end through the C ABI with host buffers: every step copies its tokens from pinned
+    # host memory and its output back. Steps are pipelined over three streams (copy-in of step
+    # k + 1 and copy-out of step k - 1 overlap the forward of step k), with double buffers.
     Ke = max(1, min(args.e2e_steps, K))
-    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(Ke)]
-    for k in range(Ke + args.warmup):
-        flush.zero_()
-        if k >= args.warmup:
-            e2e_ev[k - args.warmup][0].record(stream)
-        x_dev.copy_(x_host, non_blocking=True)
-        forward(x_dev)
-        out_host.copy_(out, non_blocking=True)
-        if k >= args.warmup:
-            e2e_ev[k - args.warmup][1].record(stream)
+    x_host = D["x"].cpu().pin_memory()
+    out_host = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
+    x_dev = [torch.empty_like(D["x"]) for _ in range(2)]
+    o_dev = [torch.empty_like(out) for _ in range(2)]
+    s_in, s_cmp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    ev = lambda: torch.cuda.Event()
+    x_ready, x_free = [ev(), ev()], [ev(), ev()]
+    o_ready, o_free = [ev(), ev()], [ev(), ev()]
+    e2e_t0, e2e_t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
-    e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_ev)
+
+    def e2e_steps(n, timed):
+        for k in range(n):
+            b = k & 1
+            with torch.cuda.stream(s_in):
+                if k == 0 and timed:
+                    e2e_t0.record(s_in)
+                if k >= 2:
+                    s_in.wait_event(x_free[b])
+                x_dev[b].copy_(x_host, non_blocking=True)
+                x_ready[b].record(s_in)
+            with torch.cuda.stream(s_cmp):
+                s_cmp.wait_event(x_ready[b])
+                if k >= 2:
+                    s_cmp.wait_event(o_free[b])
+                cm.clearmoe_ffn_forward(h, x_dev[b], D["W1"], D["b1"], D["U"], D["S"], D["Vh"],
+                                        D["residuals"], D["Wg"], D["bg"], o_dev[b], stream=s_cmp)
+                x_free[b].record(s_cmp)
+                o_ready[b].record(s_cmp)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(o_ready[b])
+                out_host[b].copy_(o_dev[b], non_blocking=True)
+                o_free[b].record(s_out)
+                if k == n - 1 and timed:
+                    e2e_t1.record(s_out)
+        torch.cuda.synchronize()
+
+    e2e_steps(args.warmup, False)
+    if dist:
+        dist.barrier()
+    e2e_steps(Ke, True)
+    e2e_ms = e2e_t0.elapsed_time(e2e_t1)
+    if not torch.equal(out_host[(Ke - 1) & 1].cuda(), o_dev[(Ke - 1) & 1]):
+        raise RuntimeError("end-to-end output copy mismatch")
     if dist:
         t = torch.tensor([e2e_ms], device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)

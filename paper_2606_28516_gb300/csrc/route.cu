@@ -3,7 +3,10 @@
 //   per-expert histogram, exclusive prefix sum, and the stable permutation perm[slot] = token.
 //
 // One cooperative launch of co-resident CTAs; CTA b owns a contiguous range of `chunk` tokens.
-//   phase 1: stream x once from HBM, router logits and argmax per token, local histogram;
+//   phase 1: stream x once from HBM, router logits and argmax per token, local histogram.
+//            bf16: one CTA per SM; a producer thread copies the CTA's rows, 16 at a time, into a
+//            ring of shared-memory stages with 1-D bulk copies (mbarrier-tracked, so the bytes in
+//            flight cost no registers) and eight consumer warps take one 16-row stage each;
 //   grid-wide wait (bounded, on a monotone arrival counter);
 //   phase 2: each CTA sums the histograms of the CTAs before it and writes its tokens' slots in
 //            token order (ranks from warp match masks), which makes the sort stable.
@@ -16,8 +19,11 @@
 
 namespace cm {
 
-constexpr int RT_THREADS = 256;
-constexpr int RT_WARPS = RT_THREADS / 32;
+constexpr int RT_THREADS = 256;                 // fp32 router: 8 warps
+constexpr int RT_BF16_THREADS = 288;            // bf16 router: 8 consumer warps + 1 producer warp
+constexpr int RT_MAX_WARPS = RT_BF16_THREADS / 32;
+constexpr int RT_STAGE_ROWS = 16;               // rows per ring stage (one MMA row group)
+constexpr int RT_RING_BYTES = 192 * 1024;       // shared-memory ring budget (bf16 router)
 
 __device__ __forceinline__ uint4 ldg_nc_v4(const uint4* p) {
     uint4 v;
@@ -55,18 +61,47 @@ __host__ __device__ inline size_t frag_bytes(int dtype, int d, int E) {
     if (dtype == CLEARMOE_BF16) return (size_t)((E + 7) / 8) * (d / 32) * 32 * 16;
     return (size_t)E * d * 4;
 }
-static size_t route_smem(int dtype, int d, int E, int chunk) {
-    return ((frag_bytes(dtype, d, E) + 15) & ~(size_t)15) + (size_t)((chunk + 15) & ~15);
+
+// Dynamic shared memory: [router weights] [bf16: ring of S stages] [bf16: 2 S mbarriers]. The
+// chosen expert of each row goes to idx in global memory and is read back from there (the CTA's
+// own writes, visible block-wide after __syncthreads), so the footprint does not grow with T.
+// The ring has one slot per consumer warp (S = 8, or 4 when eight stages do not fit): consumer
+// warp w alone reads slot w, for stages w, w + S, ..., so each of its mbarrier waits is for the
+// phase right after the one it last consumed (a parity wait cannot tell phases two apart).
+struct RouteLayout {
+    size_t ring, bars, total;
+    int S, stage_bytes;
+};
+__host__ __device__ inline RouteLayout route_layout(int dtype, int d, int E) {
+    RouteLayout L;
+    const size_t frag = (frag_bytes(dtype, d, E) + 127) & ~(size_t)127;
+    L.stage_bytes = RT_STAGE_ROWS * d * 2;
+    L.S = 0;
+    L.ring = frag;
+    if (dtype == CLEARMOE_BF16) L.S = (8 * L.stage_bytes <= RT_RING_BYTES) ? 8 : 4;
+    L.bars = (L.ring + (size_t)L.S * L.stage_bytes + 15) & ~(size_t)15;
+    L.total = L.bars + (size_t)2 * L.S * 8;
+    return L;
+}
+static size_t route_smem(int dtype, int d, int E) { return route_layout(dtype, d, E).total; }
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
 }
 
 template <bool BF16>
-__global__ void __launch_bounds__(RT_THREADS) route_kernel(const RouteArgs a, const int chunk) {
-    extern __shared__ __align__(16) unsigned char smem[];
+__global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_kernel(const RouteArgs a, const int chunk) {
+    constexpr int NTHREADS = BF16 ? RT_BF16_THREADS : RT_THREADS;
+    constexpr int NWARPS = NTHREADS / 32;
+    constexpr int NCONS_MAX = 8;  // warps computing logits (bf16: the first S warps)
+    extern __shared__ __align__(128) unsigned char smem[];
     __shared__ int s_count[CM_MAX_E];
     __shared__ int s_base[CM_MAX_E];
     __shared__ int s_tot[CM_MAX_E];
     __shared__ int s_run[CM_MAX_E];
-    __shared__ int s_wc[RT_WARPS][CM_MAX_E];
+    __shared__ int s_wc[RT_MAX_WARPS][CM_MAX_E];
     __shared__ int s_abort;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -75,18 +110,33 @@ __global__ void __launch_bounds__(RT_THREADS) route_kernel(const RouteArgs a, co
     const int nrows = (int)max((int64_t)0, min((int64_t)chunk, a.T - row0));
     const int nchunk = d / 32;
     const int NT = (E + 7) / 8;
-    uint8_t* sidx = smem + ((frag_bytes(BF16 ? CLEARMOE_BF16 : CLEARMOE_F32, d, E) + 15) & ~15);
+    const RouteLayout lay = route_layout(BF16 ? CLEARMOE_BF16 : CLEARMOE_F32, d, E);
+    const int32_t* my_idx = a.idx + row0;  // this CTA's rows, written in phase 1
 
     if (tid < CM_MAX_E) s_count[tid] = 0;
     if (tid == 0) s_abort = 0;
 
     // ---------------- phase 1: router logits + argmax for this CTA's rows
     if constexpr (BF16) {
+        const int S = lay.S, SB = lay.stage_bytes;
+        const uint32_t ring = smem_u32(smem + lay.ring);
+        const uint32_t bar0 = smem_u32(smem + lay.bars);
+        auto full_bar = [&](int s) { return bar0 + 8u * s; };
+        auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
+        const int nstages = (nrows + RT_STAGE_ROWS - 1) / RT_STAGE_ROWS;
+        volatile int* abort_flag = &s_abort;
+        if (tid == 0) {
+            for (int s = 0; s < S; ++s) {
+                mbar_init(full_bar(s), 1);
+                mbar_init(empty_bar(s), 1);
+            }
+            mbar_fence_init();
+        }
         // B fragments of W_g: [n-tile][32-column chunk][lane] -> 8 consecutive bf16 of row
         // nt*8 + lane/4, columns chunk*32 + (lane%4)*8.
         uint4* bfrag = reinterpret_cast<uint4*>(smem);
         const uint16_t* W = static_cast<const uint16_t*>(a.Wg);
-        for (int i = tid; i < NT * nchunk * 32; i += RT_THREADS) {
+        for (int i = tid; i < NT * nchunk * 32; i += NTHREADS) {
             const int l = i & 31, c = (i >> 5) % nchunk, nt = (i >> 5) / nchunk;
             const int e = nt * 8 + (l >> 2);
             uint4 v = make_uint4(0, 0, 0, 0);
@@ -94,87 +144,95 @@ __global__ void __launch_bounds__(RT_THREADS) route_kernel(const RouteArgs a, co
             bfrag[i] = v;
         }
         __syncthreads();
-        const uint16_t* bgp = static_cast<const uint16_t*>(a.bg);
-        const int g = lane >> 2, tig = lane & 3;
-        const int ngroups = (nrows + 15) / 16;
-        const uint4 zero = make_uint4(0, 0, 0, 0);
-        for (int grp = warp; grp < ngroups; grp += RT_WARPS) {
-            const int iA = grp * 16 + g, iB = iA + 8;
-            const bool vA = iA < nrows, vB = iB < nrows;
-            const uint4* pA = reinterpret_cast<const uint4*>(
-                                  static_cast<const uint16_t*>(a.x) + (row0 + (vA ? iA : 0)) * d) + tig;
-            const uint4* pB = reinterpret_cast<const uint4*>(
-                                  static_cast<const uint16_t*>(a.x) + (row0 + (vB ? iB : 0)) * d) + tig;
-            float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-            for (int c0 = 0; c0 < nchunk; c0 += 8) {
-                uint4 xa[8], xb[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int c = c0 + i;
-                    xa[i] = (vA && c < nchunk) ? ldg_nc_v4(pA + 4 * c) : zero;
-                    xb[i] = (vB && c < nchunk) ? ldg_nc_v4(pB + 4 * c) : zero;
+        if (warp == NCONS_MAX) {
+            // ---- producer: stage k = rows [16 k, 16 k + 16) of this CTA, ring slot k % S
+            if (lane == 0) {
+                const unsigned char* xb = static_cast<const unsigned char*>(a.x) + row0 * d * 2;
+                int k = 0;
+                for (; k < nstages; ++k) {
+                    const int s = k % S;
+                    if (!mbar_wait(empty_bar(s), ((k / S) & 1) ^ 1, abort_flag, a.status, (uint64_t)a.wait_limit_ns))
+                        break;
+                    const int rows = min(RT_STAGE_ROWS, nrows - k * RT_STAGE_ROWS);
+                    const uint32_t bytes = (uint32_t)rows * d * 2;
+                    mbar_arrive_expect_tx(full_bar(s), bytes);
+                    bulk_g2s(ring + s * SB, xb + (size_t)k * SB, bytes, full_bar(s));
                 }
+                if (k < nstages) {  // gave up: let the copies in flight land before moving on
+                    for (int j = max(0, k - S); j < k; ++j)
+                        mbar_wait(full_bar(j % S), (j / S) & 1, nullptr, a.status, 10000000ull);
+                }
+            }
+        } else if (warp < S) {
+            // ---- consumers: warp w owns slot w and takes stages w, w + S, w + 2 S, ...
+            const uint16_t* bgp = static_cast<const uint16_t*>(a.bg);
+            const int g = lane >> 2, tig = lane & 3;
+            const uint4 zero = make_uint4(0, 0, 0, 0);
+            for (int k = warp; k < nstages; k += S) {
+                const int s = warp;
+                if (!mbar_wait(full_bar(s), (k / S) & 1, abort_flag, a.status, (uint64_t)a.wait_limit_ns)) break;
+                const int rows = min(RT_STAGE_ROWS, nrows - k * RT_STAGE_ROWS);
+                const bool vA = g < rows, vB = g + 8 < rows;
+                const unsigned char* st = smem + lay.ring + (size_t)s * SB;
+                const uint4* pA = reinterpret_cast<const uint4*>(st + (size_t)g * d * 2) + tig;
+                const uint4* pB = reinterpret_cast<const uint4*>(st + (size_t)(g + 8) * d * 2) + tig;
+                float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+                for (int c = 0; c < nchunk; ++c) {
+                    const uint4 xa = vA ? pA[4 * c] : zero;
+                    const uint4 xb = vB ? pB[4 * c] : zero;
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int c = c0 + i;
-                    if (c < nchunk) {
-#pragma unroll
-                        for (int nt = 0; nt < 2; ++nt) {
-                            if (nt < NT) {
-                                const uint4 w = bfrag[(nt * nchunk + c) * 32 + lane];
-                                mma_bf16_16816(acc[nt], xa[i].x, xb[i].x, xa[i].y, xb[i].y, w.x, w.y);
-                                mma_bf16_16816(acc[nt], xa[i].z, xb[i].z, xa[i].w, xb[i].w, w.z, w.w);
-                            }
+                    for (int nt = 0; nt < 2; ++nt) {
+                        if (nt < NT) {
+                            const uint4 w = bfrag[(nt * nchunk + c) * 32 + lane];
+                            mma_bf16_16816(acc[nt], xa.x, xb.x, xa.y, xb.y, w.x, w.y);
+                            mma_bf16_16816(acc[nt], xa.z, xb.z, xa.w, xb.w, w.z, w.w);
                         }
                     }
                 }
-            }
-            // D fragment: acc[nt][0..1] = row g, experts nt*8 + 2*tig + {0,1}; [2..3] = row g+8
-            float bA = -INFINITY, bB = -INFINITY;
-            int eA = 0x7fffffff, eB = 0x7fffffff;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty_bar(s));  // the stage's rows are in registers now
+                // D fragment: acc[nt][0..1] = row g, experts nt*8 + 2*tig + {0,1}; [2..3] = row g+8
+                float bA = -INFINITY, bB = -INFINITY;
+                int eA = 0x7fffffff, eB = 0x7fffffff;
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt) {
+                for (int nt = 0; nt < 2; ++nt) {
 #pragma unroll
-                for (int j = 0; j < 2; ++j) {
-                    const int e = nt * 8 + 2 * tig + j;
-                    if (nt < NT && e < E) {
-                        const uint16_t bb = bgp[e];
-                        const float bias = __uint_as_float((uint32_t)bb << 16);
-                        arg_better(bA, eA, acc[nt][j] + bias, e);
-                        arg_better(bB, eB, acc[nt][2 + j] + bias, e);
+                    for (int j = 0; j < 2; ++j) {
+                        const int e = nt * 8 + 2 * tig + j;
+                        if (nt < NT && e < E) {
+                            const uint16_t bb = bgp[e];
+                            const float bias = __uint_as_float((uint32_t)bb << 16);
+                            arg_better(bA, eA, acc[nt][j] + bias, e);
+                            arg_better(bB, eB, acc[nt][2 + j] + bias, e);
+                        }
                     }
                 }
-            }
 #pragma unroll
-            for (int off = 1; off <= 2; off <<= 1) {
-                const float ovA = __shfl_xor_sync(0xffffffffu, bA, off);
-                const int oeA = __shfl_xor_sync(0xffffffffu, eA, off);
-                const float ovB = __shfl_xor_sync(0xffffffffu, bB, off);
-                const int oeB = __shfl_xor_sync(0xffffffffu, eB, off);
-                arg_better(bA, eA, ovA, oeA);
-                arg_better(bB, eB, ovB, oeB);
-            }
-            if (eA > E - 1) eA = 0;  // only reachable with non-finite logits
-            if (eB > E - 1) eB = 0;
-            if (tig == 0) {
-                if (vA) {
-                    a.idx[row0 + iA] = eA;
-                    sidx[iA] = (uint8_t)eA;
+                for (int off = 1; off <= 2; off <<= 1) {
+                    const float ovA = __shfl_xor_sync(0xffffffffu, bA, off);
+                    const int oeA = __shfl_xor_sync(0xffffffffu, eA, off);
+                    const float ovB = __shfl_xor_sync(0xffffffffu, bB, off);
+                    const int oeB = __shfl_xor_sync(0xffffffffu, eB, off);
+                    arg_better(bA, eA, ovA, oeA);
+                    arg_better(bB, eB, ovB, oeB);
                 }
-                if (vB) {
-                    a.idx[row0 + iB] = eB;
-                    sidx[iB] = (uint8_t)eB;
+                if (eA > E - 1) eA = 0;  // only reachable with non-finite logits
+                if (eB > E - 1) eB = 0;
+                if (tig == 0) {
+                    const int iA = k * RT_STAGE_ROWS + g, iB = iA + 8;
+                    if (vA) a.idx[row0 + iA] = eA;
+                    if (vB) a.idx[row0 + iB] = eB;
                 }
             }
         }
     } else {
         float* Wf = reinterpret_cast<float*>(smem);
         const float* W = static_cast<const float*>(a.Wg);
-        for (int i = tid; i < E * d; i += RT_THREADS) Wf[i] = W[i];
+        for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = W[i];
         __syncthreads();
         const float* bgp = static_cast<const float*>(a.bg);
         const float* X = static_cast<const float*>(a.x);
-        for (int i = warp; i < nrows; i += RT_WARPS) {
+        for (int i = warp; i < nrows; i += NWARPS) {
             const float* xr = X + (row0 + i) * d;
             float acc[CM_MAX_E];
 #pragma unroll
@@ -197,16 +255,13 @@ __global__ void __launch_bounds__(RT_THREADS) route_kernel(const RouteArgs a, co
                 }
             }
             if (be > E - 1) be = 0;
-            if (lane == 0) {
-                a.idx[row0 + i] = be;
-                sidx[i] = (uint8_t)be;
-            }
+            if (lane == 0) a.idx[row0 + i] = be;
         }
     }
     __syncthreads();
 
     // ---------------- local histogram, published for the other CTAs
-    for (int i = tid; i < nrows; i += RT_THREADS) atomicAdd(&s_count[sidx[i]], 1);
+    for (int i = tid; i < nrows; i += NTHREADS) atomicAdd(&s_count[my_idx[i]], 1);
     __syncthreads();
     if (tid < E) a.cta_counts[(size_t)blockIdx.x * CM_MAX_E + tid] = s_count[tid];
     __threadfence();
@@ -229,7 +284,7 @@ __global__ void __launch_bounds__(RT_THREADS) route_kernel(const RouteArgs a, co
     if (s_abort) return;
 
     // ---------------- phase 2: global offsets, then this CTA's slots in token order
-    for (int e = warp; e < E; e += RT_WARPS) {
+    for (int e = warp; e < E; e += NWARPS) {
         int before = 0, total = 0;
         for (int b = lane; b < (int)gridDim.x; b += 32) {
             const int c = __ldcg(&a.cta_counts[(size_t)b * CM_MAX_E + e]);
@@ -262,19 +317,19 @@ __global__ void __launch_bounds__(RT_THREADS) route_kernel(const RouteArgs a, co
         if (blockIdx.x == 0) a.offsets[E] = run;
     }
     const unsigned lt = (1u << lane) - 1u;
-    for (int i0 = 0; i0 < nrows; i0 += RT_THREADS) {
-        if (tid < RT_WARPS * CM_MAX_E) (&s_wc[0][0])[tid] = 0;
+    for (int i0 = 0; i0 < nrows; i0 += NTHREADS) {
+        if (tid < NWARPS * CM_MAX_E) (&s_wc[0][0])[tid] = 0;
         __syncthreads();
         const int i = i0 + tid;
         const bool valid = i < nrows;
-        const int e = valid ? (int)sidx[i] : CM_MAX_E + 1;
+        const int e = valid ? (int)my_idx[i] : CM_MAX_E + 1;
         const unsigned same = __match_any_sync(0xffffffffu, e);
         const int rank = __popc(same & lt);
         if (valid && rank == 0) s_wc[warp][e] = __popc(same);
         __syncthreads();
         if (tid < E) {
             int run = s_run[tid];
-            for (int w = 0; w < RT_WARPS; ++w) {
+            for (int w = 0; w < NWARPS; ++w) {
                 const int c = s_wc[w][tid];
                 s_wc[w][tid] = run;
                 run += c;
@@ -292,19 +347,22 @@ int route_max_ctas(int num_sms, int, int, int) { return num_sms * 8; }
 int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* chunk) {
     const bool bf16 = dtype == CLEARMOE_BF16;
     int occ = 0;
-    int64_t want = (int64_t)num_sms * 2;
+    int64_t want = (int64_t)num_sms * (bf16 ? 1 : 2);  // bf16: one CTA per SM owns the ring
     int64_t ch = ((T + want - 1) / want + 15) / 16 * 16;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaFuncSetAttribute((const void*)route_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
-        cudaFuncSetAttribute((const void*)route_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+            if (cudaFuncSetAttribute((const void*)route_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 220 * 1024) != cudaSuccess ||
+            cudaFuncSetAttribute((const void*)route_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 220 * 1024) != cudaSuccess)
+            return -1;
         attr_set = true;
     }
+    const size_t smem = route_smem(dtype, d, E);
     for (int iter = 0; iter < 4; ++iter) {
-        const size_t smem = route_smem(dtype, d, E, (int)ch);
         cudaError_t err = cudaOccupancyMaxActiveBlocksPerMultiprocessorWithFlags(
             &occ, bf16 ? (const void*)route_kernel<true> : (const void*)route_kernel<false>,
-            RT_THREADS, smem, cudaOccupancyDefault);
+            bf16 ? RT_BF16_THREADS : RT_THREADS, smem, cudaOccupancyDefault);
         if (err != cudaSuccess) return -1;
         if (occ <= 0) return -2;
         const int64_t maxg = (int64_t)occ * num_sms;
@@ -320,15 +378,10 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
 
 cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s) {
     const bool bf16 = a.dtype == CLEARMOE_BF16;
-    const size_t smem = route_smem(a.dtype, a.d, a.E, chunk);
-    const void* fn = bf16 ? (const void*)route_kernel<true> : (const void*)route_kernel<false>;
-    if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-    }
+    const size_t smem = route_smem(a.dtype, a.d, a.E);  // the attribute is set by route_grid
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(RT_THREADS);
+    cfg.blockDim = dim3(bf16 ? RT_BF16_THREADS : RT_THREADS);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
