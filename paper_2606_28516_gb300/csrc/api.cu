@@ -20,9 +20,8 @@ struct clearmoe_layer {
     int32_t* counts;    // [CM_MAX_E]
     int32_t* offsets;   // [CM_MAX_E + 1]
     int32_t* cta_counts;  // [route_max_ctas x CM_MAX_E]
-    unsigned long long* barrier;
+    unsigned int* barrier;  // the routing kernel's grid barrier: arrivals, generation
     int32_t* status;
-    unsigned long long barrier_total;
     int64_t wait_limit_ns;
     int32_t phantom;
     int64_t last_T;
@@ -76,12 +75,11 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
     a.offsets = L->offsets;
     a.cta_counts = L->cta_counts;
     a.barrier = L->barrier;
-    a.target = L->barrier_total + (unsigned long long)grid + (unsigned long long)L->phantom;
+    a.arrivals = (unsigned int)grid + (unsigned int)L->phantom;
     a.wait_limit_ns = L->wait_limit_ns;
     a.status = L->status;
     const int rc = cuda_fail(cm::launch_route(a, grid, chunk, s));
     if (rc == CLEARMOE_OK) {
-        L->barrier_total += (unsigned long long)grid;
         L->last_T = T;
         L->last_E = E;
     }
@@ -429,9 +427,8 @@ int clearmoe_layer_status(clearmoe_layer* L) {
     if (st != 0) {
         if (cudaMemset(L->status, 0, 4) != cudaSuccess) return CLEARMOE_ECUDA;
         if (st == CLEARMOE_ETIMEOUT) {
-            // arrivals of a launch that gave up no longer match the host's count: start afresh
+            // a launch that gave up left arrivals behind: start the grid barrier afresh
             if (cudaMemset(L->barrier, 0, 8) != cudaSuccess) return CLEARMOE_ECUDA;
-            L->barrier_total = 0;
         }
         if (cudaDeviceSynchronize() != cudaSuccess) return CLEARMOE_ECUDA;
     }

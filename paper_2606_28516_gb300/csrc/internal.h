@@ -20,8 +20,8 @@ struct RouteArgs {
     int32_t* counts;
     int32_t* offsets;
     int32_t* cta_counts;           // [max_route_ctas x CM_MAX_E] scratch
-    unsigned long long* barrier;   // monotone arrival counter
-    unsigned long long target;     // counter value that releases this launch
+    unsigned int* barrier;         // [0] arrivals, [1] generation: a self-resetting grid barrier
+    unsigned int arrivals;         // arrivals that release the wait (the grid; more in fault tests)
     int64_t wait_limit_ns;
     int32_t* status;
 };

@@ -15,8 +15,8 @@
 
 namespace {
 
-// Scratch layout (int32 words): [0, 2) arrival counter (uint64), [2] status word used when the
-// caller passes no status pointer, [16, 16 + MAX_CTAS * CM_MAX_E) per-CTA histograms.
+// Scratch layout (int32 words): [0, 2) the grid barrier (arrivals, generation), [2] status word
+// used when the caller passes no status pointer, [16, 16 + MAX_CTAS * CM_MAX_E) per-CTA histograms.
 constexpr int kNoallocMaxCtas = 1024;
 constexpr int kHistOffset = 16;
 constexpr int kScratchWords = kHistOffset + kNoallocMaxCtas * CM_MAX_E;  // 65,600 bytes
@@ -84,8 +84,8 @@ extern "C" int clearmoe_route_noalloc(const void* x, int64_t T, int32_t d, int32
     if (grid > kNoallocMaxCtas) return CLEARMOE_EUNSUPPORTED;  // beyond the scratch's capacity
 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    // The array keeps the previous call's contents: the arrival counter and the spare status
-    // word must start at zero (the histograms are fully rewritten before they are read).
+    // The array keeps the previous call's contents: the grid barrier and the spare status word
+    // are cleared (the histograms are fully rewritten before they are read).
     if (cudaMemsetAsync(scratch, 0, kHistOffset * sizeof(int32_t), s) != cudaSuccess ||
         (status && cudaMemsetAsync(status, 0, sizeof(int32_t), s) != cudaSuccess)) {
         (void)cudaGetLastError();
@@ -104,8 +104,8 @@ extern "C" int clearmoe_route_noalloc(const void* x, int64_t T, int32_t d, int32
     a.counts = counts;
     a.offsets = offsets;
     a.cta_counts = scratch + kHistOffset;
-    a.barrier = reinterpret_cast<unsigned long long*>(scratch);
-    a.target = (unsigned long long)grid;
+    a.barrier = reinterpret_cast<unsigned int*>(scratch);
+    a.arrivals = (unsigned int)grid;
     a.wait_limit_ns = 1000000000LL;
     a.status = status ? status : scratch + 2;
     const cudaError_t e = cm::launch_route(a, grid, chunk, s);

@@ -14,6 +14,8 @@
 // straight from registers: the 16-byte loads of x are coalesced, and the K order of each
 // fragment is permuted identically for x and W_g, which leaves every dot product unchanged.
 // fp32 tokens: fp32 FMA on the CUDA cores (an fp32 router decision needs fp32 products).
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -43,12 +45,6 @@ __device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint3
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
-    unsigned long long v;
-    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
-    return v;
-}
-
 // better (value, index) with the lower index winning exact ties
 __device__ __forceinline__ void arg_better(float& bv, int& be, float v, int e) {
     if (v > bv || (v == bv && e < be)) {
@@ -69,10 +65,12 @@ __host__ __device__ inline size_t frag_bytes(int dtype, int d, int E) {
 // warp w alone reads slot w, for stages w, w + S, ..., so each of its mbarrier waits is for the
 // phase right after the one it last consumed (a parity wait cannot tell phases two apart).
 struct RouteLayout {
-    size_t ring, bars, total;
+    size_t ring, bars, sidx, total;
     int S, stage_bytes;
+    bool sidx_in_smem;
 };
-__host__ __device__ inline RouteLayout route_layout(int dtype, int d, int E) {
+constexpr size_t RT_SMEM_MAX = 220 * 1024;
+__host__ __device__ inline RouteLayout route_layout(int dtype, int d, int E, int chunk) {
     RouteLayout L;
     const size_t frag = (frag_bytes(dtype, d, E) + 127) & ~(size_t)127;
     L.stage_bytes = RT_STAGE_ROWS * d * 2;
@@ -80,10 +78,13 @@ __host__ __device__ inline RouteLayout route_layout(int dtype, int d, int E) {
     L.ring = frag;
     if (dtype == CLEARMOE_BF16) L.S = (8 * L.stage_bytes <= RT_RING_BYTES) ? 8 : 4;
     L.bars = (L.ring + (size_t)L.S * L.stage_bytes + 15) & ~(size_t)15;
-    L.total = L.bars + (size_t)2 * L.S * 8;
+    L.sidx = L.bars + (size_t)2 * L.S * 8;
+    // expert ids of the CTA's rows: in shared memory when they fit, else read back from idx
+    L.sidx_in_smem = L.sidx + (size_t)chunk <= RT_SMEM_MAX;
+    L.total = L.sidx + (L.sidx_in_smem ? (size_t)chunk : 0);
     return L;
 }
-static size_t route_smem(int dtype, int d, int E) { return route_layout(dtype, d, E).total; }
+static size_t route_smem(int dtype, int d, int E, int chunk) { return route_layout(dtype, d, E, chunk).total; }
 
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
@@ -110,8 +111,14 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     const int nrows = (int)max((int64_t)0, min((int64_t)chunk, a.T - row0));
     const int nchunk = d / 32;
     const int NT = (E + 7) / 8;
-    const RouteLayout lay = route_layout(BF16 ? CLEARMOE_BF16 : CLEARMOE_F32, d, E);
-    const int32_t* my_idx = a.idx + row0;  // this CTA's rows, written in phase 1
+    const RouteLayout lay = route_layout(BF16 ? CLEARMOE_BF16 : CLEARMOE_F32, d, E, chunk);
+    uint8_t* sidx = lay.sidx_in_smem ? smem + lay.sidx : nullptr;
+    auto expert_of = [&](int i) -> int { return sidx ? (int)sidx[i] : __ldcg(a.idx + row0 + i); };
+    auto record = [&](int i, int e) {  // phase 1 result of row i: idx, local id copy, histogram
+        a.idx[row0 + i] = e;
+        if (sidx) sidx[i] = (uint8_t)e;
+        atomicAdd(&s_count[e], 1);
+    };
 
     if (tid < CM_MAX_E) s_count[tid] = 0;
     if (tid == 0) s_abort = 0;
@@ -220,8 +227,8 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 if (eB > E - 1) eB = 0;
                 if (tig == 0) {
                     const int iA = k * RT_STAGE_ROWS + g, iB = iA + 8;
-                    if (vA) a.idx[row0 + iA] = eA;
-                    if (vB) a.idx[row0 + iB] = eB;
+                    if (vA) record(iA, eA);
+                    if (vB) record(iB, eB);
                 }
             }
         }
@@ -255,29 +262,38 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 }
             }
             if (be > E - 1) be = 0;
-            if (lane == 0) a.idx[row0 + i] = be;
+            if (lane == 0) record(i, be);
         }
     }
     __syncthreads();
 
-    // ---------------- local histogram, published for the other CTAs
-    for (int i = tid; i < nrows; i += NTHREADS) atomicAdd(&s_count[my_idx[i]], 1);
-    __syncthreads();
-    if (tid < E) a.cta_counts[(size_t)blockIdx.x * CM_MAX_E + tid] = s_count[tid];
-    __threadfence();
-    __syncthreads();
+    // ---------------- the local histogram (built in phase 1), published for the other CTAs by the
+    // thread that arrives at the grid barrier
 
-    // ---------------- grid-wide wait (bounded)
+    // ---------------- grid-wide wait (bounded), self-resetting: the last of `arrivals` CTAs zeroes
+    // the arrival count and bumps the generation that the others wait on, so nothing carries over
+    // to the next launch and the host keeps no barrier state.
     if (tid == 0) {
-        atomicAdd(a.barrier, 1ULL);
-        const uint64_t t0 = globaltimer();
-        while (ld_acquire_u64(a.barrier) < a.target) {
-            if (globaltimer() - t0 > (uint64_t)a.wait_limit_ns) {
-                s_abort = 1;
-                set_status(a.status, CLEARMOE_ETIMEOUT);
-                break;
+        unsigned int* arrived = a.barrier;
+        unsigned int* generation = a.barrier + 1;
+        for (int e = 0; e < E; ++e) a.cta_counts[(size_t)blockIdx.x * CM_MAX_E + e] = s_count[e];
+        const unsigned int gen0 = ld_acquire_u32(generation);
+        __threadfence();  // the histogram is visible before this CTA's arrival
+        unsigned int prev;
+        asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(prev) : "l"(arrived) : "memory");
+        if (prev == a.arrivals - 1) {
+            st_release_u32(generation, gen0 + 1);  // release everyone, then reset for the next launch
+            atomicExch(arrived, 0u);
+        } else {
+            const uint64_t t0 = globaltimer();
+            while (ld_acquire_u32(generation) == gen0) {
+                if (globaltimer() - t0 > (uint64_t)a.wait_limit_ns) {
+                    s_abort = 1;
+                    set_status(a.status, CLEARMOE_ETIMEOUT);
+                    break;
+                }
+                __nanosleep(64);
             }
-            __nanosleep(64);
         }
     }
     __syncthreads();
@@ -322,7 +338,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         __syncthreads();
         const int i = i0 + tid;
         const bool valid = i < nrows;
-        const int e = valid ? (int)my_idx[i] : CM_MAX_E + 1;
+        const int e = valid ? expert_of(i) : CM_MAX_E + 1;
         const unsigned same = __match_any_sync(0xffffffffu, e);
         const int rank = __popc(same & lt);
         if (valid && rank == 0) s_wc[warp][e] = __popc(same);
@@ -349,6 +365,8 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
     int occ = 0;
     int64_t want = (int64_t)num_sms * (bf16 ? 1 : 2);  // bf16: one CTA per SM owns the ring
     int64_t ch = ((T + want - 1) / want + 15) / 16 * 16;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
     static bool attr_set = false;
     if (!attr_set) {
             if (cudaFuncSetAttribute((const void*)route_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -358,12 +376,21 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
             return -1;
         attr_set = true;
     }
-    const size_t smem = route_smem(dtype, d, E);
+    // occupancy queries are cached: (dtype, d, E, shared-memory bytes) -> CTAs per SM
+    static struct { int dtype, d, E; size_t smem; int occ; } cache[32];
+    static int ncache = 0;
     for (int iter = 0; iter < 4; ++iter) {
-        cudaError_t err = cudaOccupancyMaxActiveBlocksPerMultiprocessorWithFlags(
-            &occ, bf16 ? (const void*)route_kernel<true> : (const void*)route_kernel<false>,
-            bf16 ? RT_BF16_THREADS : RT_THREADS, smem, cudaOccupancyDefault);
-        if (err != cudaSuccess) return -1;
+        const size_t smem = route_smem(dtype, d, E, (int)ch);
+        occ = -1;
+        for (int i = 0; i < ncache; ++i)
+            if (cache[i].dtype == dtype && cache[i].d == d && cache[i].E == E && cache[i].smem == smem) occ = cache[i].occ;
+        if (occ < 0) {
+            cudaError_t err = cudaOccupancyMaxActiveBlocksPerMultiprocessorWithFlags(
+                &occ, bf16 ? (const void*)route_kernel<true> : (const void*)route_kernel<false>,
+                bf16 ? RT_BF16_THREADS : RT_THREADS, smem, cudaOccupancyDefault);
+            if (err != cudaSuccess) return -1;
+            if (ncache < 32) cache[ncache++] = {dtype, d, E, smem, occ};
+        }
         if (occ <= 0) return -2;
         const int64_t maxg = (int64_t)occ * num_sms;
         if (want <= maxg) break;
@@ -378,7 +405,7 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
 
 cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s) {
     const bool bf16 = a.dtype == CLEARMOE_BF16;
-    const size_t smem = route_smem(a.dtype, a.d, a.E);  // the attribute is set by route_grid
+    const size_t smem = route_smem(a.dtype, a.d, a.E, chunk);  // the attribute is set by route_grid
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(bf16 ? RT_BF16_THREADS : RT_THREADS);
