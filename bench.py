@@ -37,9 +37,15 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 STAGES = ("route", "fc1_gelu", "basis", "grouped")
 KERNEL_OF_STAGE = {"route": "route_kernel", "fc1_gelu": "tc_gemm_kernel<256, gather>",
                    "basis": "tc_gemm_kernel<128, dense>", "grouped": "tc_gemm_kernel<256, grouped>"}
-# DRAM traffic per launch from the committed ncu capture (profiles/), with the hash of the kernel
-# source it was taken on; a different hash means the kernel changed and the figure is void.
-TRAFFIC = {}
+# DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from the committed ncu
+# capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel sources
+# it was taken on; a different hash means the kernels changed and the figure is void.
+TRAFFIC = {
+    "route": {"bytes": 78.453760e6, "src": "669263211c688d5d"},
+    "fc1_gelu": {"bytes": 337.098752e6, "src": "669263211c688d5d"},
+    "basis": {"bytes": 321.049856e6, "src": "669263211c688d5d"},
+    "grouped": {"bytes": 423.497728e6, "src": "669263211c688d5d"},
+}
 
 
 def workloads():
@@ -378,6 +384,10 @@ def main():
             tf = work[st]["flops"] / d_s / 1e12
             per_stage[st] = {"us": avg[st] * 1e3, "TFLOP_s": tf,
                              "tensor_frac": tf / pk["bf16_tflops_sustained"]}
+
+    for st in STAGES:  # per-kernel DRAM traffic where the committed capture still applies
+        t = TRAFFIC.get(st)
+        per_stage[st]["traffic"] = t["bytes"] if t and t["src"] == source_hash() else None
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
