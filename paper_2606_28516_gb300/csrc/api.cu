@@ -302,11 +302,14 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     std::memset(&g3, 0, sizeof(g3));
     g3.status = L->status;
     g3.wait_limit_ns = L->wait_limit_ns;
-    if (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, bn3) ||
+    // The 2-SM kernel loads half of each 256-column B tile per CTA of the pair: 128-row boxes.
+    const bool pair3 = cm::tc2_supported(cm::TC_GROUPED, d);
+    const int box3 = pair3 ? 128 : bn3;
+    if (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, box3) ||
         encode_tmap_bf16(&g3.tmA1, L->z, T, H, 128))
         return CLEARMOE_ECUDA;
     for (int e = 0; e < E; ++e)
-        if (encode_tmap_bf16(&g3.tmB1[e], residual_e[e], d, H, bn3)) return CLEARMOE_ECUDA;
+        if (encode_tmap_bf16(&g3.tmB1[e], residual_e[e], d, H, box3)) return CLEARMOE_ECUDA;
     g3.mode = cm::TC_GROUPED;
     g3.epi = cm::TC_EPI_SCATTER;
     g3.M = T;
@@ -318,7 +321,12 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g3.rows = L->perm;
     g3.C = out;
     g3.ldc = d;
-    rc = cuda_fail(cm::launch_tc_gemm(g3, L->num_sms, s));
+    if (pair3) {
+        g3.tmem_cols = 512;
+        rc = cuda_fail(cm::launch_tc_gemm2(g3, L->num_sms, s));
+    } else {
+        rc = cuda_fail(cm::launch_tc_gemm(g3, L->num_sms, s));
+    }
     mark(L, 4, s);
     return rc;
 }

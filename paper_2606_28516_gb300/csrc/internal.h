@@ -82,8 +82,12 @@ struct TcGemmArgs {
     int64_t ldc;
     int32_t* status;
     int64_t wait_limit_ns;
+    int tmem_cols;  // 2-SM kernel: tensor-memory columns per CTA (256: one accumulator, 512: two)
 };
 int tc_pick_bn(int mode, int N);
+// 2-SM (cta_group::2) variant for the dense and grouped modes, 256 x 256 tiles per CTA pair.
+bool tc2_supported(int mode, int N);
+cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_tc_gemm(const TcGemmArgs& a, int num_sms, cudaStream_t s);
 
 // Encode a 2-D bf16 row-major [rows x cols] tensor map, box {64, box_rows}, 128-byte swizzle.

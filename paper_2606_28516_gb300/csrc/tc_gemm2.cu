@@ -1,0 +1,377 @@
+// 2-SM bf16 GEMMs of the CLEAR-MoE FFN (tcgen05 cta_group::2, sm_103a).
+//
+// A cluster of two CTAs (one per SM of a pair) computes a 256 x 256 tile: CTA r loads A rows
+// [m0 + 128 r, +128) and B rows [n0 + 128 r, +128) into its own shared memory, and one thread of
+// the even CTA issues tcgen05.mma.cta_group::2 (M = 256, N = 256, K = 16), which reads A split by M
+// and B split by N across the two CTAs and leaves rows [128 r, +128) of the accumulator in CTA r's
+// tensor memory. Each SM thus holds half of the B tile: a k-block costs it 32 KB of operands for
+// 128 x 256 x 64 MACs instead of 48 KB, so a 6-stage ring covers the load latency.
+//
+// Hand-offs: both CTAs' TMA loads complete on the even CTA's full barrier (the odd CTA's loads
+// name it through the cluster); the even CTA's MMA commits arrive on both CTAs' empty / tfull
+// barriers (multicast); the epilogue warps of both CTAs arrive on the even CTA's tempty barrier.
+// Modes: dense (one K segment, epilogue bias+GELU / plain store) and grouped (the residual
+// experts: tile pairs never straddle an expert, K chain [z | t] x [W_e | U_r], row scatter).
+// Every wait is bounded; both CTAs always reach the closing cluster barrier.
+#include "common.cuh"
+#include "internal.h"
+
+namespace cm {
+namespace t2 {
+constexpr int BM = 128;                        // rows per CTA; the pair covers 256
+constexpr int BN = 256;                        // columns per pair tile
+constexpr int BH = BN / 2;                     // B rows per CTA
+constexpr int BK = 64;
+constexpr int A_BYTES = BM * BK * 2;           // 16 KB
+constexpr int B_BYTES = BH * BK * 2;           // 16 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES; // 32 KB
+constexpr int STAGES = 6;
+constexpr int NUM_EPI = 8;
+constexpr int WARP_MMA = 8, WARP_TMA = 9;
+constexpr int THREADS = 32 * (WARP_TMA + 1);
+constexpr int HALF = BN / 2;                   // columns per epilogue warp
+constexpr int CW = 32;
+constexpr int STG_ROW = CW * 2 + 16;
+constexpr int STG_BYTES = NUM_EPI * 32 * STG_ROW;
+constexpr int NBARS = 2 * STAGES + 5;
+constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + NBARS * 8 + 128;
+}  // namespace t2
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t smem_addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int32_t c0, int32_t c1,
+                                                 uint32_t bar_cluster) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar_cluster)
+        : "memory");
+}
+__device__ __forceinline__ void umma2_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void umma2_commit_both(uint32_t bar) {  // arrive on bar in both CTAs
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            bar),
+        "h"((unsigned short)3)
+        : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+
+struct PairTile {
+    int64_t m0;  // first row of the pair tile (CTA r starts at m0 + 128 r)
+    int64_t hi;  // rows >= hi belong to another expert or lie past T
+    int n0;
+    int e;
+};
+
+__device__ __forceinline__ PairTile decode_pair(const TcGemmArgs& a, int unit, int n_tiles, const int* s_prefix) {
+    PairTile t;
+    const int mp = unit / n_tiles;
+    t.n0 = (unit % n_tiles) * t2::BN;
+    if (a.mode == TC_GROUPED) {
+        int e = 0;
+        while (e + 1 < a.E && s_prefix[e + 1] <= mp) ++e;
+        t.m0 = (int64_t)a.offsets[e] + (int64_t)(mp - s_prefix[e]) * 2 * t2::BM;
+        t.hi = a.offsets[e + 1];
+        t.e = e;
+    } else {
+        t.m0 = (int64_t)mp * 2 * t2::BM;
+        t.hi = a.M;
+        t.e = 0;
+    }
+    return t;
+}
+
+template <int MODE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
+    tc_gemm2_kernel(const __grid_constant__ TcGemmArgs a) {
+    using namespace t2;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    unsigned char* sm = smem_raw + ((1024 - (raw_addr & 1023)) & 1023);
+    unsigned char* stg = sm + STAGES * STAGE_BYTES;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(stg + STG_BYTES);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NBARS);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    int* s_prefix = reinterpret_cast<int*>(tmem_slot + 4);  // [CM_MAX_E + 1]
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_rank();
+    const bool leader = rank == 0;
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+    auto tfull_bar = [&](int i) { return bar0 + 8u * (2 * STAGES + i); };
+    auto tempty_bar = [&](int i) { return bar0 + 8u * (2 * STAGES + 2 + i); };
+    const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+    const uint64_t lim = (uint64_t)a.wait_limit_ns;
+
+    const int n_tiles = a.N / BN;
+    const int nk0 = (a.K0 + BK - 1) / BK;
+    const int nk1 = MODE == TC_GROUPED ? (a.K1 + BK - 1) / BK : 0;
+    const int nkb = nk0 + nk1;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(full_bar(s), 1);   // the even CTA's producer arrives; both CTAs' bytes land here
+            mbar_init(empty_bar(s), 1);  // one multicast commit per stage
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(tfull_bar(i), 1);
+            mbar_init(tempty_bar(i), 2 * NUM_EPI);  // epilogue warps of both CTAs
+        }
+        mbar_init(drain_bar, 1);
+        *abort_flag = 0;
+        if (MODE == TC_GROUPED) {
+            int acc = 0;
+            for (int e = 0; e < a.E; ++e) {
+                s_prefix[e] = acc;
+                acc += (a.offsets[e + 1] - a.offsets[e] + 2 * BM - 1) / (2 * BM);
+            }
+            s_prefix[a.E] = acc;
+        }
+        mbar_fence_init();
+    }
+    // Tensor memory for the pair: allocated collectively by one warp of each CTA. The two CTAs
+    // must see the same base (the even CTA's MMAs name it for both); a mismatch aborts cleanly.
+    if (warp == WARP_MMA) {
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(a.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();  // barriers initialised and TMEM bases written in both CTAs
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    uint32_t peer_base;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(peer_base) : "r"(map_to_rank(smem_u32(tmem_slot), rank ^ 1)));
+    const bool tmem_ok = peer_base == tmem_base;
+    if (!tmem_ok && threadIdx.x == 0) set_status(a.status, CLEARMOE_ECUDA);
+    const int nacc = a.tmem_cols >= 2 * BN ? 2 : 1;  // accumulator buffers
+
+    int m_pairs;
+    if (MODE == TC_GROUPED)
+        m_pairs = s_prefix[a.E];
+    else
+        m_pairs = (int)((a.M + 2 * BM - 1) / (2 * BM));
+    const int num_units = tmem_ok ? m_pairs * n_tiles : 0;
+    const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
+
+    if (warp == WARP_TMA) {
+        // ------------------------------------------------ producers (both CTAs)
+        if (lane == 0) {
+            const uint32_t full_leader0 = map_to_rank(full_bar(0), 0);
+            int stage = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            for (int u = cid; u < num_units && ok; u += ncl) {
+                const PairTile t = decode_pair(a, u, n_tiles, s_prefix);
+                const int am = (int)(t.m0 + (int64_t)rank * BM);
+                const int bn = t.n0 + (int)rank * BH;
+                for (int kb = 0; kb < nkb; ++kb) {
+                    if (!mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sA = smem_u32(sm + stage * STAGE_BYTES);
+                    const uint32_t sB = sA + A_BYTES;
+                    const uint32_t fb = full_leader0 + 8u * stage;  // the even CTA's full barrier
+                    if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * STAGE_BYTES);
+                    const CUtensorMap* mA;
+                    const CUtensorMap* mB;
+                    int kk;
+                    if (MODE != TC_GROUPED) {
+                        mA = &a.tmA0;
+                        mB = &a.tmB0;
+                        kk = kb * BK;
+                    } else if (kb < nk1) {  // z x W_e^res
+                        mA = &a.tmA1;
+                        mB = &a.tmB1[t.e];
+                        kk = kb * BK;
+                    } else {  // t x U_r
+                        mA = &a.tmA0;
+                        mB = &a.tmB0;
+                        kk = (kb - nk1) * BK;
+                    }
+                    tma_load_2d_pair(sA, mA, kk, am, fb);
+                    tma_load_2d_pair(sB, mB, kk, bn, fb);
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        ph ^= 1;
+                    }
+                }
+            }
+        }
+    } else if (warp == WARP_MMA) {
+        // ------------------------------------------------ MMA issuer (even CTA)
+        if (leader && lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(2 * BM, BN);
+            int stage = 0;
+            uint32_t ph = 0;
+            int acc = 0;
+            uint32_t aph = 0;
+            bool ok = true;
+            for (int u = cid; u < num_units && ok; u += ncl) {
+                if (!mbar_wait(tempty_bar(acc), aph ^ 1, abort_flag, a.status, lim)) break;
+                tc_fence_after();
+                const uint32_t dtm = tmem_base + acc * BN;
+                for (int kb = 0; kb < nkb; ++kb) {
+                    if (!mbar_wait(full_bar(stage), ph, abort_flag, a.status, lim)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sA = smem_u32(sm + stage * STAGE_BYTES);
+                    const uint32_t sB = sA + A_BYTES;
+                    int kvalid;
+                    if (MODE != TC_GROUPED || kb < nk1)
+                        kvalid = MODE != TC_GROUPED ? min(BK, a.K0 - kb * BK) : min(BK, a.K1 - kb * BK);
+                    else
+                        kvalid = min(BK, a.K0 - (kb - nk1) * BK);
+                    const int steps = kvalid >> 4;
+                    for (int k = 0; k < steps; ++k)
+                        umma2_bf16(dtm, sdesc_kmajor_sw128(sA + k * 32), sdesc_kmajor_sw128(sB + k * 32), idesc,
+                                   (kb > 0 || k > 0) ? 1u : 0u);
+                    umma2_commit_both(empty_bar(stage));
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        ph ^= 1;
+                    }
+                }
+                if (!ok) break;
+                umma2_commit_both(tfull_bar(acc));
+                if (++acc == nacc) {
+                    acc = 0;
+                    aph ^= 1;
+                }
+            }
+            asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(drain_bar)
+                         : "memory");
+            mbar_wait(drain_bar, 0, nullptr, a.status, 10000000ull);
+        }
+        __syncwarp();
+    } else if (warp < NUM_EPI) {
+        // ------------------------------------------------ epilogue (both CTAs, own 128 rows)
+        const int q = warp & 3;
+        const int c_lo = (warp >> 2) * HALF;
+        unsigned char* wstg = stg + warp * 32 * STG_ROW;
+        constexpr int LPR = CW / 8, RPP = 32 / LPR;
+        const uint32_t tempty_leader0 = map_to_rank(tempty_bar(0), 0);
+        int acc = 0;
+        uint32_t aph = 0;
+        for (int u = cid; u < num_units; u += ncl) {
+            const PairTile t = decode_pair(a, u, n_tiles, s_prefix);
+            if (!mbar_wait(tfull_bar(acc), aph, abort_flag, a.status, lim)) break;
+            tc_fence_after();
+            const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
+            int64_t orow = -1;
+            if (mrow < t.hi) orow = (a.epi == TC_EPI_SCATTER) ? (int64_t)a.rows[mrow] : mrow;
+            for (int c = c_lo; c < c_lo + HALF; c += CW) {
+                uint32_t v[32];
+                const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
+                CM_TMEM_LD_X16(taddr, v);
+                CM_TMEM_LD_X16(taddr + 16, (v + 16));
+                tmem_wait_ld();
+                float f[CW];
+#pragma unroll
+                for (int j = 0; j < CW; ++j) f[j] = __uint_as_float(v[j]);
+                const int nb = t.n0 + c;
+                if (a.epi == TC_EPI_BIAS_GELU) {
+                    const uint4* bp = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.bias) + nb);
+#pragma unroll
+                    for (int j8 = 0; j8 < CW / 8; ++j8) {
+                        const uint4 b = __ldg(bp + j8);
+                        const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+                        for (int h = 0; h < 4; ++h) {
+                            const float2 g = gelu_pair_as(
+                                __fadd2_rn(make_float2(f[j8 * 8 + 2 * h], f[j8 * 8 + 2 * h + 1]),
+                                           make_float2(bf16_lo(bw[h]), bf16_hi(bw[h]))));
+                            f[j8 * 8 + 2 * h] = g.x;
+                            f[j8 * 8 + 2 * h + 1] = g.y;
+                        }
+                    }
+                }
+                uint4* dst = reinterpret_cast<uint4*>(wstg + lane * STG_ROW);
+#pragma unroll
+                for (int j8 = 0; j8 < CW / 8; ++j8)
+                    dst[j8] = make_uint4(pack_bf16(f[8 * j8], f[8 * j8 + 1]), pack_bf16(f[8 * j8 + 2], f[8 * j8 + 3]),
+                                         pack_bf16(f[8 * j8 + 4], f[8 * j8 + 5]), pack_bf16(f[8 * j8 + 6], f[8 * j8 + 7]));
+                __syncwarp();
+#pragma unroll
+                for (int p = 0; p < LPR; ++p) {
+                    const int rr = p * RPP + lane / LPR;
+                    const int64_t o = __shfl_sync(0xffffffffu, orow, rr);
+                    const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * STG_ROW + (lane % LPR) * 16);
+                    if (o >= 0)
+                        *reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.C) + o * a.ldc + nb + (lane % LPR) * 8) = val;
+                }
+                __syncwarp();
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(tempty_leader0 + 8u * acc);  // the even CTA's tempty
+            if (++acc == nacc) {
+                acc = 0;
+                aph ^= 1;
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();  // no copy, commit or remote arrival is left in flight towards either CTA
+    tc_fence_after();
+    if (warp == WARP_MMA)
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(a.tmem_cols)
+                     : "memory");
+}
+
+bool tc2_supported(int mode, int N) { return (mode == TC_DENSE || mode == TC_GROUPED) && N % t2::BN == 0; }
+
+cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
+    static bool attr[3] = {false, false, false};
+    const void* fn = a.mode == TC_GROUPED ? (const void*)tc_gemm2_kernel<TC_GROUPED> : (const void*)tc_gemm2_kernel<TC_DENSE>;
+    if (!attr[a.mode]) {
+        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, t2::SMEM);
+        if (e != cudaSuccess) return e;
+        attr[a.mode] = true;
+    }
+    const int n_tiles = a.N / t2::BN;
+    int64_t m_pairs = (a.M + 2 * t2::BM - 1) / (2 * t2::BM);
+    if (a.mode == TC_GROUPED) m_pairs += a.E;
+    const int64_t units = m_pairs * n_tiles;
+    int64_t clusters = units < num_sms / 2 ? units : num_sms / 2;
+    if (clusters <= 0) return cudaSuccess;
+    const dim3 grid((unsigned)(2 * clusters));
+    if (a.mode == TC_GROUPED)
+        tc_gemm2_kernel<TC_GROUPED><<<grid, t2::THREADS, t2::SMEM, s>>>(a);
+    else
+        tc_gemm2_kernel<TC_DENSE><<<grid, t2::THREADS, t2::SMEM, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace cm
