@@ -16,7 +16,8 @@ struct clearmoe_layer {
     void* z;            // [max_tokens x hidden]  hidden states, expert-sorted order
     void* t;            // [max_tokens x max_r]   shared-basis coefficients
     int32_t* idx;       // [max_tokens]
-    int32_t* perm;      // [max_tokens]
+    int32_t* perm;      // [max_tokens]  perm[slot] = token
+    int32_t* inv;       // [max_tokens]  inv[token] = slot
     int32_t* counts;    // [CM_MAX_E]
     int32_t* offsets;   // [CM_MAX_E + 1]
     int32_t* cta_counts;  // [route_max_ctas x CM_MAX_E]
@@ -43,7 +44,7 @@ int cuda_fail(cudaError_t e) {
 }
 
 void free_ws(clearmoe_layer* L) {
-    void* ptrs[] = {L->z, L->t, L->idx, L->perm, L->counts, L->offsets, L->cta_counts, L->barrier, L->status};
+    void* ptrs[] = {L->z, L->t, L->idx, L->perm, L->inv, L->counts, L->offsets, L->cta_counts, L->barrier, L->status};
     for (void* p : ptrs)
         if (p) cudaFree(p);
 }
@@ -71,6 +72,7 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
     a.bg = router->b;
     a.idx = L->idx;
     a.perm = L->perm;
+    a.inv = L->inv;
     a.counts = L->counts;
     a.offsets = L->offsets;
     a.cta_counts = L->cta_counts;
@@ -146,6 +148,7 @@ int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out)
               cudaMalloc(&L->t, T * D.max_r * L->esz) == cudaSuccess &&
               cudaMalloc((void**)&L->idx, T * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->perm, T * 4) == cudaSuccess &&
+              cudaMalloc((void**)&L->inv, T * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->counts, CM_MAX_E * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->offsets, (CM_MAX_E + 1) * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->cta_counts, ncta * CM_MAX_E * 4) == cudaSuccess &&
@@ -265,20 +268,31 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     std::memset(&g, 0, sizeof(g));
     g.status = L->status;
     g.wait_limit_ns = L->wait_limit_ns;
-    // fc1 + b1 + GELU, A rows gathered by perm
-    if (encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
-    g.mode = cm::TC_GATHER;
+    // fc1 + b1 + GELU into z in expert order. 2-SM kernel: x read in token order by TMA, each
+    // output row stored at its slot inv[token]; otherwise A rows are gathered by perm.
     g.epi = cm::TC_EPI_BIAS_GELU;
     g.M = T;
     g.N = H;
     g.K0 = d;
-    g.gather_src = x;
-    g.gather_ld = d;
-    g.rows = L->perm;
     g.bias = b1;
     g.C = L->z;
     g.ldc = H;
-    if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
+    if (cm::tc2_supported(cm::TC_DENSE, H)) {
+        if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, 128))
+            return CLEARMOE_ECUDA;
+        g.mode = cm::TC_DENSE;
+        g.rows = L->inv;
+        g.tmem_cols = 512;
+        rc = cuda_fail(cm::launch_tc_gemm2(g, L->num_sms, s));
+    } else {
+        if (encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
+        g.mode = cm::TC_GATHER;
+        g.gather_src = x;
+        g.gather_ld = d;
+        g.rows = L->perm;
+        rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s));
+    }
+    if (rc) return rc;
     mark(L, 2, s);
     // t = diag(S_r) Vh_r z
     cm::TcGemmArgs g2;
@@ -374,7 +388,9 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     std::memset(&g, 0, sizeof(g));
     g.status = L->status;
     g.wait_limit_ns = L->wait_limit_ns;
-    if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
+    const bool pair1 = cm::tc2_supported(cm::TC_DENSE, H), pair2 = cm::tc2_supported(cm::TC_DENSE, d);
+    if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, pair1 ? 128 : bn1))
+        return CLEARMOE_ECUDA;
     g.mode = cm::TC_DENSE;
     g.epi = cm::TC_EPI_BIAS_GELU;
     g.M = T;
@@ -383,13 +399,15 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     g.bias = b1;
     g.C = L->z;
     g.ldc = H;
-    if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
+    g.tmem_cols = 512;
+    if ((rc = cuda_fail(pair1 ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s))))
+        return rc;
     mark(L, 1, s);
     cm::TcGemmArgs g2;
     std::memset(&g2, 0, sizeof(g2));
     g2.status = L->status;
     g2.wait_limit_ns = L->wait_limit_ns;
-    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, W2, d, H, bn2))
+    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, W2, d, H, pair2 ? 128 : bn2))
         return CLEARMOE_ECUDA;
     g2.mode = cm::TC_DENSE;
     g2.epi = cm::TC_EPI_STORE;
@@ -398,7 +416,8 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     g2.K0 = H;
     g2.C = out;
     g2.ldc = d;
-    rc = cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s));
+    g2.tmem_cols = 512;
+    rc = cuda_fail(pair2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
     mark(L, 2, s);
     return rc;
 }

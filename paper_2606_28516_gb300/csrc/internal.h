@@ -17,6 +17,7 @@ struct RouteArgs {
     const void* bg;
     int32_t* idx;
     int32_t* perm;
+    int32_t* inv;                  // nullable: inv[token] = slot, the inverse of perm
     int32_t* counts;
     int32_t* offsets;
     int32_t* cta_counts;           // [max_route_ctas x CM_MAX_E] scratch
@@ -73,7 +74,8 @@ struct TcGemmArgs {
     CUtensorMap tmB1[16];
     const void* gather_src;    // gather: rows of A0 read directly (bf16 [.. x K0])
     int64_t gather_ld;         // elements
-    const int32_t* rows;       // gather: A row of output row m; scatter: output row of slot m
+    const int32_t* rows;       // gather: A row of output row m; scatter (the 2-SM kernel: whenever
+                               // set): C row of output row m
     const int32_t* offsets;    // grouped: [E + 1]
     int E;
     const void* bias;          // bf16 [N]

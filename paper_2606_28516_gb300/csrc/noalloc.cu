@@ -101,6 +101,7 @@ extern "C" int clearmoe_route_noalloc(const void* x, int64_t T, int32_t d, int32
     a.bg = router->b;
     a.idx = idx;
     a.perm = perm;
+    a.inv = nullptr;
     a.counts = counts;
     a.offsets = offsets;
     a.cta_counts = scratch + kHistOffset;

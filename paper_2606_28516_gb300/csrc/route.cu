@@ -353,7 +353,11 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
             s_run[tid] = run;
         }
         __syncthreads();
-        if (valid) a.perm[s_base[e] + s_wc[warp][e] + rank] = (int32_t)(row0 + i);
+        if (valid) {
+            const int slot = s_base[e] + s_wc[warp][e] + rank;
+            a.perm[slot] = (int32_t)(row0 + i);
+            if (a.inv) a.inv[row0 + i] = slot;
+        }
         __syncthreads();
     }
 }

@@ -11,7 +11,8 @@
 // name it through the cluster); the even CTA's MMA commits arrive on both CTAs' empty / tfull
 // barriers (multicast); the epilogue warps of both CTAs arrive on the even CTA's tempty barrier.
 // Modes: dense (one K segment, epilogue bias+GELU / plain store) and grouped (the residual
-// experts: tile pairs never straddle an expert, K chain [z | t] x [W_e | U_r], row scatter).
+// experts: tile pairs never straddle an expert, K chain [z | t] x [W_e | U_r]). With a.rows set,
+// output row m goes to C[a.rows[m]] (fc1: inv[token] = slot; grouped: perm[slot] = token).
 // Every wait is bounded; both CTAs always reach the closing cluster barrier.
 #include "common.cuh"
 #include "internal.h"
@@ -288,7 +289,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
             tc_fence_after();
             const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
             int64_t orow = -1;
-            if (mrow < t.hi) orow = (a.epi == TC_EPI_SCATTER) ? (int64_t)a.rows[mrow] : mrow;
+            if (mrow < t.hi) orow = a.rows ? (int64_t)a.rows[mrow] : mrow;
             for (int c = c_lo; c < c_lo + HALF; c += CW) {
                 uint32_t v[32];
                 const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
@@ -353,6 +354,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
 bool tc2_supported(int mode, int N) { return (mode == TC_DENSE || mode == TC_GROUPED) && N % t2::BN == 0; }
 
 cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
+    if (!tc2_supported(a.mode, a.N) || a.epi == TC_EPI_SCALE || (a.tmem_cols != 256 && a.tmem_cols != 512))
+        return cudaErrorInvalidValue;
     static bool attr[3] = {false, false, false};
     const void* fn = a.mode == TC_GROUPED ? (const void*)tc_gemm2_kernel<TC_GROUPED> : (const void*)tc_gemm2_kernel<TC_DENSE>;
     if (!attr[a.mode]) {
