@@ -27,12 +27,13 @@ constexpr int A_BYTES = BM * BK * 2;           // 16 KB
 constexpr int B_BYTES = BH * BK * 2;           // 16 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES; // 32 KB
 constexpr int STAGES = 6;
-constexpr int NUM_EPI = 8;
-constexpr int WARP_MMA = 8, WARP_TMA = 9;
+constexpr int NUM_EPI = 16;                    // four per TMEM lane quarter
+constexpr int WARP_MMA = NUM_EPI, WARP_TMA = NUM_EPI + 1;
 constexpr int THREADS = 32 * (WARP_TMA + 1);
-constexpr int HALF = BN / 2;                   // columns per epilogue warp
-constexpr int CW = 32;
-constexpr int STG_ROW = CW * 2 + 16;
+constexpr int WCOLS = BN / (NUM_EPI / 4);      // columns per epilogue warp
+constexpr int CW = 32;                         // columns per tensor-memory read
+constexpr int SW = 16;                         // columns per staged store pass
+constexpr int STG_ROW = SW * 2 + 16;           // 48-byte rows: conflict-free 16-byte writes
 constexpr int STG_BYTES = NUM_EPI * 32 * STG_ROW;
 constexpr int NBARS = 2 * STAGES + 5;
 constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + NBARS * 8 + 128;
@@ -230,6 +231,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
         // ------------------------------------------------ MMA issuer (even CTA)
         if (leader && lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(2 * BM, BN);
+            // Stage s's descriptors are the stage-0 ones plus the byte offset / 16 in the start
+            // address field (every shared address here is below 256 KB, so the field never carries).
+            const uint64_t dA0 = sdesc_kmajor_sw128(smem_u32(sm));
             int stage = 0;
             uint32_t ph = 0;
             int acc = 0;
@@ -245,17 +249,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sA = smem_u32(sm + stage * STAGE_BYTES);
-                    const uint32_t sB = sA + A_BYTES;
-                    int kvalid;
-                    if (MODE != TC_GROUPED || kb < nk1)
-                        kvalid = MODE != TC_GROUPED ? min(BK, a.K0 - kb * BK) : min(BK, a.K1 - kb * BK);
+                    const uint64_t da = dA0 + (uint64_t)((stage * STAGE_BYTES) >> 4);
+                    const uint64_t db = da + (uint64_t)(A_BYTES >> 4);
+                    int krem;
+                    if (MODE != TC_GROUPED)
+                        krem = a.K0 - kb * BK;
                     else
-                        kvalid = min(BK, a.K0 - (kb - nk1) * BK);
-                    const int steps = kvalid >> 4;
-                    for (int k = 0; k < steps; ++k)
-                        umma2_bf16(dtm, sdesc_kmajor_sw128(sA + k * 32), sdesc_kmajor_sw128(sB + k * 32), idesc,
-                                   (kb > 0 || k > 0) ? 1u : 0u);
+                        krem = kb < nk1 ? a.K1 - kb * BK : a.K0 - (kb - nk1) * BK;
+                    if (krem >= BK) {
+#pragma unroll
+                        for (int k = 0; k < BK / 16; ++k)  // 16 K-elements = 32 bytes = 2 descriptor units
+                            umma2_bf16(dtm, da + 2 * k, db + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                    } else {
+                        for (int k = 0; k < (krem >> 4); ++k)
+                            umma2_bf16(dtm, da + 2 * k, db + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                    }
                     umma2_commit_both(empty_bar(stage));
                     if (++stage == STAGES) {
                         stage = 0;
@@ -276,10 +284,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
         __syncwarp();
     } else if (warp < NUM_EPI) {
         // ------------------------------------------------ epilogue (both CTAs, own 128 rows)
-        const int q = warp & 3;
-        const int c_lo = (warp >> 2) * HALF;
+        const int q = warp & 3;  // a warp reads the TMEM lanes of its index mod 4
+        const int c_lo = (warp >> 2) * WCOLS;
         unsigned char* wstg = stg + warp * 32 * STG_ROW;
-        constexpr int LPR = CW / 8, RPP = 32 / LPR;
+        constexpr int LPR = SW / 8, RPP = 32 / LPR;
         const uint32_t tempty_leader0 = map_to_rank(tempty_bar(0), 0);
         int acc = 0;
         uint32_t aph = 0;
@@ -290,8 +298,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
             const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
             int64_t orow = -1;
             if (mrow < t.hi) orow = a.rows ? (int64_t)a.rows[mrow] : mrow;
-            for (int c = c_lo; c < c_lo + HALF; c += CW) {
-                uint32_t v[32];
+            for (int c = c_lo; c < c_lo + WCOLS; c += CW) {
+                uint32_t v[CW];
                 const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
                 CM_TMEM_LD_X16(taddr, v);
                 CM_TMEM_LD_X16(taddr + 16, (v + 16));
@@ -316,21 +324,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
                         }
                     }
                 }
-                uint4* dst = reinterpret_cast<uint4*>(wstg + lane * STG_ROW);
 #pragma unroll
-                for (int j8 = 0; j8 < CW / 8; ++j8)
-                    dst[j8] = make_uint4(pack_bf16(f[8 * j8], f[8 * j8 + 1]), pack_bf16(f[8 * j8 + 2], f[8 * j8 + 3]),
-                                         pack_bf16(f[8 * j8 + 4], f[8 * j8 + 5]), pack_bf16(f[8 * j8 + 6], f[8 * j8 + 7]));
-                __syncwarp();
+                for (int s0 = 0; s0 < CW; s0 += SW) {
+                    uint4* dst = reinterpret_cast<uint4*>(wstg + lane * STG_ROW);
 #pragma unroll
-                for (int p = 0; p < LPR; ++p) {
-                    const int rr = p * RPP + lane / LPR;
-                    const int64_t o = __shfl_sync(0xffffffffu, orow, rr);
-                    const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * STG_ROW + (lane % LPR) * 16);
-                    if (o >= 0)
-                        *reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.C) + o * a.ldc + nb + (lane % LPR) * 8) = val;
+                    for (int j8 = 0; j8 < SW / 8; ++j8) {
+                        const float* g = f + s0 + 8 * j8;
+                        dst[j8] = make_uint4(pack_bf16(g[0], g[1]), pack_bf16(g[2], g[3]), pack_bf16(g[4], g[5]),
+                                             pack_bf16(g[6], g[7]));
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int p = 0; p < LPR; ++p) {
+                        const int rr = p * RPP + lane / LPR;
+                        const int64_t o = __shfl_sync(0xffffffffu, orow, rr);
+                        const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * STG_ROW + (lane % LPR) * 16);
+                        if (o >= 0)
+                            *reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.C) + o * a.ldc + nb + s0 +
+                                                      (lane % LPR) * 8) = val;
+                    }
+                    __syncwarp();
                 }
-                __syncwarp();
             }
             tc_fence_before();
             __syncwarp();
