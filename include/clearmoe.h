@@ -124,8 +124,10 @@ int clearmoe_layer_status(clearmoe_layer* layer);
 
 /* Fault injection for tests of the bounded waits: the grid-wide wait of the routing kernel
  * gives up after wait_limit_ns nanoseconds (default 1e9) and, when phantom_arrivals > 0, waits
- * for that many arrivals more than can ever come, so the wait runs out and the call reports
- * CLEARMOE_ETIMEOUT through clearmoe_layer_status. phantom_arrivals = 0 restores normal use. */
+ * for the histograms of that many CTAs more than the launch has, so the wait runs out and the
+ * call reports CLEARMOE_ETIMEOUT through clearmoe_layer_status (the layer stays usable: the next
+ * launch needs no reset). phantom_arrivals = 0 restores normal use; a launch whose grid plus
+ * phantom_arrivals exceeds the histogram scratch returns CLEARMOE_EUNSUPPORTED. */
 int clearmoe_debug_set_wait(clearmoe_layer* layer, int64_t wait_limit_ns, int32_t phantom_arrivals);
 
 /* Per-stage timing: when n >= 5, clearmoe_ffn_forward records events[0] before its first kernel
@@ -142,15 +144,16 @@ int clearmoe_set_profile_events(clearmoe_layer* layer, void* const* events, int3
  * (idx [T], counts [E], offsets [E + 1], perm [T]: caller-owned int32 device outputs) for tokens
  * x [T x d] of dtype `dtype` and the router W [E x d], b [E] in that dtype.
  *   - It calls no cudaMalloc, cudaFree or other allocating routine. Its scratch (per-CTA expert
- *     histograms, the arrival counter of the grid-wide wait, a spare status word) is one static
- *     device array of 65,600 bytes that every GPU loading the library holds until exit; it serves
- *     up to 1,024 routing CTAs (two per SM on GPUs with up to 512 SMs). A launch that would need
- *     more returns CLEARMOE_EUNSUPPORTED and enqueues nothing.
+ *     histograms, the launch epoch that tags them, a spare status word) is one static device
+ *     array of 65,600 bytes that every GPU loading the library holds until exit; it serves up to
+ *     512 routing CTAs (two per SM on GPUs with up to 256 SMs). A launch that would need more
+ *     returns CLEARMOE_EUNSUPPORTED and enqueues nothing.
  *   - The first call on a device looks up the array's device address (once per device, with that
  *     device current); make that first call before any stream capture.
- *   - Every call shares the array and it keeps the last call's contents; each call clears what
- *     must start at zero. Calls whose work overlaps on the GPU (other streams, other host
- *     threads) race on the array: serialise them.
+ *   - Every call shares the array and it keeps the last call's contents, on purpose: the epoch
+ *     only grows and the histogram words carry it, so nothing needs clearing but the status
+ *     word. Calls whose work overlaps on the GPU (other streams, other host threads) race on the
+ *     array: serialise them.
  *   - status (optional int32 device pointer, else NULL) is set to 0 at the start of the call and
  *     receives CLEARMOE_ETIMEOUT if the bounded grid-wide wait (1 s) runs out, in which case the
  *     outputs are undefined.

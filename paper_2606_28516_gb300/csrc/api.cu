@@ -20,8 +20,8 @@ struct clearmoe_layer {
     int32_t* inv;       // [max_tokens]  inv[token] = slot
     int32_t* counts;    // [CM_MAX_E]
     int32_t* offsets;   // [CM_MAX_E + 1]
-    int32_t* cta_counts;  // [route_max_ctas x CM_MAX_E]
-    unsigned int* barrier;  // the routing kernel's grid barrier: arrivals, generation
+    unsigned long long* cta_words;  // [route_max_ctas x CM_MAX_E] the routing kernel's histogram words
+    unsigned long long* epoch;      // the routing kernel's launch epoch
     int32_t* status;
     int64_t wait_limit_ns;
     int32_t phantom;
@@ -44,7 +44,7 @@ int cuda_fail(cudaError_t e) {
 }
 
 void free_ws(clearmoe_layer* L) {
-    void* ptrs[] = {L->z, L->t, L->idx, L->perm, L->inv, L->counts, L->offsets, L->cta_counts, L->barrier, L->status};
+    void* ptrs[] = {L->z, L->t, L->idx, L->perm, L->inv, L->counts, L->offsets, L->cta_words, L->epoch, L->status};
     for (void* p : ptrs)
         if (p) cudaFree(p);
 }
@@ -59,10 +59,12 @@ int check_common(const clearmoe_layer* L, const void* x, int64_t T) {
 int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router, int E,
              cudaStream_t s) {
     int grid = 0, chunk = 0;
-    if (cm::route_grid(T, L->desc.d, E, L->desc.dtype, L->num_sms, &grid, &chunk) != 0)
-        return CLEARMOE_ECUDA;
-    if (grid > cm::route_max_ctas(L->num_sms, L->desc.dtype, L->desc.d, E)) return CLEARMOE_EUNSUPPORTED;
+    const int g = cm::route_grid(T, L->desc.d, E, L->desc.dtype, L->num_sms, &grid, &chunk);
+    if (g) return g == -2 ? CLEARMOE_EUNSUPPORTED : CLEARMOE_ECUDA;
+    if (grid + L->phantom > cm::route_max_ctas(L->num_sms, L->desc.dtype, L->desc.d, E))
+        return CLEARMOE_EUNSUPPORTED;
     cm::RouteArgs a;
+    std::memset(&a, 0, sizeof(a));
     a.x = x;
     a.T = T;
     a.d = L->desc.d;
@@ -75,8 +77,8 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
     a.inv = L->inv;
     a.counts = L->counts;
     a.offsets = L->offsets;
-    a.cta_counts = L->cta_counts;
-    a.barrier = L->barrier;
+    a.cta_words = L->cta_words;
+    a.epoch = L->epoch;
     a.arrivals = (unsigned int)grid + (unsigned int)L->phantom;
     a.wait_limit_ns = L->wait_limit_ns;
     a.status = L->status;
@@ -151,11 +153,13 @@ int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out)
               cudaMalloc((void**)&L->inv, T * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->counts, CM_MAX_E * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->offsets, (CM_MAX_E + 1) * 4) == cudaSuccess &&
-              cudaMalloc((void**)&L->cta_counts, ncta * CM_MAX_E * 4) == cudaSuccess &&
-              cudaMalloc((void**)&L->barrier, 8) == cudaSuccess &&
+              cudaMalloc((void**)&L->cta_words, ncta * CM_MAX_E * 8) == cudaSuccess &&
+              cudaMalloc((void**)&L->epoch, 8) == cudaSuccess &&
               cudaMalloc((void**)&L->status, 4) == cudaSuccess;
     if (ok) {
-        ok = cudaMemset(L->barrier, 0, 8) == cudaSuccess && cudaMemset(L->status, 0, 4) == cudaSuccess &&
+        ok = cudaMemset(L->epoch, 0, 8) == cudaSuccess &&
+             cudaMemset(L->cta_words, 0, ncta * CM_MAX_E * 8) == cudaSuccess &&
+             cudaMemset(L->status, 0, 4) == cudaSuccess &&
              cudaDeviceSynchronize() == cudaSuccess;
     }
     if (!ok) {
@@ -452,11 +456,8 @@ int clearmoe_layer_status(clearmoe_layer* L) {
     int32_t st = 0;
     if (cudaMemcpy(&st, L->status, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return CLEARMOE_ECUDA;
     if (st != 0) {
+        // (a routing launch that gave up has already retired its tag: nothing else to reset)
         if (cudaMemset(L->status, 0, 4) != cudaSuccess) return CLEARMOE_ECUDA;
-        if (st == CLEARMOE_ETIMEOUT) {
-            // a launch that gave up left arrivals behind: start the grid barrier afresh
-            if (cudaMemset(L->barrier, 0, 8) != cudaSuccess) return CLEARMOE_ECUDA;
-        }
         if (cudaDeviceSynchronize() != cudaSuccess) return CLEARMOE_ECUDA;
     }
     return st;

@@ -20,14 +20,15 @@ struct RouteArgs {
     int32_t* inv;                  // nullable: inv[token] = slot, the inverse of perm
     int32_t* counts;
     int32_t* offsets;
-    int32_t* cta_counts;           // [max_route_ctas x CM_MAX_E] scratch
-    unsigned int* barrier;         // [0] arrivals, [1] generation: a self-resetting grid barrier
-    unsigned int arrivals;         // arrivals that release the wait (the grid; more in fault tests)
+    unsigned long long* cta_words; // [max_route_ctas x CM_MAX_E] histogram words, tag << 32 | count
+    unsigned long long* epoch;     // the last launch's tag (only grows; zero-initialised once)
+    unsigned int arrivals;         // histogram rows awaited (the grid; more in fault tests)
     int64_t wait_limit_ns;
     int32_t* status;
 };
 
-// Grid of the routing kernel for T tokens (co-resident CTAs); chunk = rows per CTA.
+// Grid of the routing kernel for T tokens (co-resident CTAs); chunk = rows per CTA. Returns 0,
+// -1 on a CUDA error, -2 when no launch shape fits.
 int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* chunk);
 int route_max_ctas(int num_sms, int dtype, int d, int E);
 cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s);

@@ -5,9 +5,10 @@
 // allocation there), processes held to a fixed device-memory budget, and latency-critical loops
 // where cudaMalloc's implicit device-wide synchronisation is not acceptable. The handle-based
 // calls allocate their workspace in clearmoe_layer_create, so this entry point offers the routing
-// kernel without a handle: its scratch (the per-CTA expert histograms, the arrival counter of the
-// grid-wide wait and a status word) is a file-scope device array that every GPU loading the
-// library holds until the process exits.
+// kernel without a handle: its scratch (the per-CTA expert histograms, the launch epoch that tags
+// them and a status word) is a file-scope device array that every GPU loading the library holds
+// until the process exits.
+#include <cstring>
 #include <mutex>
 
 #include "common.cuh"
@@ -15,11 +16,12 @@
 
 namespace {
 
-// Scratch layout (int32 words): [0, 2) the grid barrier (arrivals, generation), [2] status word
-// used when the caller passes no status pointer, [16, 16 + MAX_CTAS * CM_MAX_E) per-CTA histograms.
-constexpr int kNoallocMaxCtas = 1024;
+// Scratch layout (int32 words): [0, 2) the routing kernel's 64-bit launch epoch, [2] status word
+// used when the caller passes no status pointer, [16, 16 + 2 * MAX_CTAS * CM_MAX_E) the per-CTA
+// histogram words (64-bit: launch tag << 32 | count).
+constexpr int kNoallocMaxCtas = 512;
 constexpr int kHistOffset = 16;
-constexpr int kScratchWords = kHistOffset + kNoallocMaxCtas * CM_MAX_E;  // 65,600 bytes
+constexpr int kScratchWords = kHistOffset + 2 * kNoallocMaxCtas * CM_MAX_E;  // 65,600 bytes
 
 static __device__ __align__(256) int32_t g_route_scratch[kScratchWords];
 
@@ -80,18 +82,21 @@ extern "C" int clearmoe_route_noalloc(const void* x, int64_t T, int32_t d, int32
     int rc = scratch_for_current_device(&scratch, &num_sms);
     if (rc) return rc;
     int grid = 0, chunk = 0;
-    if (cm::route_grid(T, d, E, dtype, num_sms, &grid, &chunk) != 0) return CLEARMOE_ECUDA;
+    const int g = cm::route_grid(T, d, E, dtype, num_sms, &grid, &chunk);
+    if (g) return g == -2 ? CLEARMOE_EUNSUPPORTED : CLEARMOE_ECUDA;
     if (grid > kNoallocMaxCtas) return CLEARMOE_EUNSUPPORTED;  // beyond the scratch's capacity
 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    // The array keeps the previous call's contents: the grid barrier and the spare status word
-    // are cleared (the histograms are fully rewritten before they are read).
-    if (cudaMemsetAsync(scratch, 0, kHistOffset * sizeof(int32_t), s) != cudaSuccess ||
+    // The array keeps the previous call's contents, which is what the epoch needs (zero when the
+    // module loads, then only growing); the histogram words are tagged with it, so they need no
+    // clearing. Only the spare status word and the caller's status are cleared.
+    if (cudaMemsetAsync(scratch + 2, 0, sizeof(int32_t), s) != cudaSuccess ||
         (status && cudaMemsetAsync(status, 0, sizeof(int32_t), s) != cudaSuccess)) {
         (void)cudaGetLastError();
         return CLEARMOE_ECUDA;
     }
     cm::RouteArgs a;
+    std::memset(&a, 0, sizeof(a));
     a.x = x;
     a.T = T;
     a.d = d;
@@ -104,8 +109,8 @@ extern "C" int clearmoe_route_noalloc(const void* x, int64_t T, int32_t d, int32
     a.inv = nullptr;
     a.counts = counts;
     a.offsets = offsets;
-    a.cta_counts = scratch + kHistOffset;
-    a.barrier = reinterpret_cast<unsigned int*>(scratch);
+    a.cta_words = reinterpret_cast<unsigned long long*>(scratch + kHistOffset);
+    a.epoch = reinterpret_cast<unsigned long long*>(scratch);
     a.arrivals = (unsigned int)grid;
     a.wait_limit_ns = 1000000000LL;
     a.status = status ? status : scratch + 2;

@@ -7,12 +7,16 @@
 //            bf16: one CTA per SM; a producer thread copies the CTA's rows, 16 at a time, into a
 //            ring of shared-memory stages with 1-D bulk copies (mbarrier-tracked, so the bytes in
 //            flight cost no registers) and eight consumer warps take one 16-row stage each;
-//   grid-wide wait (bounded, on a monotone arrival counter);
+//   exchange: each CTA publishes its histogram as 64-bit words (launch tag << 32 | count), ranks
+//            its rows locally, then polls every CTA's row (one row per thread) until all carry
+//            this launch's tag, which is both the grid-wide wait (bounded) and the load of the
+//            counts;
 //   phase 2: each CTA sums the histograms of the CTAs before it and writes its tokens' slots in
-//            token order (ranks from warp match masks), which makes the sort stable.
-// bf16 tokens: the d x E contraction runs on the legacy warp MMA (m16n8k16, fp32 accumulate)
-// straight from registers: the 16-byte loads of x are coalesced, and the K order of each
-// fragment is permuted identically for x and W_g, which leaves every dot product unchanged.
+//            token order (local ranks from warp match masks), which makes the sort stable.
+// bf16 tokens: the d x E contraction runs on the legacy warp MMA (m16n8k16, fp32 accumulate):
+// x fragments from the shared-memory stage, W_g fragments staged once in shared memory (reading
+// them through L1 in the inner loop was measured slower), and the K order of each fragment is
+// permuted identically for x and W_g, which leaves every dot product unchanged.
 // fp32 tokens: fp32 FMA on the CUDA cores (an fp32 router decision needs fp32 products).
 #include <mutex>
 
@@ -25,7 +29,6 @@ constexpr int RT_THREADS = 256;                 // fp32 router: 8 warps
 constexpr int RT_BF16_THREADS = 288;            // bf16 router: 8 consumer warps + 1 producer warp
 constexpr int RT_MAX_WARPS = RT_BF16_THREADS / 32;
 constexpr int RT_STAGE_ROWS = 16;               // rows per ring stage (one MMA row group)
-constexpr int RT_RING_BYTES = 192 * 1024;       // shared-memory ring budget (bf16 router)
 
 __device__ __forceinline__ uint4 ldg_nc_v4(const uint4* p) {
     uint4 v;
@@ -53,35 +56,42 @@ __device__ __forceinline__ void arg_better(float& bv, int& be, float v, int e) {
     }
 }
 
+// bf16: W_g rows in shared memory with a 64-byte pad, so that the 16-byte B-fragment reads of a
+// quarter warp (two rows, four 16-byte column groups each) hit all 32 banks once. Token stages
+// stay contiguous (one bulk copy per 16 rows, 2-way conflicts on the A-fragment reads): neither
+// per-row copies into padded rows nor a 128-byte-swizzled tensor copy was measured faster.
+__host__ __device__ inline int wrow_bytes(int d) { return d * 2 + 64; }
 __host__ __device__ inline size_t frag_bytes(int dtype, int d, int E) {
-    if (dtype == CLEARMOE_BF16) return (size_t)((E + 7) / 8) * (d / 32) * 32 * 16;
+    if (dtype == CLEARMOE_BF16) return (size_t)E * wrow_bytes(d);
     return (size_t)E * d * 4;
 }
 
-// Dynamic shared memory: [router weights] [bf16: ring of S stages] [bf16: 2 S mbarriers]. The
-// chosen expert of each row goes to idx in global memory and is read back from there (the CTA's
-// own writes, visible block-wide after __syncthreads), so the footprint does not grow with T.
+// Dynamic shared memory: [router weights] [bf16: ring of S stages] [bf16: 2 S + 1 mbarriers]
+// [per-row word: expert | local rank << 8, when chunk words fit; else that word lives in idx in
+// global memory (the CTA's own rows, visible block-wide after __syncthreads) until phase 2
+// rewrites idx with the expert alone], so the footprint does not grow with T.
 // The ring has one slot per consumer warp (S = 8, or 4 when eight stages do not fit): consumer
 // warp w alone reads slot w, for stages w, w + S, ..., so each of its mbarrier waits is for the
 // phase right after the one it last consumed (a parity wait cannot tell phases two apart).
+constexpr size_t RT_SMEM_MAX = 220 * 1024;
 struct RouteLayout {
     size_t ring, bars, sidx, total;
     int S, stage_bytes;
     bool sidx_in_smem;
 };
-constexpr size_t RT_SMEM_MAX = 220 * 1024;
 __host__ __device__ inline RouteLayout route_layout(int dtype, int d, int E, int chunk) {
     RouteLayout L;
     const size_t frag = (frag_bytes(dtype, d, E) + 127) & ~(size_t)127;
     L.stage_bytes = RT_STAGE_ROWS * d * 2;
     L.S = 0;
     L.ring = frag;
-    if (dtype == CLEARMOE_BF16) L.S = (8 * L.stage_bytes <= RT_RING_BYTES) ? 8 : 4;
+    if (dtype == CLEARMOE_BF16)  // eight slots when they fit beside W_g and the barriers, else four
+        L.S = (L.ring + 8 * (size_t)L.stage_bytes + 17 * 8 <= RT_SMEM_MAX) ? 8 : 4;
     L.bars = (L.ring + (size_t)L.S * L.stage_bytes + 15) & ~(size_t)15;
-    L.sidx = L.bars + (size_t)2 * L.S * 8;
+    L.sidx = L.bars + (size_t)(2 * L.S + 1) * 8;  // bf16: ring barriers + the W_g barrier
     // expert ids of the CTA's rows: in shared memory when they fit, else read back from idx
-    L.sidx_in_smem = L.sidx + (size_t)chunk <= RT_SMEM_MAX;
-    L.total = L.sidx + (L.sidx_in_smem ? (size_t)chunk : 0);
+    L.sidx_in_smem = L.sidx + (size_t)chunk * 4 <= RT_SMEM_MAX;
+    L.total = L.sidx + (L.sidx_in_smem ? (size_t)chunk * 4 : 0);
     return L;
 }
 static size_t route_smem(int dtype, int d, int E, int chunk) { return route_layout(dtype, d, E, chunk).total; }
@@ -100,10 +110,11 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ int s_count[CM_MAX_E];
     __shared__ int s_base[CM_MAX_E];
-    __shared__ int s_tot[CM_MAX_E];
     __shared__ int s_run[CM_MAX_E];
     __shared__ int s_wc[RT_MAX_WARPS][CM_MAX_E];
+    __shared__ int s_part[RT_MAX_WARPS][CM_MAX_E];
     __shared__ int s_abort;
+    __shared__ uint32_t s_tag;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int E = a.E, d = a.d;
@@ -112,16 +123,26 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     const int nchunk = d / 32;
     const int NT = (E + 7) / 8;
     const RouteLayout lay = route_layout(BF16 ? CLEARMOE_BF16 : CLEARMOE_F32, d, E, chunk);
-    uint8_t* sidx = lay.sidx_in_smem ? smem + lay.sidx : nullptr;
-    auto expert_of = [&](int i) -> int { return sidx ? (int)sidx[i] : __ldcg(a.idx + row0 + i); };
-    auto record = [&](int i, int e) {  // phase 1 result of row i: idx, local id copy, histogram
+    // per-row word: the expert after phase 1, expert | local rank << 8 after the local ranking
+    uint32_t* sinfo = lay.sidx_in_smem ? reinterpret_cast<uint32_t*>(smem + lay.sidx) : nullptr;
+    auto info_of = [&](int i) -> uint32_t { return sinfo ? sinfo[i] : (uint32_t)__ldcg(a.idx + row0 + i); };
+    auto set_info = [&](int i, uint32_t v) {
+        if (sinfo)
+            sinfo[i] = v;
+        else
+            a.idx[row0 + i] = (int32_t)v;
+    };
+    auto record = [&](int i, int e) {  // phase 1 result of row i: idx, the row's word, histogram
         a.idx[row0 + i] = e;
-        if (sidx) sidx[i] = (uint8_t)e;
+        if (sinfo) sinfo[i] = (uint32_t)e;
         atomicAdd(&s_count[e], 1);
     };
 
     if (tid < CM_MAX_E) s_count[tid] = 0;
     if (tid == 0) s_abort = 0;
+    // the launch epoch, read now and used after phase 1 (the load's latency hides behind it)
+    unsigned long long ep0 = 0;
+    if (tid == 0) asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(ep0) : "l"(a.epoch) : "memory");
 
     // ---------------- phase 1: router logits + argmax for this CTA's rows
     if constexpr (BF16) {
@@ -132,28 +153,28 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
         const int nstages = (nrows + RT_STAGE_ROWS - 1) / RT_STAGE_ROWS;
         volatile int* abort_flag = &s_abort;
-        if (tid == 0) {
+        // ---- producer: stage k = rows [16 k, 16 k + 16) of this CTA, ring slot k % S. Its thread
+        // initialises the barriers, copies W_g's rows into shared memory (first in its queue, on
+        // their own barrier) and then streams the stages.
+        const bool producer = tid == NCONS_MAX * 32;
+        const uint32_t wbar = bar0 + 8u * (2 * S);
+        const int WRB = wrow_bytes(d);
+        if (producer) {
             for (int s = 0; s < S; ++s) {
                 mbar_init(full_bar(s), 1);
                 mbar_init(empty_bar(s), 1);
             }
+            mbar_init(wbar, 1);
             mbar_fence_init();
         }
-        // B fragments of W_g: [n-tile][32-column chunk][lane] -> 8 consecutive bf16 of row
-        // nt*8 + lane/4, columns chunk*32 + (lane%4)*8.
-        uint4* bfrag = reinterpret_cast<uint4*>(smem);
-        const uint16_t* W = static_cast<const uint16_t*>(a.Wg);
-        for (int i = tid; i < NT * nchunk * 32; i += NTHREADS) {
-            const int l = i & 31, c = (i >> 5) % nchunk, nt = (i >> 5) / nchunk;
-            const int e = nt * 8 + (l >> 2);
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (e < E) v = *reinterpret_cast<const uint4*>(W + (size_t)e * d + c * 32 + (l & 3) * 8);
-            bfrag[i] = v;
+        __syncthreads();  // barriers initialised
+        if (producer) {
+            mbar_arrive_expect_tx(wbar, (uint32_t)E * d * 2);
+            const unsigned char* Wb = static_cast<const unsigned char*>(a.Wg);
+            for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(smem) + e * WRB, Wb + (size_t)e * d * 2, d * 2, wbar);
         }
-        __syncthreads();
         if (warp == NCONS_MAX) {
-            // ---- producer: stage k = rows [16 k, 16 k + 16) of this CTA, ring slot k % S
-            if (lane == 0) {
+            if (producer) {
                 const unsigned char* xb = static_cast<const unsigned char*>(a.x) + row0 * d * 2;
                 int k = 0;
                 for (; k < nstages; ++k) {
@@ -169,13 +190,23 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                     for (int j = max(0, k - S); j < k; ++j)
                         mbar_wait(full_bar(j % S), (j / S) & 1, nullptr, a.status, 10000000ull);
                 }
+                mbar_wait(wbar, 0, nullptr, a.status, 10000000ull);  // W_g's rows have landed too
             }
         } else if (warp < S) {
             // ---- consumers: warp w owns slot w and takes stages w, w + S, w + 2 S, ...
             const uint16_t* bgp = static_cast<const uint16_t*>(a.bg);
             const int g = lane >> 2, tig = lane & 3;
             const uint4 zero = make_uint4(0, 0, 0, 0);
-            for (int k = warp; k < nstages; k += S) {
+            // B fragment of n-tile nt, 32-column chunk c: 8 consecutive bf16 of W_g row nt*8 + g,
+            // columns c*32 + tig*8 (rows past E are zero)
+            const uint4* wfr[2];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+                wfr[nt] = (nt < NT && nt * 8 + g < E)
+                              ? reinterpret_cast<const uint4*>(smem + (size_t)(nt * 8 + g) * WRB + tig * 16)
+                              : nullptr;
+            const bool w_ok = nstages == 0 || mbar_wait(wbar, 0, abort_flag, a.status, (uint64_t)a.wait_limit_ns);
+            for (int k = warp; w_ok && k < nstages; k += S) {
                 const int s = warp;
                 if (!mbar_wait(full_bar(s), (k / S) & 1, abort_flag, a.status, (uint64_t)a.wait_limit_ns)) break;
                 const int rows = min(RT_STAGE_ROWS, nrows - k * RT_STAGE_ROWS);
@@ -183,21 +214,37 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 const unsigned char* st = smem + lay.ring + (size_t)s * SB;
                 const uint4* pA = reinterpret_cast<const uint4*>(st + (size_t)g * d * 2) + tig;
                 const uint4* pB = reinterpret_cast<const uint4*>(st + (size_t)(g + 8) * d * 2) + tig;
-                float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-                for (int c = 0; c < nchunk; ++c) {
-                    const uint4 xa = vA ? pA[4 * c] : zero;
-                    const uint4 xb = vB ? pB[4 * c] : zero;
+                // four independent accumulator chains (K steps 4j + q go to chain q), summed at the end
+                float part[2][4][4];
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) part[nt][q][i] = 0.f;
+                for (int c = 0; c < nchunk; c += 2) {  // d % 64 == 0: nchunk is even
+                    const uint4 xa0 = vA ? pA[4 * c] : zero, xa1 = vA ? pA[4 * c + 4] : zero;
+                    const uint4 xb0 = vB ? pB[4 * c] : zero, xb1 = vB ? pB[4 * c + 4] : zero;
 #pragma unroll
                     for (int nt = 0; nt < 2; ++nt) {
                         if (nt < NT) {
-                            const uint4 w = bfrag[(nt * nchunk + c) * 32 + lane];
-                            mma_bf16_16816(acc[nt], xa.x, xb.x, xa.y, xb.y, w.x, w.y);
-                            mma_bf16_16816(acc[nt], xa.z, xb.z, xa.w, xb.w, w.z, w.w);
+                            const uint4 w0 = wfr[nt] ? wfr[nt][4 * c] : zero;
+                            const uint4 w1 = wfr[nt] ? wfr[nt][4 * c + 4] : zero;
+                            mma_bf16_16816(part[nt][0], xa0.x, xb0.x, xa0.y, xb0.y, w0.x, w0.y);
+                            mma_bf16_16816(part[nt][1], xa0.z, xb0.z, xa0.w, xb0.w, w0.z, w0.w);
+                            mma_bf16_16816(part[nt][2], xa1.x, xb1.x, xa1.y, xb1.y, w1.x, w1.y);
+                            mma_bf16_16816(part[nt][3], xa1.z, xb1.z, xa1.w, xb1.w, w1.z, w1.w);
                         }
                     }
                 }
                 __syncwarp();
-                if (lane == 0) mbar_arrive(empty_bar(s));  // the stage's rows are in registers now
+                if (lane == 0) mbar_arrive(empty_bar(s));  // the stage is no longer read
+                float acc[2][4];
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        acc[nt][i] = (part[nt][0][i] + part[nt][1][i]) + (part[nt][2][i] + part[nt][3][i]);
                 // D fragment: acc[nt][0..1] = row g, experts nt*8 + 2*tig + {0,1}; [2..3] = row g+8
                 float bA = -INFINITY, bB = -INFINITY;
                 int eA = 0x7fffffff, eB = 0x7fffffff;
@@ -267,102 +314,160 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     }
     __syncthreads();
 
-    // ---------------- the local histogram (built in phase 1), published for the other CTAs by the
-    // thread that arrives at the grid barrier
-
-    // ---------------- grid-wide wait (bounded), self-resetting: the last of `arrivals` CTAs zeroes
-    // the arrival count and bumps the generation that the others wait on, so nothing carries over
-    // to the next launch and the host keeps no barrier state.
-    if (tid == 0) {
-        unsigned int* arrived = a.barrier;
-        unsigned int* generation = a.barrier + 1;
-        for (int e = 0; e < E; ++e) a.cta_counts[(size_t)blockIdx.x * CM_MAX_E + e] = s_count[e];
-        const unsigned int gen0 = ld_acquire_u32(generation);
-        __threadfence();  // the histogram is visible before this CTA's arrival
-        unsigned int prev;
-        asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(prev) : "l"(arrived) : "memory");
-        if (prev == a.arrivals - 1) {
-            st_release_u32(generation, gen0 + 1);  // release everyone, then reset for the next launch
-            atomicExch(arrived, 0u);
-        } else {
-            const uint64_t t0 = globaltimer();
-            while (ld_acquire_u32(generation) == gen0) {
-                if (globaltimer() - t0 > (uint64_t)a.wait_limit_ns) {
-                    s_abort = 1;
-                    set_status(a.status, CLEARMOE_ETIMEOUT);
-                    break;
-                }
-                __nanosleep(64);
-            }
-        }
-    }
+    // ---------------- exchange of the histograms. The launch tag is the low word of epoch + 1,
+    // where *a.epoch only grows (the last launch's tag, raised at the end of every launch, also
+    // one that timed out), so no row left by an earlier launch carries this launch's tag and
+    // nothing is reset between launches. Each 8-byte word is written and read whole, so a word
+    // with the right tag holds this launch's count.
+    if (tid == 0) s_tag = (uint32_t)(ep0 + 1);
     __syncthreads();
-    if (s_abort) return;
+    const uint32_t tag = s_tag;
+    if (tid < E) {
+        const unsigned long long w = ((unsigned long long)tag << 32) | (uint32_t)s_count[tid];
+        asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(a.cta_words + (size_t)blockIdx.x * CM_MAX_E + tid),
+                     "l"(w)
+                     : "memory");
+    }
 
-    // ---------------- phase 2: global offsets, then this CTA's slots in token order
-    for (int e = warp; e < E; e += NWARPS) {
-        int before = 0, total = 0;
-        for (int b = lane; b < (int)gridDim.x; b += 32) {
-            const int c = __ldcg(&a.cta_counts[(size_t)b * CM_MAX_E + e]);
-            total += c;
-            if (b < (int)blockIdx.x) before += c;
-        }
-#pragma unroll
-        for (int off = 16; off >= 1; off >>= 1) {
-            before += __shfl_xor_sync(0xffffffffu, before, off);
-            total += __shfl_xor_sync(0xffffffffu, total, off);
-        }
-        if (lane == 0) {
-            s_base[e] = before;
-            s_tot[e] = total;
-        }
-    }
-    __syncthreads();
-    if (tid == 0) {
-        int run = 0;
-        for (int e = 0; e < E; ++e) {
-            const int t = s_tot[e];
-            s_base[e] += run;
-            if (blockIdx.x == 0) {
-                a.counts[e] = t;
-                a.offsets[e] = run;
-            }
-            run += t;
-            s_run[e] = 0;
-        }
-        if (blockIdx.x == 0) a.offsets[E] = run;
-    }
+    // ---------------- local ranks: row i's rank among this CTA's earlier rows of the same expert
+    // (warp match masks, then a per-expert prefix over warps and over passes), which makes the
+    // final order stable. Done while the other CTAs publish.
+    // Per pass of NTHREADS rows: each warp's count per expert goes to s_wc; then lane e of every
+    // warp adds the counts of the warps before it (independent loads, no serial chain) to the
+    // running count of earlier passes, s_run; the last warp advances s_run.
     const unsigned lt = (1u << lane) - 1u;
+    if (tid < CM_MAX_E) s_run[tid] = 0;
     for (int i0 = 0; i0 < nrows; i0 += NTHREADS) {
         if (tid < NWARPS * CM_MAX_E) (&s_wc[0][0])[tid] = 0;
         __syncthreads();
         const int i = i0 + tid;
         const bool valid = i < nrows;
-        const int e = valid ? expert_of(i) : CM_MAX_E + 1;
+        const int e = valid ? (int)(info_of(i) & 0xffu) : CM_MAX_E + 1;
         const unsigned same = __match_any_sync(0xffffffffu, e);
         const int rank = __popc(same & lt);
         if (valid && rank == 0) s_wc[warp][e] = __popc(same);
         __syncthreads();
-        if (tid < E) {
-            int run = s_run[tid];
-            for (int w = 0; w < NWARPS; ++w) {
-                const int c = s_wc[w][tid];
-                s_wc[w][tid] = run;
-                run += c;
+        int pre = 0, own = 0;  // lane l < E: expert l's rows in this CTA before this warp's rows
+        if (lane < E) {
+            pre = s_run[lane];
+            for (int w = 0; w < warp; ++w) pre += s_wc[w][lane];
+            own = s_wc[warp][lane];
+        }
+        const int base_e = __shfl_sync(0xffffffffu, pre, valid ? e : 0);
+        if (valid) set_info(i, (uint32_t)e | ((uint32_t)(base_e + rank) << 8));
+        __syncthreads();  // every warp has read s_run and s_wc
+        if (warp == NWARPS - 1 && lane < E) s_run[lane] = pre + own;
+    }
+
+    // ---------------- bounded wait for every CTA's row. Thread t takes rows t, t + NTHREADS, ...;
+    // a row is read with 16-byte loads (its words issued together: one round trip), added to
+    // the sums over the CTAs before this one and over all CTAs once all its words carry this
+    // launch's tag, and not read again, so later polls touch only the rows still missing.
+    // `arrivals` rows are awaited (more than the grid only in fault tests).
+    int before[CM_MAX_E], total[CM_MAX_E];
+#pragma unroll
+    for (int e = 0; e < CM_MAX_E; ++e) before[e] = total[e] = 0;
+    {
+        const uint64_t t0 = globaltimer();
+        uint32_t done = 0;  // bit j: row tid + j * NTHREADS has been added
+        while (true) {
+            int ok = 1;
+            for (int j = 0, b = tid; b < (int)a.arrivals; ++j, b += NTHREADS) {
+                if ((done >> j) & 1u) continue;
+                const unsigned long long* row = a.cta_words + (size_t)b * CM_MAX_E;
+                unsigned long long w[CM_MAX_E];
+#pragma unroll
+                for (int q = 0; q < CM_MAX_E / 2; ++q)
+                    if (2 * q < E)
+                        asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];"
+                                     : "=l"(w[2 * q]), "=l"(w[2 * q + 1])
+                                     : "l"(row + 2 * q)
+                                     : "memory");
+                bool valid = true;
+#pragma unroll
+                for (int e = 0; e < CM_MAX_E; ++e)
+                    if (e < E && (uint32_t)(w[e] >> 32) != tag) valid = false;
+                if (!valid) {
+                    ok = 0;
+                    continue;
+                }
+                done |= 1u << j;
+#pragma unroll
+                for (int e = 0; e < CM_MAX_E; ++e) {
+                    if (e < E) {
+                        const int c = (int)(uint32_t)w[e];
+                        total[e] += c;
+                        if (b < (int)blockIdx.x) before[e] += c;
+                    }
+                }
             }
-            s_run[tid] = run;
+            if (__syncthreads_and(ok)) break;
+            if (tid == 0 && globaltimer() - t0 > (uint64_t)a.wait_limit_ns) s_abort = 1;
+            __syncthreads();
+            if (s_abort) {
+                if (tid == 0) {
+                    set_status(a.status, CLEARMOE_ETIMEOUT);
+                    atomicMax(a.epoch, ep0 + 1);  // this launch's tag is spent
+                }
+                return;
+            }
+            __nanosleep(64);
         }
-        __syncthreads();
-        if (valid) {
-            const int slot = s_base[e] + s_wc[warp][e] + rank;
-            a.perm[slot] = (int32_t)(row0 + i);
-            if (a.inv) a.inv[row0 + i] = slot;
+    }
+    if (blockIdx.x == 0 && tid == 0) atomicMax(a.epoch, ep0 + 1);  // every CTA has read the epoch
+    if (s_abort) return;  // a wait of phase 1 gave up (status already set)
+
+    // ---------------- phase 2: global offsets, then this CTA's slots in token order. Sums by warp
+    // shuffles, per-warp partials in shared memory, then warp 0 lane e adds expert e's partials
+    // and scans the totals over experts.
+#pragma unroll
+    for (int e = 0; e < CM_MAX_E; ++e) {
+        if (e < E) {
+            const int vb = __reduce_add_sync(0xffffffffu, before[e]);
+            const int vt = __reduce_add_sync(0xffffffffu, total[e]);
+            if (lane == 0) {
+                s_wc[warp][e] = vb;
+                s_part[warp][e] = vt;
+            }
         }
-        __syncthreads();
+    }
+    __syncthreads();
+    if (warp == 0) {
+        int bef = 0, tot = 0;
+        if (lane < E) {
+            for (int w = 0; w < NWARPS; ++w) {
+                bef += s_wc[w][lane];
+                tot += s_part[w][lane];
+            }
+        }
+        int incl = tot;  // inclusive scan of the totals over experts (lanes)
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += v;
+        }
+        if (lane < E) {
+            s_base[lane] = incl - tot + bef;
+            if (blockIdx.x == 0) {
+                a.counts[lane] = tot;
+                a.offsets[lane] = incl - tot;
+                if (lane == E - 1) a.offsets[E] = incl;
+            }
+        }
+    }
+    __syncthreads();
+    for (int i = tid; i < nrows; i += NTHREADS) {
+        const uint32_t v = info_of(i);  // this thread's own word from the ranking pass
+        const int e = (int)(v & 0xffu);
+        const int slot = s_base[e] + (int)(v >> 8);
+        a.perm[slot] = (int32_t)(row0 + i);
+        if (a.inv) a.inv[row0 + i] = slot;
+        if (!sinfo) a.idx[row0 + i] = e;
     }
 }
 
-int route_max_ctas(int num_sms, int, int, int) { return num_sms * 8; }
+// At most 32 rows of the histogram exchange per thread (a 32-bit mask of rows read).
+int route_max_ctas(int num_sms, int, int, int) { return min(num_sms * 8, 32 * RT_THREADS); }
 
 int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* chunk) {
     const bool bf16 = dtype == CLEARMOE_BF16;
@@ -402,6 +507,7 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
         ch = ((T + want - 1) / want + 15) / 16 * 16;
     }
     if (ch < 16) ch = 16;
+    if (ch >= ((int64_t)1 << 24)) return -2;  // a row's local rank must fit in 24 bits
     *chunk = (int)ch;
     *grid = (int)((T + ch - 1) / ch);
     return 0;
