@@ -6,8 +6,9 @@ experts with the scatter) over one batch of synthetic ViT tokens, through the li
 The default workload is the DeiT-B / ViT-B-shaped layer (T = 256 images x 197 tokens = 50,432,
 d = 768, H = 3,072, E = 8, r = 128, bf16), the shape the GEMM target is quoted on.
 
-  value  tokens/s over K timed steps (inputs resident in HBM), CUDA events on the launch stream,
-         L2 flushed (a 256 MB write) before every step, outside the timed events
+  value  tokens/s over K timed steps (inputs resident in HBM), CUDA events on the launch stream
+         around each step only, L2 flushed (a 256 MB write) before every step, outside the events
+  stages per-kernel durations from a second pass with an event between consecutive kernels
   e2e    the same call with x copied from pinned host memory and out copied back inside each step
   roofline  the dominant kernel's algorithmic FLOPs (or bytes) per launch / its event-timed duration
   cpu_baseline  the float64 CPU oracle on a bounded sample of the same workload (rank 0, N = 1)
@@ -35,16 +36,18 @@ METRIC = ("CLEAR-MoE FFN tokens/sec/layer (1×GB300) + % HBM peak (dispatch), "
           "% tensor peak (GEMMs)")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 STAGES = ("route", "fc1_gelu", "basis", "grouped")
-KERNEL_OF_STAGE = {"route": "route_kernel", "fc1_gelu": "tc_gemm_kernel<256, gather>",
-                   "basis": "tc_gemm_kernel<128, dense>", "grouped": "tc_gemm_kernel<256, grouped>"}
+KERNEL_OF_STAGE = {"route": "cm::route_kernel<1>",
+                   "fc1_gelu": "cm::tc_gemm2_kernel<0> (2-SM dense, rows stored at inv[token])",
+                   "basis": "cm::tc_gemm_kernel<128, 0>",
+                   "grouped": "cm::tc_gemm2_kernel<2> (2-SM grouped, rows stored at perm[slot])"}
 # DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from the committed ncu
 # capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel sources
 # it was taken on; a different hash means the kernels changed and the figure is void.
 TRAFFIC = {
-    "route": {"bytes": 78.453760e6, "src": "669263211c688d5d"},
-    "fc1_gelu": {"bytes": 337.098752e6, "src": "669263211c688d5d"},
-    "basis": {"bytes": 321.049856e6, "src": "669263211c688d5d"},
-    "grouped": {"bytes": 423.497728e6, "src": "669263211c688d5d"},
+    "route": {"bytes": 78.336768e6, "src": "5d42463a6e4f5296"},
+    "fc1_gelu": {"bytes": 337.993216e6, "src": "5d42463a6e4f5296"},
+    "basis": {"bytes": 321.057536e6, "src": "5d42463a6e4f5296"},
+    "grouped": {"bytes": 426.601728e6, "src": "5d42463a6e4f5296"},
 }
 
 
@@ -259,8 +262,11 @@ def main():
     torch.cuda.synchronize()
     assert cm.clearmoe_layer_status(h) == 0
 
+    # Headline: K forwards, each bracketed by events on the launching stream and nothing between
+    # its kernels (an event between two launches would cancel the programmatic launch overlap of
+    # the GEMM kernels). The L2 flush before each step lies outside the events.
     K = args.steps
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
@@ -268,36 +274,49 @@ def main():
         wall0 = time.perf_counter()
         for k in range(K):
             flush.zero_()
-            cm.clearmoe_set_profile_events(h, ev[k])
+            ev[k][0].record(stream)
             forward()
+            ev[k][1].record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - wall0
-    cm.clearmoe_set_profile_events(h, [])
     if dist:
         dist.barrier()
     assert cm.clearmoe_layer_status(h) == 0
-    stage_ms = {st: [ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)]
-                for i, st in enumerate(STAGES)}
-    step_ms = [ev[k][0].elapsed_time(ev[k][4]) for k in range(K)]
+    step_ms = [ev[k][0].elapsed_time(ev[k][1]) for k in range(K)]
     total_ms = float(sum(step_ms))
+
+    # Per-kernel durations (roofline, stage breakdown): a second timed pass with an event between
+    # consecutive kernels, recorded by the library on the launching stream.
+    Ks = min(K, 300)
+    sev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(Ks)]
+    torch.cuda.synchronize()
+    for k in range(Ks):
+        flush.zero_()
+        cm.clearmoe_set_profile_events(h, sev[k])
+        forward()
+    torch.cuda.synchronize()
+    cm.clearmoe_set_profile_events(h, [])
+    assert cm.clearmoe_layer_status(h) == 0
+    stage_ms = {st: [sev[k][i].elapsed_time(sev[k][i + 1]) for k in range(Ks)]
+                for i, st in enumerate(STAGES)}
     if dist:
         t = torch.tensor([total_ms], device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         total_ms = float(t.item())
     value = world * s.T * K / (total_ms / 1e3)
 
-    # same-GPU dense FFN, same timing rules
-    dense_ms = []
+    # same-GPU dense FFN, same timing rules (events around each forward only)
     dout = torch.empty_like(out)
-    dev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(min(K, 200))]
+    dev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(min(K, 300))]
     for k in range(len(dev) + args.warmup):
         flush.zero_()
         if k >= args.warmup:
-            cm.clearmoe_set_profile_events(h, dev[k - args.warmup])
+            dev[k - args.warmup][0].record(stream)
         cm.clearmoe_dense_ffn_forward(h, D["x"], D["W1"], D["b1"], D["W2"], dout)
+        if k >= args.warmup:
+            dev[k - args.warmup][1].record(stream)
     torch.cuda.synchronize()
-    cm.clearmoe_set_profile_events(h, [])
-    dense_ms = [e[0].elapsed_time(e[2]) for e in dev]
+    dense_ms = [e[0].elapsed_time(e[1]) for e in dev]
     dense_value = s.T / (statistics.mean(dense_ms) / 1e3)
 
     # End to end through the C ABI with host buffers: every step copies its tokens from pinned
@@ -414,6 +433,8 @@ def main():
         "cpu_baseline": cpu,
         "clocks": clk.summary(),
         "stages": per_stage,
+        "stage_timing": f"separate pass of {Ks} steps with an event between consecutive kernels "
+                        "(which also cancels their programmatic launch overlap)",
         "layer_roofline_frac": layer_roofline_s(s, pk) / (mean_step / 1e3),
         "dense_ffn": {"value": dense_value, "unit": "tokens/s",
                       "ms_per_step": statistics.mean(dense_ms)},

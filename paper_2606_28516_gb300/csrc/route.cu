@@ -116,6 +116,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     __shared__ int s_abort;
     __shared__ uint32_t s_tag;
 
+    pdl_launch_dependents();  // the GEMM that follows may set itself up meanwhile
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int E = a.E, d = a.d;
     const int64_t row0 = (int64_t)blockIdx.x * chunk;

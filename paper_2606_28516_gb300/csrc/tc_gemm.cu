@@ -81,6 +81,7 @@ __device__ __forceinline__ TileInfo decode_tile(const TcGemmArgs& a, int tile, i
 template <int BN, int MODE>
 __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THREADS_TMA, 1)
     tc_gemm_kernel(const __grid_constant__ TcGemmArgs a) {
+    pdl_launch_dependents();
     using C = TcCfg<BN>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
@@ -116,7 +117,16 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
         }
         mbar_init(drain_bar, 1);
         *abort_flag = 0;
-        if (MODE == TC_GROUPED) {
+        mbar_fence_init();
+    }
+    if (warp == TC_WARP_MMA) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    // everything above overlaps the predecessor kernel; from here on its results are read
+    pdl_wait();
+    if (MODE == TC_GROUPED) {
+        if (threadIdx.x == 0) {
             int acc = 0;
             for (int e = 0; e < a.E; ++e) {
                 s_prefix[e] = acc;
@@ -124,12 +134,8 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
             }
             s_prefix[a.E] = acc;
         }
-        mbar_fence_init();
+        __syncthreads();
     }
-    if (warp == TC_WARP_MMA) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
     int m_tiles;
@@ -375,8 +381,17 @@ static cudaError_t launch_one(const TcGemmArgs& a, int num_sms, cudaStream_t s) 
     int64_t tiles = m_tiles * n_tiles;
     const int grid = (int)(tiles < num_sms ? tiles : num_sms);
     if (grid <= 0) return cudaSuccess;
-    tc_gemm_kernel<BN, MODE><<<grid, MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THREADS_TMA, C::SMEM, s>>>(a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THREADS_TMA);
+    cfg.dynamicSmemBytes = C::SMEM;
+    cfg.stream = s;
+    cudaLaunchAttribute attr_pdl[1];
+    attr_pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr_pdl[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr_pdl;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, tc_gemm_kernel<BN, MODE>, a);
 }
 
 template <int MODE>

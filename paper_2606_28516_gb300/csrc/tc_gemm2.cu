@@ -118,6 +118,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* s_prefix = reinterpret_cast<int*>(tmem_slot + 4);  // [CM_MAX_E + 1]
 
+    pdl_launch_dependents();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = cluster_rank();
     const bool leader = rank == 0;
@@ -145,14 +146,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
         }
         mbar_init(drain_bar, 1);
         *abort_flag = 0;
-        if (MODE == TC_GROUPED) {
-            int acc = 0;
-            for (int e = 0; e < a.E; ++e) {
-                s_prefix[e] = acc;
-                acc += (a.offsets[e + 1] - a.offsets[e] + 2 * BM - 1) / (2 * BM);
-            }
-            s_prefix[a.E] = acc;
-        }
         mbar_fence_init();
     }
     // Tensor memory for the pair: allocated collectively by one warp of each CTA. The two CTAs
@@ -167,6 +160,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
     __syncthreads();
     cluster_sync();  // barriers initialised and TMEM bases written in both CTAs
     tc_fence_after();
+    // everything above overlaps the predecessor kernel; from here on its results are read
+    pdl_wait();
+    if (MODE == TC_GROUPED) {
+        if (threadIdx.x == 0) {
+            int acc = 0;
+            for (int e = 0; e < a.E; ++e) {
+                s_prefix[e] = acc;
+                acc += (a.offsets[e + 1] - a.offsets[e] + 2 * BM - 1) / (2 * BM);
+            }
+            s_prefix[a.E] = acc;
+        }
+        __syncthreads();
+    }
     const uint32_t tmem_base = *tmem_slot;
     uint32_t peer_base;
     asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(peer_base) : "r"(map_to_rank(smem_u32(tmem_slot), rank ^ 1)));
@@ -383,12 +389,18 @@ cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     const int64_t units = m_pairs * n_tiles;
     int64_t clusters = units < num_sms / 2 ? units : num_sms / 2;
     if (clusters <= 0) return cudaSuccess;
-    const dim3 grid((unsigned)(2 * clusters));
-    if (a.mode == TC_GROUPED)
-        tc_gemm2_kernel<TC_GROUPED><<<grid, t2::THREADS, t2::SMEM, s>>>(a);
-    else
-        tc_gemm2_kernel<TC_DENSE><<<grid, t2::THREADS, t2::SMEM, s>>>(a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(2 * clusters));
+    cfg.blockDim = dim3(t2::THREADS);
+    cfg.dynamicSmemBytes = t2::SMEM;
+    cfg.stream = s;
+    cudaLaunchAttribute attr_pdl[1];
+    attr_pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr_pdl[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr_pdl;
+    cfg.numAttrs = 1;
+    if (a.mode == TC_GROUPED) return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<TC_GROUPED>, a);
+    return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<TC_DENSE>, a);
 }
 
 }  // namespace cm
