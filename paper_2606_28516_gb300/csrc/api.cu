@@ -281,7 +281,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g.bias = b1;
     g.C = L->z;
     g.ldc = H;
-    if (cm::tc2_supported(cm::TC_DENSE, H)) {
+    if (cm::tc2_supported(cm::TC_DENSE, H) && H <= cm::TC2_BIAS_CAP) {
         if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, 128))
             return CLEARMOE_ECUDA;
         g.mode = cm::TC_DENSE;
@@ -392,7 +392,8 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     std::memset(&g, 0, sizeof(g));
     g.status = L->status;
     g.wait_limit_ns = L->wait_limit_ns;
-    const bool pair1 = cm::tc2_supported(cm::TC_DENSE, H), pair2 = cm::tc2_supported(cm::TC_DENSE, d);
+    const bool pair1 = cm::tc2_supported(cm::TC_DENSE, H) && H <= cm::TC2_BIAS_CAP;
+    const bool pair2 = cm::tc2_supported(cm::TC_DENSE, d);
     if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, pair1 ? 128 : bn1))
         return CLEARMOE_ECUDA;
     g.mode = cm::TC_DENSE;

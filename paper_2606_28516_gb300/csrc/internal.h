@@ -88,7 +88,9 @@ struct TcGemmArgs {
     int tmem_cols;  // 2-SM kernel: tensor-memory columns per CTA (256: one accumulator, 512: two)
 };
 int tc_pick_bn(int mode, int N);
-// 2-SM (cta_group::2) variant for the dense and grouped modes, 256 x 256 tiles per CTA pair.
+// 2-SM (cta_group::2) variant for the dense and grouped modes, 256 x 256 tiles per CTA pair; its
+// bias + GELU epilogue stages the bias in shared memory, for N <= TC2_BIAS_CAP.
+constexpr int TC2_BIAS_CAP = 4096;
 bool tc2_supported(int mode, int N);
 cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_tc_gemm(const TcGemmArgs& a, int num_sms, cudaStream_t s);

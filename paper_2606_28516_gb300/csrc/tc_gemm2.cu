@@ -33,10 +33,13 @@ constexpr int THREADS = 32 * (WARP_TMA + 1);
 constexpr int WCOLS = BN / (NUM_EPI / 4);      // columns per epilogue warp
 constexpr int CW = 32;                         // columns per tensor-memory read
 constexpr int SW = 16;                         // columns per staged store pass
-constexpr int STG_ROW = SW * 2 + 16;           // 48-byte rows: conflict-free 16-byte writes
+// Staging: 32-byte rows (16 bf16); the two 16-byte chunks of row r swap places when bit 2 of r is
+// set, which makes both the row-wise writes and the 2-lanes-per-row reads conflict-free.
+constexpr int STG_ROW = SW * 2;
 constexpr int STG_BYTES = NUM_EPI * 32 * STG_ROW;
+constexpr int BIAS_CAP = TC2_BIAS_CAP;         // fp32 bias staged in shared memory (N <= BIAS_CAP)
 constexpr int NBARS = 2 * STAGES + 5;
-constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + NBARS * 8 + 128;
+constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + BIAS_CAP * 4 + NBARS * 8 + 128;
 }  // namespace t2
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -113,7 +116,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
     const uint32_t raw_addr = smem_u32(smem_raw);
     unsigned char* sm = smem_raw + ((1024 - (raw_addr & 1023)) & 1023);
     unsigned char* stg = sm + STAGES * STAGE_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(stg + STG_BYTES);
+    float* s_bias = reinterpret_cast<float*>(stg + STG_BYTES);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(s_bias + BIAS_CAP);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NBARS);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* s_prefix = reinterpret_cast<int*>(tmem_slot + 4);  // [CM_MAX_E + 1]
@@ -147,6 +151,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
         mbar_init(drain_bar, 1);
         *abort_flag = 0;
         mbar_fence_init();
+    }
+    // The bias (a weight, not produced by the previous kernel) as fp32, once per CTA.
+    if (MODE == TC_DENSE && a.epi == TC_EPI_BIAS_GELU && warp < NUM_EPI) {
+        const uint16_t* b = static_cast<const uint16_t*>(a.bias);
+        for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = __uint_as_float((uint32_t)b[n] << 16);
     }
     // Tensor memory for the pair: allocated collectively by one warp of each CTA. The two CTAs
     // must see the same base (the even CTA's MMAs name it for both); a mismatch aborts cleanly.
@@ -315,36 +324,37 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
                 for (int j = 0; j < CW; ++j) f[j] = __uint_as_float(v[j]);
                 const int nb = t.n0 + c;
                 if (a.epi == TC_EPI_BIAS_GELU) {
-                    const uint4* bp = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.bias) + nb);
+                    const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
 #pragma unroll
-                    for (int j8 = 0; j8 < CW / 8; ++j8) {
-                        const uint4 b = __ldg(bp + j8);
-                        const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-                        for (int h = 0; h < 4; ++h) {
-                            const float2 g = gelu_pair_as(
-                                __fadd2_rn(make_float2(f[j8 * 8 + 2 * h], f[j8 * 8 + 2 * h + 1]),
-                                           make_float2(bf16_lo(bw[h]), bf16_hi(bw[h]))));
-                            f[j8 * 8 + 2 * h] = g.x;
-                            f[j8 * 8 + 2 * h + 1] = g.y;
-                        }
+                    for (int j4 = 0; j4 < CW / 4; ++j4) {
+                        const float4 b = bp[j4];
+                        const float2 g0 = gelu_pair_as(
+                            __fadd2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), make_float2(b.x, b.y)));
+                        const float2 g1 = gelu_pair_as(
+                            __fadd2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), make_float2(b.z, b.w)));
+                        f[4 * j4] = g0.x;
+                        f[4 * j4 + 1] = g0.y;
+                        f[4 * j4 + 2] = g1.x;
+                        f[4 * j4 + 3] = g1.y;
                     }
                 }
 #pragma unroll
                 for (int s0 = 0; s0 < CW; s0 += SW) {
-                    uint4* dst = reinterpret_cast<uint4*>(wstg + lane * STG_ROW);
+                    unsigned char* dst = wstg + lane * STG_ROW;
 #pragma unroll
                     for (int j8 = 0; j8 < SW / 8; ++j8) {
                         const float* g = f + s0 + 8 * j8;
-                        dst[j8] = make_uint4(pack_bf16(g[0], g[1]), pack_bf16(g[2], g[3]), pack_bf16(g[4], g[5]),
-                                             pack_bf16(g[6], g[7]));
+                        *reinterpret_cast<uint4*>(dst + ((j8 ^ ((lane >> 2) & 1)) << 4)) =
+                            make_uint4(pack_bf16(g[0], g[1]), pack_bf16(g[2], g[3]), pack_bf16(g[4], g[5]),
+                                       pack_bf16(g[6], g[7]));
                     }
                     __syncwarp();
 #pragma unroll
                     for (int p = 0; p < LPR; ++p) {
                         const int rr = p * RPP + lane / LPR;
                         const int64_t o = __shfl_sync(0xffffffffu, orow, rr);
-                        const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * STG_ROW + (lane % LPR) * 16);
+                        const int ch = (lane % LPR) ^ ((rr >> 2) & 1);
+                        const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * STG_ROW + ch * 16);
                         if (o >= 0)
                             *reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.C) + o * a.ldc + nb + s0 +
                                                       (lane % LPR) * 8) = val;
@@ -371,10 +381,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
                      : "memory");
 }
 
+// (a dense launch with the bias + GELU epilogue also needs N <= BIAS_CAP; launch_tc_gemm2 rejects
+// a larger one)
 bool tc2_supported(int mode, int N) { return (mode == TC_DENSE || mode == TC_GROUPED) && N % t2::BN == 0; }
 
 cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
-    if (!tc2_supported(a.mode, a.N) || a.epi == TC_EPI_SCALE || (a.tmem_cols != 256 && a.tmem_cols != 512))
+    if (!tc2_supported(a.mode, a.N) || a.epi == TC_EPI_SCALE || (a.tmem_cols != 256 && a.tmem_cols != 512) ||
+        (a.epi == TC_EPI_BIAS_GELU && (a.mode != TC_DENSE || a.N > t2::BIAS_CAP)))
         return cudaErrorInvalidValue;
     static bool attr[3] = {false, false, false};
     const void* fn = a.mode == TC_GROUPED ? (const void*)tc_gemm2_kernel<TC_GROUPED> : (const void*)tc_gemm2_kernel<TC_DENSE>;
