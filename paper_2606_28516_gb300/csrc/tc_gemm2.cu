@@ -27,7 +27,7 @@ constexpr int A_BYTES = BM * BK * 2;           // 16 KB
 constexpr int B_BYTES = BH * BK * 2;           // 16 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES; // 32 KB
 constexpr int STAGES = 6;
-constexpr int NUM_EPI = 16;                    // four per TMEM lane quarter
+constexpr int NUM_EPI = 8;                     // two per TMEM lane quarter
 constexpr int WARP_MMA = NUM_EPI, WARP_TMA = NUM_EPI + 1;
 constexpr int THREADS = 32 * (WARP_TMA + 1);
 constexpr int WCOLS = BN / (NUM_EPI / 4);      // columns per epilogue warp
@@ -313,6 +313,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
             const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
             int64_t orow = -1;
             if (mrow < t.hi) orow = a.rows ? (int64_t)a.rows[mrow] : mrow;
+            // this lane stores rows p * RPP + lane / LPR of the warp's 32 (p < LPR), 16-byte chunk
+            // lane % LPR: their destinations, once per tile
+            uint16_t* dst_row[LPR];
+#pragma unroll
+            for (int p = 0; p < LPR; ++p) {
+                const int64_t o = __shfl_sync(0xffffffffu, orow, p * RPP + lane / LPR);
+                dst_row[p] = o >= 0 ? static_cast<uint16_t*>(a.C) + o * a.ldc + t.n0 + (lane % LPR) * 8 : nullptr;
+            }
             for (int c = c_lo; c < c_lo + WCOLS; c += CW) {
                 uint32_t v[CW];
                 const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
@@ -352,12 +360,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
 #pragma unroll
                     for (int p = 0; p < LPR; ++p) {
                         const int rr = p * RPP + lane / LPR;
-                        const int64_t o = __shfl_sync(0xffffffffu, orow, rr);
                         const int ch = (lane % LPR) ^ ((rr >> 2) & 1);
                         const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * STG_ROW + ch * 16);
-                        if (o >= 0)
-                            *reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.C) + o * a.ldc + nb + s0 +
-                                                      (lane % LPR) * 8) = val;
+                        if (dst_row[p]) *reinterpret_cast<uint4*>(dst_row[p] + (c + s0)) = val;
                     }
                     __syncwarp();
                 }

@@ -69,6 +69,17 @@ def test_kernel_horner_form_is_exact():
     assert np.array_equal(_poly_kernel(m), -_poly_plain(au))
 
 
+def test_relu_as_half_sum_is_exact():
+    """The kernel forms max(u, 0) as the fma u * 0.5 + |u| / 2 (m = -|u| / 2 negated): exact
+    wherever halving is (|u| >= 2^-125; below that GELU(u) rounds to zero in bf16 anyway)."""
+    rng = np.random.default_rng(5)
+    u = np.concatenate([rng.standard_normal(500_000) * 10.0 ** rng.integers(-30, 30, 500_000),
+                        [0.0, -0.0, 2.0 ** -125, -(2.0 ** -125), 3.4e38, -3.4e38]]).astype(np.float32)
+    m = (np.float32(-0.5) * np.abs(u)).astype(np.float32)
+    r = _fma32(np.full_like(u, 0.5), u, -m)
+    assert np.array_equal(r + np.float32(0), np.maximum(u, np.float32(0)) + np.float32(0))
+
+
 def test_bf16_rounding_agrees_on_realistic_preactivations():
     torch = __import__("pytest").importorskip("torch")
     u = (np.random.default_rng(0).standard_normal(2_000_000) * 0.6).astype(np.float32)
