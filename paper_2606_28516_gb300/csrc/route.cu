@@ -102,7 +102,11 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
                  : "memory");
 }
 
-template <bool BF16>
+// W_g's B fragments held in registers (bf16, E <= 8, d <= RT_WREG_D): 4 registers per 32 columns
+constexpr int RT_WREG_D = 768;
+inline bool route_wreg(int dtype, int d, int E) { return dtype == CLEARMOE_BF16 && E <= 8 && d <= RT_WREG_D; }
+
+template <bool BF16, bool WREG>
 __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_kernel(const RouteArgs a, const int chunk) {
     constexpr int NTHREADS = BF16 ? RT_BF16_THREADS : RT_THREADS;
     constexpr int NWARPS = NTHREADS / 32;
@@ -207,6 +211,12 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                               ? reinterpret_cast<const uint4*>(smem + (size_t)(nt * 8 + g) * WRB + tig * 16)
                               : nullptr;
             const bool w_ok = nstages == 0 || mbar_wait(wbar, 0, abort_flag, a.status, (uint64_t)a.wait_limit_ns);
+            constexpr int NWC = WREG ? RT_WREG_D / 32 : 1;  // register copy of the fragments (WREG)
+            uint4 wreg[NWC];
+            if constexpr (WREG) {
+#pragma unroll
+                for (int c = 0; c < NWC; ++c) wreg[c] = (c < nchunk && wfr[0] && w_ok) ? wfr[0][4 * c] : zero;
+            }
             for (int k = warp; w_ok && k < nstages; k += S) {
                 const int s = warp;
                 if (!mbar_wait(full_bar(s), (k / S) & 1, abort_flag, a.status, (uint64_t)a.wait_limit_ns)) break;
@@ -223,18 +233,33 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                     for (int q = 0; q < 4; ++q)
 #pragma unroll
                         for (int i = 0; i < 4; ++i) part[nt][q][i] = 0.f;
-                for (int c = 0; c < nchunk; c += 2) {  // d % 64 == 0: nchunk is even
-                    const uint4 xa0 = vA ? pA[4 * c] : zero, xa1 = vA ? pA[4 * c + 4] : zero;
-                    const uint4 xb0 = vB ? pB[4 * c] : zero, xb1 = vB ? pB[4 * c + 4] : zero;
+                if constexpr (WREG) {
 #pragma unroll
-                    for (int nt = 0; nt < 2; ++nt) {
-                        if (nt < NT) {
-                            const uint4 w0 = wfr[nt] ? wfr[nt][4 * c] : zero;
-                            const uint4 w1 = wfr[nt] ? wfr[nt][4 * c + 4] : zero;
-                            mma_bf16_16816(part[nt][0], xa0.x, xb0.x, xa0.y, xb0.y, w0.x, w0.y);
-                            mma_bf16_16816(part[nt][1], xa0.z, xb0.z, xa0.w, xb0.w, w0.z, w0.w);
-                            mma_bf16_16816(part[nt][2], xa1.x, xb1.x, xa1.y, xb1.y, w1.x, w1.y);
-                            mma_bf16_16816(part[nt][3], xa1.z, xb1.z, xa1.w, xb1.w, w1.z, w1.w);
+                    for (int c = 0; c < NWC; c += 2) {  // one n-tile, fragments in registers
+                        if (c < nchunk) {
+                            const uint4 xa0 = vA ? pA[4 * c] : zero, xa1 = vA ? pA[4 * c + 4] : zero;
+                            const uint4 xb0 = vB ? pB[4 * c] : zero, xb1 = vB ? pB[4 * c + 4] : zero;
+                            const uint4 w0 = wreg[c], w1 = wreg[c + 1];
+                            mma_bf16_16816(part[0][0], xa0.x, xb0.x, xa0.y, xb0.y, w0.x, w0.y);
+                            mma_bf16_16816(part[0][1], xa0.z, xb0.z, xa0.w, xb0.w, w0.z, w0.w);
+                            mma_bf16_16816(part[0][2], xa1.x, xb1.x, xa1.y, xb1.y, w1.x, w1.y);
+                            mma_bf16_16816(part[0][3], xa1.z, xb1.z, xa1.w, xb1.w, w1.z, w1.w);
+                        }
+                    }
+                } else {
+                    for (int c = 0; c < nchunk; c += 2) {  // d % 64 == 0: nchunk is even
+                        const uint4 xa0 = vA ? pA[4 * c] : zero, xa1 = vA ? pA[4 * c + 4] : zero;
+                        const uint4 xb0 = vB ? pB[4 * c] : zero, xb1 = vB ? pB[4 * c + 4] : zero;
+#pragma unroll
+                        for (int nt = 0; nt < 2; ++nt) {
+                            if (nt < NT) {
+                                const uint4 w0 = wfr[nt] ? wfr[nt][4 * c] : zero;
+                                const uint4 w1 = wfr[nt] ? wfr[nt][4 * c + 4] : zero;
+                                mma_bf16_16816(part[nt][0], xa0.x, xb0.x, xa0.y, xb0.y, w0.x, w0.y);
+                                mma_bf16_16816(part[nt][1], xa0.z, xb0.z, xa0.w, xb0.w, w0.z, w0.w);
+                                mma_bf16_16816(part[nt][2], xa1.x, xb1.x, xa1.y, xb1.y, w1.x, w1.y);
+                                mma_bf16_16816(part[nt][3], xa1.z, xb1.z, xa1.w, xb1.w, w1.z, w1.w);
+                            }
                         }
                     }
                 }
@@ -479,10 +504,12 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
     std::lock_guard<std::mutex> lock(mu);
     static bool attr_set = false;
     if (!attr_set) {
-            if (cudaFuncSetAttribute((const void*)route_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            if (cudaFuncSetAttribute((const void*)route_kernel<true, false>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 220 * 1024) != cudaSuccess ||
+            cudaFuncSetAttribute((const void*)route_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  220 * 1024) != cudaSuccess ||
-            cudaFuncSetAttribute((const void*)route_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 220 * 1024) != cudaSuccess)
+            cudaFuncSetAttribute((const void*)route_kernel<false, false>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 220 * 1024) != cudaSuccess)
             return -1;
         attr_set = true;
     }
@@ -495,9 +522,11 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
         for (int i = 0; i < ncache; ++i)
             if (cache[i].dtype == dtype && cache[i].d == d && cache[i].E == E && cache[i].smem == smem) occ = cache[i].occ;
         if (occ < 0) {
+            const void* fn = !bf16 ? (const void*)route_kernel<false, false>
+                             : route_wreg(dtype, d, E) ? (const void*)route_kernel<true, true>
+                                                       : (const void*)route_kernel<true, false>;
             cudaError_t err = cudaOccupancyMaxActiveBlocksPerMultiprocessorWithFlags(
-                &occ, bf16 ? (const void*)route_kernel<true> : (const void*)route_kernel<false>,
-                bf16 ? RT_BF16_THREADS : RT_THREADS, smem, cudaOccupancyDefault);
+                &occ, fn, bf16 ? RT_BF16_THREADS : RT_THREADS, smem, cudaOccupancyDefault);
             if (err != cudaSuccess) return -1;
             if (ncache < 32) cache[ncache++] = {dtype, d, E, smem, occ};
         }
@@ -527,8 +556,9 @@ cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (bf16) return cudaLaunchKernelEx(&cfg, route_kernel<true>, a, chunk);
-    return cudaLaunchKernelEx(&cfg, route_kernel<false>, a, chunk);
+    if (!bf16) return cudaLaunchKernelEx(&cfg, route_kernel<false, false>, a, chunk);
+    if (route_wreg(a.dtype, a.d, a.E)) return cudaLaunchKernelEx(&cfg, route_kernel<true, true>, a, chunk);
+    return cudaLaunchKernelEx(&cfg, route_kernel<true, false>, a, chunk);
 }
 
 }  // namespace cm
