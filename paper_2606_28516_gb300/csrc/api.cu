@@ -281,12 +281,12 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g.bias = b1;
     g.C = L->z;
     g.ldc = H;
-    if (cm::tc2_supported(cm::TC_DENSE, H) && H <= cm::TC2_BIAS_CAP) {
-        if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, 128))
+    const int p1 = H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;  // 2-SM tile width
+    if (p1) {
+        if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, p1 / 2))
             return CLEARMOE_ECUDA;
         g.mode = cm::TC_DENSE;
         g.rows = L->inv;
-        g.tmem_cols = 512;
         rc = cuda_fail(cm::launch_tc_gemm2(g, L->num_sms, s));
     } else {
         if (encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
@@ -298,12 +298,13 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     }
     if (rc) return rc;
     mark(L, 2, s);
-    // t = diag(S_r) Vh_r z
+    // t = diag(S_r) Vh_r z (the 2-SM kernel when r is a multiple of 128: more of z in flight per SM)
     cm::TcGemmArgs g2;
     std::memset(&g2, 0, sizeof(g2));
     g2.status = L->status;
     g2.wait_limit_ns = L->wait_limit_ns;
-    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, Vh_r, r, H, bn2))
+    const int p2 = cm::tc2_pick_bn(cm::TC_DENSE, r);
+    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, Vh_r, r, H, p2 ? p2 / 2 : bn2))
         return CLEARMOE_ECUDA;
     g2.mode = cm::TC_DENSE;
     g2.epi = cm::TC_EPI_SCALE;
@@ -313,16 +314,17 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g2.scale = S_r;
     g2.C = L->t;
     g2.ldc = r;
-    if ((rc = cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s)))) return rc;
+    rc = cuda_fail(p2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
+    if (rc) return rc;
     mark(L, 3, s);
     // out[perm[slot]] = [t | z] [U_r | W_e^res]^T per expert sub-batch
     cm::TcGemmArgs g3;
     std::memset(&g3, 0, sizeof(g3));
     g3.status = L->status;
     g3.wait_limit_ns = L->wait_limit_ns;
-    // The 2-SM kernel loads half of each 256-column B tile per CTA of the pair: 128-row boxes.
-    const bool pair3 = cm::tc2_supported(cm::TC_GROUPED, d);
-    const int box3 = pair3 ? 128 : bn3;
+    // The 2-SM kernel loads half of each pair tile's B rows per CTA: boxes of p3 / 2 rows.
+    const int p3 = cm::tc2_pick_bn(cm::TC_GROUPED, d);
+    const int box3 = p3 ? p3 / 2 : bn3;
     if (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, box3) ||
         encode_tmap_bf16(&g3.tmA1, L->z, T, H, 128))
         return CLEARMOE_ECUDA;
@@ -339,12 +341,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g3.rows = L->perm;
     g3.C = out;
     g3.ldc = d;
-    if (pair3) {
-        g3.tmem_cols = 512;
-        rc = cuda_fail(cm::launch_tc_gemm2(g3, L->num_sms, s));
-    } else {
-        rc = cuda_fail(cm::launch_tc_gemm(g3, L->num_sms, s));
-    }
+    rc = cuda_fail(p3 ? cm::launch_tc_gemm2(g3, L->num_sms, s) : cm::launch_tc_gemm(g3, L->num_sms, s));
     mark(L, 4, s);
     return rc;
 }
@@ -392,9 +389,9 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     std::memset(&g, 0, sizeof(g));
     g.status = L->status;
     g.wait_limit_ns = L->wait_limit_ns;
-    const bool pair1 = cm::tc2_supported(cm::TC_DENSE, H) && H <= cm::TC2_BIAS_CAP;
-    const bool pair2 = cm::tc2_supported(cm::TC_DENSE, d);
-    if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, pair1 ? 128 : bn1))
+    const int pair1 = H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;  // 2-SM tile widths
+    const int pair2 = cm::tc2_pick_bn(cm::TC_DENSE, d);
+    if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, pair1 ? pair1 / 2 : bn1))
         return CLEARMOE_ECUDA;
     g.mode = cm::TC_DENSE;
     g.epi = cm::TC_EPI_BIAS_GELU;
@@ -404,7 +401,6 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     g.bias = b1;
     g.C = L->z;
     g.ldc = H;
-    g.tmem_cols = 512;
     if ((rc = cuda_fail(pair1 ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s))))
         return rc;
     mark(L, 1, s);
@@ -412,7 +408,7 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     std::memset(&g2, 0, sizeof(g2));
     g2.status = L->status;
     g2.wait_limit_ns = L->wait_limit_ns;
-    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, W2, d, H, pair2 ? 128 : bn2))
+    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, W2, d, H, pair2 ? pair2 / 2 : bn2))
         return CLEARMOE_ECUDA;
     g2.mode = cm::TC_DENSE;
     g2.epi = cm::TC_EPI_STORE;
@@ -421,7 +417,6 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     g2.K0 = H;
     g2.C = out;
     g2.ldc = d;
-    g2.tmem_cols = 512;
     rc = cuda_fail(pair2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
     mark(L, 2, s);
     return rc;

@@ -85,13 +85,13 @@ struct TcGemmArgs {
     int64_t ldc;
     int32_t* status;
     int64_t wait_limit_ns;
-    int tmem_cols;  // 2-SM kernel: tensor-memory columns per CTA (256: one accumulator, 512: two)
 };
 int tc_pick_bn(int mode, int N);
-// 2-SM (cta_group::2) variant for the dense and grouped modes, 256 x 256 tiles per CTA pair; its
-// bias + GELU epilogue stages the bias in shared memory, for N <= TC2_BIAS_CAP.
+// 2-SM (cta_group::2) variant for the dense and grouped modes: 256 x BN tiles per CTA pair, BN =
+// tc2_pick_bn(mode, N) (256 or 128; 0 = shape not supported; each CTA's B box is BN / 2 rows).
+// Its bias + GELU and column-scale epilogues stage the vector in shared memory (N <= TC2_BIAS_CAP).
 constexpr int TC2_BIAS_CAP = 4096;
-bool tc2_supported(int mode, int N);
+int tc2_pick_bn(int mode, int N);
 cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_tc_gemm(const TcGemmArgs& a, int num_sms, cudaStream_t s);
 

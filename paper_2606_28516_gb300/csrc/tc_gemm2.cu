@@ -18,29 +18,32 @@
 #include "internal.h"
 
 namespace cm {
-namespace t2 {
-constexpr int BM = 128;                        // rows per CTA; the pair covers 256
-constexpr int BN = 256;                        // columns per pair tile
-constexpr int BH = BN / 2;                     // B rows per CTA
-constexpr int BK = 64;
-constexpr int A_BYTES = BM * BK * 2;           // 16 KB
-constexpr int B_BYTES = BH * BK * 2;           // 16 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES; // 32 KB
-constexpr int STAGES = 6;
-constexpr int NUM_EPI = 8;                     // two per TMEM lane quarter
-constexpr int WARP_MMA = NUM_EPI, WARP_TMA = NUM_EPI + 1;
-constexpr int THREADS = 32 * (WARP_TMA + 1);
-constexpr int WCOLS = BN / (NUM_EPI / 4);      // columns per epilogue warp
-constexpr int CW = 32;                         // columns per tensor-memory read
-constexpr int SW = 16;                         // columns per staged store pass
-// Staging: 32-byte rows (16 bf16); the two 16-byte chunks of row r swap places when bit 2 of r is
-// set, which makes both the row-wise writes and the 2-lanes-per-row reads conflict-free.
-constexpr int STG_ROW = SW * 2;
-constexpr int STG_BYTES = NUM_EPI * 32 * STG_ROW;
-constexpr int BIAS_CAP = TC2_BIAS_CAP;         // fp32 bias staged in shared memory (N <= BIAS_CAP)
-constexpr int NBARS = 2 * STAGES + 5;
-constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + BIAS_CAP * 4 + NBARS * 8 + 128;
-}  // namespace t2
+// Tile configuration by pair-tile width BN (256 or 128 columns).
+template <int BN_>
+struct T2 {
+    static constexpr int BM = 128;                        // rows per CTA; the pair covers 256
+    static constexpr int BN = BN_;                        // columns per pair tile
+    static constexpr int BH = BN / 2;                     // B rows per CTA
+    static constexpr int BK = 64;
+    static constexpr int A_BYTES = BM * BK * 2;           // 16 KB
+    static constexpr int B_BYTES = BH * BK * 2;           // 16 KB (BN 256) / 8 KB (BN 128)
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int STAGES = BN == 256 ? 6 : 8;      // 192 KB of operands either way
+    static constexpr int NUM_EPI = 8;                     // two per TMEM lane quarter
+    static constexpr int WARP_MMA = NUM_EPI, WARP_TMA = NUM_EPI + 1;
+    static constexpr int THREADS = 32 * (WARP_TMA + 1);
+    static constexpr int WCOLS = BN / (NUM_EPI / 4);      // columns per epilogue warp
+    static constexpr int CW = 32;                         // columns per tensor-memory read
+    static constexpr int SW = 16;                         // columns per staged store pass
+    // Staging: 32-byte rows (16 bf16); the two 16-byte chunks of row r swap places when bit 2 of r
+    // is set, which makes both the row-wise writes and the 2-lanes-per-row reads conflict-free.
+    static constexpr int STG_ROW = SW * 2;
+    static constexpr int STG_BYTES = NUM_EPI * 32 * STG_ROW;
+    static constexpr int BIAS_CAP = TC2_BIAS_CAP;         // fp32 bias / scale staged in shared memory
+    static constexpr int NBARS = 2 * STAGES + 5;
+    static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + BIAS_CAP * 4 + NBARS * 8 + 128;
+    static constexpr int TMEM_COLS = 2 * BN;              // two accumulators
+};
 
 __device__ __forceinline__ uint32_t cluster_rank() {
     uint32_t r;
@@ -90,28 +93,35 @@ struct PairTile {
     int e;
 };
 
+template <int BN>
 __device__ __forceinline__ PairTile decode_pair(const TcGemmArgs& a, int unit, int n_tiles, const int* s_prefix) {
+    constexpr int BM = T2<BN>::BM;
     PairTile t;
     const int mp = unit / n_tiles;
-    t.n0 = (unit % n_tiles) * t2::BN;
+    t.n0 = (unit % n_tiles) * BN;
     if (a.mode == TC_GROUPED) {
         int e = 0;
         while (e + 1 < a.E && s_prefix[e + 1] <= mp) ++e;
-        t.m0 = (int64_t)a.offsets[e] + (int64_t)(mp - s_prefix[e]) * 2 * t2::BM;
+        t.m0 = (int64_t)a.offsets[e] + (int64_t)(mp - s_prefix[e]) * 2 * BM;
         t.hi = a.offsets[e + 1];
         t.e = e;
     } else {
-        t.m0 = (int64_t)mp * 2 * t2::BM;
+        t.m0 = (int64_t)mp * 2 * BM;
         t.hi = a.M;
         t.e = 0;
     }
     return t;
 }
 
-template <int MODE>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
+template <int BN_, int MODE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
     tc_gemm2_kernel(const __grid_constant__ TcGemmArgs a) {
-    using namespace t2;
+    using C = T2<BN_>;
+    constexpr int BM = C::BM, BN = C::BN, BH = C::BH, BK = C::BK, A_BYTES = C::A_BYTES;
+    constexpr int STAGE_BYTES = C::STAGE_BYTES, STAGES = C::STAGES, NUM_EPI = C::NUM_EPI;
+    constexpr int WARP_MMA = C::WARP_MMA, WARP_TMA = C::WARP_TMA, WCOLS = C::WCOLS, CW = C::CW, SW = C::SW;
+    constexpr int STG_ROW = C::STG_ROW, STG_BYTES = C::STG_BYTES, BIAS_CAP = C::BIAS_CAP, NBARS = C::NBARS;
+    constexpr int TMEM_COLS = C::TMEM_COLS;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     unsigned char* sm = smem_raw + ((1024 - (raw_addr & 1023)) & 1023);
@@ -152,16 +162,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
         *abort_flag = 0;
         mbar_fence_init();
     }
-    // The bias (a weight, not produced by the previous kernel) as fp32, once per CTA.
+    // The bias or the column scale (weights, not produced by the previous kernel) as fp32, once per CTA.
     if (MODE == TC_DENSE && a.epi == TC_EPI_BIAS_GELU && warp < NUM_EPI) {
         const uint16_t* b = static_cast<const uint16_t*>(a.bias);
         for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = __uint_as_float((uint32_t)b[n] << 16);
+    } else if (MODE == TC_DENSE && a.epi == TC_EPI_SCALE && warp < NUM_EPI) {
+        for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = a.scale[n];
     }
     // Tensor memory for the pair: allocated collectively by one warp of each CTA. The two CTAs
     // must see the same base (the even CTA's MMAs name it for both); a mismatch aborts cleanly.
     if (warp == WARP_MMA) {
         asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                     "r"(a.tmem_cols)
+                     "r"(TMEM_COLS)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
     }
@@ -187,7 +199,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
     asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(peer_base) : "r"(map_to_rank(smem_u32(tmem_slot), rank ^ 1)));
     const bool tmem_ok = peer_base == tmem_base;
     if (!tmem_ok && threadIdx.x == 0) set_status(a.status, CLEARMOE_ECUDA);
-    const int nacc = a.tmem_cols >= 2 * BN ? 2 : 1;  // accumulator buffers
+    constexpr int nacc = 2;  // accumulator buffers
 
     int m_pairs;
     if (MODE == TC_GROUPED)
@@ -205,7 +217,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
             uint32_t ph = 0;
             bool ok = true;
             for (int u = cid; u < num_units && ok; u += ncl) {
-                const PairTile t = decode_pair(a, u, n_tiles, s_prefix);
+                const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
                 const int am = (int)(t.m0 + (int64_t)rank * BM);
                 const int bn = t.n0 + (int)rank * BH;
                 for (int kb = 0; kb < nkb; ++kb) {
@@ -307,7 +319,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
         int acc = 0;
         uint32_t aph = 0;
         for (int u = cid; u < num_units; u += ncl) {
-            const PairTile t = decode_pair(a, u, n_tiles, s_prefix);
+            const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
             if (!mbar_wait(tfull_bar(acc), aph, abort_flag, a.status, lim)) break;
             tc_fence_after();
             const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
@@ -344,6 +356,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
                         f[4 * j4 + 1] = g0.y;
                         f[4 * j4 + 2] = g1.x;
                         f[4 * j4 + 3] = g1.y;
+                    }
+                } else if (a.epi == TC_EPI_SCALE) {
+                    const float4* sp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
+#pragma unroll
+                    for (int j4 = 0; j4 < CW / 4; ++j4) {
+                        const float4 sc = sp[j4];
+                        const float2 p0 = __fmul2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), make_float2(sc.x, sc.y));
+                        const float2 p1 = __fmul2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), make_float2(sc.z, sc.w));
+                        f[4 * j4] = p0.x;
+                        f[4 * j4 + 1] = p0.y;
+                        f[4 * j4 + 2] = p1.x;
+                        f[4 * j4 + 3] = p1.y;
                     }
                 }
 #pragma unroll
@@ -382,43 +406,53 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(t2::THREADS, 1)
     cluster_sync();  // no copy, commit or remote arrival is left in flight towards either CTA
     tc_fence_after();
     if (warp == WARP_MMA)
-        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(a.tmem_cols)
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS)
                      : "memory");
 }
 
-// (a dense launch with the bias + GELU epilogue also needs N <= BIAS_CAP; launch_tc_gemm2 rejects
-// a larger one)
-bool tc2_supported(int mode, int N) { return (mode == TC_DENSE || mode == TC_GROUPED) && N % t2::BN == 0; }
+int tc2_pick_bn(int mode, int N) {
+    if (mode != TC_DENSE && mode != TC_GROUPED) return 0;
+    if (N % 256 == 0) return 256;
+    if (N % 128 == 0) return 128;
+    return 0;
+}
 
-cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
-    if (!tc2_supported(a.mode, a.N) || a.epi == TC_EPI_SCALE || (a.tmem_cols != 256 && a.tmem_cols != 512) ||
-        (a.epi == TC_EPI_BIAS_GELU && (a.mode != TC_DENSE || a.N > t2::BIAS_CAP)))
-        return cudaErrorInvalidValue;
+template <int BN>
+static cudaError_t launch2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
+    using C = T2<BN>;
     static bool attr[3] = {false, false, false};
-    const void* fn = a.mode == TC_GROUPED ? (const void*)tc_gemm2_kernel<TC_GROUPED> : (const void*)tc_gemm2_kernel<TC_DENSE>;
+    const void* fn = a.mode == TC_GROUPED ? (const void*)tc_gemm2_kernel<BN, TC_GROUPED>
+                                          : (const void*)tc_gemm2_kernel<BN, TC_DENSE>;
     if (!attr[a.mode]) {
-        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, t2::SMEM);
+        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
         attr[a.mode] = true;
     }
-    const int n_tiles = a.N / t2::BN;
-    int64_t m_pairs = (a.M + 2 * t2::BM - 1) / (2 * t2::BM);
+    const int n_tiles = a.N / BN;
+    int64_t m_pairs = (a.M + 2 * C::BM - 1) / (2 * C::BM);
     if (a.mode == TC_GROUPED) m_pairs += a.E;
     const int64_t units = m_pairs * n_tiles;
     int64_t clusters = units < num_sms / 2 ? units : num_sms / 2;
     if (clusters <= 0) return cudaSuccess;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(2 * clusters));
-    cfg.blockDim = dim3(t2::THREADS);
-    cfg.dynamicSmemBytes = t2::SMEM;
+    cfg.blockDim = dim3(C::THREADS);
+    cfg.dynamicSmemBytes = C::SMEM;
     cfg.stream = s;
     cudaLaunchAttribute attr_pdl[1];
     attr_pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr_pdl[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr_pdl;
     cfg.numAttrs = 1;
-    if (a.mode == TC_GROUPED) return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<TC_GROUPED>, a);
-    return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<TC_DENSE>, a);
+    if (a.mode == TC_GROUPED) return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<BN, TC_GROUPED>, a);
+    return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<BN, TC_DENSE>, a);
+}
+
+cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
+    const int bn = tc2_pick_bn(a.mode, a.N);
+    const bool staged = a.epi == TC_EPI_BIAS_GELU || a.epi == TC_EPI_SCALE;  // fp32 vector in shared memory
+    if (!bn || (staged && (a.mode != TC_DENSE || a.N > TC2_BIAS_CAP))) return cudaErrorInvalidValue;
+    return bn == 256 ? launch2<256>(a, num_sms, s) : launch2<128>(a, num_sms, s);
 }
 
 }  // namespace cm
