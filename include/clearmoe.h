@@ -83,7 +83,8 @@ int clearmoe_layer_destroy(clearmoe_layer* layer);
  * the fp32 logit W_g x_t + b_g; counts_e, offsets = exclusive prefix sum of counts (E + 1
  * entries), and perm[slot] = token with the tokens of expert e in slots
  * [offsets_e, offsets_{e+1}) in increasing id order (a stable sort by expert). One fused
- * kernel; results stay in the handle (read them with clearmoe_get_routing).
+ * kernel (logits, argmax, per-range histograms and ranks) and a slot kernel; results stay in
+ * the handle (read them with clearmoe_get_routing).
  * 1 <= T <= max_tokens, 1 <= E <= max_E. */
 int clearmoe_route(clearmoe_layer* layer, const void* x, int64_t T, const clearmoe_router* router,
                    int32_t E, void* stream);
@@ -122,12 +123,11 @@ int clearmoe_get_routing(clearmoe_layer* layer, int32_t* idx, int32_t* counts, i
  * device-side error since the last call, e.g. CLEARMOE_ETIMEOUT) and clears it. */
 int clearmoe_layer_status(clearmoe_layer* layer);
 
-/* Fault injection for tests of the bounded waits: the grid-wide wait of the routing kernel
- * gives up after wait_limit_ns nanoseconds (default 1e9) and, when phantom_arrivals > 0, waits
- * for the histograms of that many CTAs more than the launch has, so the wait runs out and the
- * call reports CLEARMOE_ETIMEOUT through clearmoe_layer_status (the layer stays usable: the next
- * launch needs no reset). phantom_arrivals = 0 restores normal use; a launch whose grid plus
- * phantom_arrivals exceeds the histogram scratch returns CLEARMOE_EUNSUPPORTED. */
+/* Fault injection for tests of the bounded waits: every device-side wait of the routing kernel
+ * gives up after wait_limit_ns nanoseconds (default 1e9) and, when phantom_arrivals > 0, the
+ * routing withholds the copy of one 16-token stage (in its first CTA), so the wait for it runs
+ * out and the call reports CLEARMOE_ETIMEOUT through clearmoe_layer_status; nothing is left in
+ * flight and the layer stays usable. phantom_arrivals = 0 restores normal use. */
 int clearmoe_debug_set_wait(clearmoe_layer* layer, int64_t wait_limit_ns, int32_t phantom_arrivals);
 
 /* Per-stage timing: when n >= 5, clearmoe_ffn_forward records events[0] before its first kernel
@@ -144,18 +144,19 @@ int clearmoe_set_profile_events(clearmoe_layer* layer, void* const* events, int3
  * (idx [T], counts [E], offsets [E + 1], perm [T]: caller-owned int32 device outputs) for tokens
  * x [T x d] of dtype `dtype` and the router W [E x d], b [E] in that dtype.
  *   - It calls no cudaMalloc, cudaFree or other allocating routine. Its scratch (per-CTA expert
- *     histograms, the launch epoch that tags them, a spare status word) is one static device
- *     array of 65,600 bytes that every GPU loading the library holds until exit; it serves up to
- *     512 routing CTAs (two per SM on GPUs with up to 256 SMs). A launch that would need more
- *     returns CLEARMOE_EUNSUPPORTED and enqueues nothing.
+ *     histograms and a spare status word) is one static device array of 65,600 bytes that every
+ *     GPU loading the library holds until exit; it serves up to 1,024 routing CTAs (two per SM on
+ *     GPUs with up to 512 SMs). A launch that would need more returns CLEARMOE_EUNSUPPORTED and
+ *     enqueues nothing. Between its two kernels idx holds packed per-token words; the second
+ *     kernel leaves the experts there.
  *   - The first call on a device looks up the array's device address (once per device, with that
  *     device current); make that first call before any stream capture.
- *   - Every call shares the array and it keeps the last call's contents, on purpose: the epoch
- *     only grows and the histogram words carry it, so nothing needs clearing but the status
- *     word. Calls whose work overlaps on the GPU (other streams, other host threads) race on the
+ *   - Every call shares the array and it keeps the last call's contents; each call clears what
+ *     must start at zero (the status words; the histograms are rewritten before they are read).
+ *     Calls whose work overlaps on the GPU (other streams, other host threads) race on the
  *     array: serialise them.
  *   - status (optional int32 device pointer, else NULL) is set to 0 at the start of the call and
- *     receives CLEARMOE_ETIMEOUT if the bounded grid-wide wait (1 s) runs out, in which case the
+ *     receives CLEARMOE_ETIMEOUT if a bounded device-side wait (1 s) runs out, in which case the
  *     outputs are undefined.
  * Limits: 1 <= T <= 2^30, 1 <= E <= 16; bf16: d % 64 == 0, d <= 1024; fp32: d % 4 == 0, d <= 512;
  * x and W 16-byte aligned. Host-side errors return EINVAL / EUNSUPPORTED / ECUDA with nothing

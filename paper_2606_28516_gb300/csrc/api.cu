@@ -20,11 +20,13 @@ struct clearmoe_layer {
     int32_t* inv;       // [max_tokens]  inv[token] = slot
     int32_t* counts;    // [CM_MAX_E]
     int32_t* offsets;   // [CM_MAX_E + 1]
-    unsigned long long* cta_words;  // [route_max_ctas x CM_MAX_E] the routing kernel's histogram words
-    unsigned long long* epoch;      // the routing kernel's launch epoch
+    int32_t* cta_counts;  // [route_max_ctas x CM_MAX_E] the routing kernel's per-range histograms
+    int32_t* tinfo;       // [max_tokens] per token: expert | rank within its routing range << 8
     int32_t* status;
     int64_t wait_limit_ns;
-    int32_t phantom;
+    int32_t phantom;  // fault injection: > 0 makes the routing withhold one stage copy
+    cm::RouteArgs rt;  // the last routing launch (its consumers reuse the shape)
+    int rt_grid, rt_chunk;
     int64_t last_T;
     int32_t last_E;
     cudaEvent_t prof[8];
@@ -44,7 +46,7 @@ int cuda_fail(cudaError_t e) {
 }
 
 void free_ws(clearmoe_layer* L) {
-    void* ptrs[] = {L->z, L->t, L->idx, L->perm, L->inv, L->counts, L->offsets, L->cta_words, L->epoch, L->status};
+    void* ptrs[] = {L->z, L->t, L->idx, L->perm, L->inv, L->counts, L->offsets, L->cta_counts, L->tinfo, L->status};
     for (void* p : ptrs)
         if (p) cudaFree(p);
 }
@@ -61,9 +63,8 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
     int grid = 0, chunk = 0;
     const int g = cm::route_grid(T, L->desc.d, E, L->desc.dtype, L->num_sms, &grid, &chunk);
     if (g) return g == -2 ? CLEARMOE_EUNSUPPORTED : CLEARMOE_ECUDA;
-    if (grid + L->phantom > cm::route_max_ctas(L->num_sms, L->desc.dtype, L->desc.d, E))
-        return CLEARMOE_EUNSUPPORTED;
-    cm::RouteArgs a;
+    if (grid > cm::route_max_ctas(L->num_sms, L->desc.dtype, L->desc.d, E)) return CLEARMOE_EUNSUPPORTED;
+    cm::RouteArgs& a = L->rt;
     std::memset(&a, 0, sizeof(a));
     a.x = x;
     a.T = T;
@@ -77,17 +78,24 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
     a.inv = L->inv;
     a.counts = L->counts;
     a.offsets = L->offsets;
-    a.cta_words = L->cta_words;
-    a.epoch = L->epoch;
-    a.arrivals = (unsigned int)grid + (unsigned int)L->phantom;
+    a.cta_counts = L->cta_counts;
+    a.tinfo = L->tinfo;
+    a.debug_skip = L->phantom > 0 ? 0 : -1;
     a.wait_limit_ns = L->wait_limit_ns;
     a.status = L->status;
+    L->rt_grid = grid;
+    L->rt_chunk = chunk;
     const int rc = cuda_fail(cm::launch_route(a, grid, chunk, s));
     if (rc == CLEARMOE_OK) {
         L->last_T = T;
         L->last_E = E;
     }
     return rc;
+}
+
+// counts, offsets, perm and inv from the last routing launch
+int do_finalize(clearmoe_layer* L, cudaStream_t s) {
+    return cuda_fail(cm::launch_route_finalize(L->rt, L->rt_grid, L->rt_chunk, s));
 }
 
 inline void mark(const clearmoe_layer* L, int i, cudaStream_t s) {
@@ -153,13 +161,14 @@ int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out)
               cudaMalloc((void**)&L->inv, T * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->counts, CM_MAX_E * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->offsets, (CM_MAX_E + 1) * 4) == cudaSuccess &&
-              cudaMalloc((void**)&L->cta_words, ncta * CM_MAX_E * 8) == cudaSuccess &&
-              cudaMalloc((void**)&L->epoch, 8) == cudaSuccess &&
+              cudaMalloc((void**)&L->cta_counts, ncta * CM_MAX_E * 4) == cudaSuccess &&
+              cudaMalloc((void**)&L->tinfo, T * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->status, 4) == cudaSuccess;
     if (ok) {
-        ok = cudaMemset(L->epoch, 0, 8) == cudaSuccess &&
-             cudaMemset(L->cta_words, 0, ncta * CM_MAX_E * 8) == cudaSuccess &&
-             cudaMemset(L->status, 0, 4) == cudaSuccess &&
+        // index workspaces start at zero (valid rows), so no launch ever reads garbage indices
+        ok = cudaMemset(L->status, 0, 4) == cudaSuccess && cudaMemset(L->perm, 0, T * 4) == cudaSuccess &&
+             cudaMemset(L->inv, 0, T * 4) == cudaSuccess && cudaMemset(L->tinfo, 0, T * 4) == cudaSuccess &&
+             cudaMemset(L->idx, 0, T * 4) == cudaSuccess &&
              cudaDeviceSynchronize() == cudaSuccess;
     }
     if (!ok) {
@@ -185,7 +194,9 @@ int clearmoe_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_r
     int rc = check_common(L, x, T);
     if (rc) return rc;
     if ((rc = check_router(L, router, E))) return rc;
-    return do_route(L, x, T, router, E, static_cast<cudaStream_t>(stream));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((rc = do_route(L, x, T, router, E, s))) return rc;
+    return do_finalize(L, s);
 }
 
 int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
@@ -209,6 +220,10 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
 
     mark(L, 0, s);
     if ((rc = do_route(L, x, T, router, E, s))) return rc;
+    // bf16 with the 2-SM fc1: the fc1 epilogue assigns the slots itself (no finalize launch)
+    const int p1 = bf16 && H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;
+    const bool fused = p1 && L->rt_grid <= 256 && L->rt_grid * E <= cm::TC2_TAB_CAP;
+    if (!fused && (rc = do_finalize(L, s))) return rc;
     mark(L, 1, s);
 
     if (!bf16) {
@@ -273,7 +288,8 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g.status = L->status;
     g.wait_limit_ns = L->wait_limit_ns;
     // fc1 + b1 + GELU into z in expert order. 2-SM kernel: x read in token order by TMA, each
-    // output row stored at its slot inv[token]; otherwise A rows are gathered by perm.
+    // output row stored at its slot (formed in the epilogue, or inv[token] after the finalize
+    // kernel); otherwise A rows are gathered by perm.
     g.epi = cm::TC_EPI_BIAS_GELU;
     g.M = T;
     g.N = H;
@@ -281,12 +297,22 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g.bias = b1;
     g.C = L->z;
     g.ldc = H;
-    const int p1 = H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;  // 2-SM tile width
     if (p1) {
         if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, p1 / 2))
             return CLEARMOE_ECUDA;
         g.mode = cm::TC_DENSE;
-        g.rows = L->inv;
+        if (fused) {  // slots from the routing's per-range counts and ranks; writes perm, counts, offsets
+            g.rt_info = L->tinfo;
+            g.rt_counts = L->cta_counts;
+            g.rt_ctas = L->rt_grid;
+            g.rt_chunk = L->rt_chunk;
+            g.rt_E = E;
+            g.rt_perm = L->perm;
+            g.rt_out_counts = L->counts;
+            g.rt_out_offsets = L->offsets;
+        } else {
+            g.rows = L->inv;
+        }
         rc = cuda_fail(cm::launch_tc_gemm2(g, L->num_sms, s));
     } else {
         if (encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;

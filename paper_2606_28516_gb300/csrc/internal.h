@@ -20,18 +20,22 @@ struct RouteArgs {
     int32_t* inv;                  // nullable: inv[token] = slot, the inverse of perm
     int32_t* counts;
     int32_t* offsets;
-    unsigned long long* cta_words; // [max_route_ctas x CM_MAX_E] histogram words, tag << 32 | count
-    unsigned long long* epoch;     // the last launch's tag (only grows; zero-initialised once)
-    unsigned int arrivals;         // histogram rows awaited (the grid; more in fault tests)
+    int32_t* cta_counts;           // [grid x CM_MAX_E] per-CTA-range expert counts
+    int32_t* tinfo;                // [T] per token: expert | rank within its CTA range << 8 (may be idx)
+    int debug_skip;                // fault injection: CTA 0 withholds this stage (-1: none)
     int64_t wait_limit_ns;
     int32_t* status;
 };
 
-// Grid of the routing kernel for T tokens (co-resident CTAs); chunk = rows per CTA. Returns 0,
-// -1 on a CUDA error, -2 when no launch shape fits.
+// Grid of the routing kernel for T tokens (one or two CTAs per SM); chunk = rows per CTA (a
+// routing range). Returns 0, -1 on a CUDA error, -2 when no launch shape fits.
 int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* chunk);
 int route_max_ctas(int num_sms, int dtype, int d, int E);
+// Phase 1 of the routing: idx, cta_counts and tinfo (no grid-wide step).
 cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s);
+// The slots from the routing's output: counts, offsets, perm, inv (if set); unpacks idx when
+// tinfo == idx. Same grid and chunk as the routing launch.
+cudaError_t launch_route_finalize(const RouteArgs& a, int grid, int chunk, cudaStream_t s);
 
 // ---- exact-fp32 SIMT GEMMs (fp32 layer) ----
 struct SimtGemmArgs {
@@ -85,12 +89,23 @@ struct TcGemmArgs {
     int64_t ldc;
     int32_t* status;
     int64_t wait_limit_ns;
+    // 2-SM dense kernel only: output row m (a token) goes to its routing slot offsets[e] +
+    // (tokens of e in ranges before m's) + rank, with (e, rank) = rt_info[m] packed as e | rank << 8
+    // and m's range m / rt_chunk; the kernel forms the prefix table from rt_counts ([rt_ctas x
+    // CM_MAX_E], rt_ctas <= 256, rt_ctas * rt_E <= TC2_TAB_CAP) and writes perm, counts, offsets.
+    const int32_t* rt_info;
+    const int32_t* rt_counts;
+    int rt_ctas, rt_chunk, rt_E;
+    int32_t* rt_perm;
+    int32_t* rt_out_counts;
+    int32_t* rt_out_offsets;
 };
 int tc_pick_bn(int mode, int N);
 // 2-SM (cta_group::2) variant for the dense and grouped modes: 256 x BN tiles per CTA pair, BN =
 // tc2_pick_bn(mode, N) (256 or 128; 0 = shape not supported; each CTA's B box is BN / 2 rows).
 // Its bias + GELU and column-scale epilogues stage the vector in shared memory (N <= TC2_BIAS_CAP).
 constexpr int TC2_BIAS_CAP = 4096;
+constexpr int TC2_TAB_CAP = 2432;  // routing prefix table entries (ranges x experts)
 int tc2_pick_bn(int mode, int N);
 cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_tc_gemm(const TcGemmArgs& a, int num_sms, cudaStream_t s);

@@ -5,9 +5,10 @@
 // allocation there), processes held to a fixed device-memory budget, and latency-critical loops
 // where cudaMalloc's implicit device-wide synchronisation is not acceptable. The handle-based
 // calls allocate their workspace in clearmoe_layer_create, so this entry point offers the routing
-// kernel without a handle: its scratch (the per-CTA expert histograms, the launch epoch that tags
-// them and a status word) is a file-scope device array that every GPU loading the library holds
-// until the process exits.
+// kernels without a handle: their scratch (the per-range expert histograms and a status word) is a
+// file-scope device array that every GPU loading the library holds until the process exits; the
+// per-token words of the routing (expert | rank in range) travel through the caller's idx, which
+// the finalize kernel then rewrites with the experts alone.
 #include <cstring>
 #include <mutex>
 
@@ -16,12 +17,11 @@
 
 namespace {
 
-// Scratch layout (int32 words): [0, 2) the routing kernel's 64-bit launch epoch, [2] status word
-// used when the caller passes no status pointer, [16, 16 + 2 * MAX_CTAS * CM_MAX_E) the per-CTA
-// histogram words (64-bit: launch tag << 32 | count).
-constexpr int kNoallocMaxCtas = 512;
+// Scratch layout (int32 words): [2] status word used when the caller passes no status pointer,
+// [16, 16 + MAX_CTAS * CM_MAX_E) the per-range histograms.
+constexpr int kNoallocMaxCtas = 1024;
 constexpr int kHistOffset = 16;
-constexpr int kScratchWords = kHistOffset + 2 * kNoallocMaxCtas * CM_MAX_E;  // 65,600 bytes
+constexpr int kScratchWords = kHistOffset + kNoallocMaxCtas * CM_MAX_E;  // 65,600 bytes
 
 static __device__ __align__(256) int32_t g_route_scratch[kScratchWords];
 
@@ -87,9 +87,8 @@ extern "C" int clearmoe_route_noalloc(const void* x, int64_t T, int32_t d, int32
     if (grid > kNoallocMaxCtas) return CLEARMOE_EUNSUPPORTED;  // beyond the scratch's capacity
 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    // The array keeps the previous call's contents, which is what the epoch needs (zero when the
-    // module loads, then only growing); the histogram words are tagged with it, so they need no
-    // clearing. Only the spare status word and the caller's status are cleared.
+    // Only the spare status word and the caller's status start at zero; the histograms are
+    // fully rewritten by every launch before they are read.
     if (cudaMemsetAsync(scratch + 2, 0, sizeof(int32_t), s) != cudaSuccess ||
         (status && cudaMemsetAsync(status, 0, sizeof(int32_t), s) != cudaSuccess)) {
         (void)cudaGetLastError();
@@ -109,12 +108,13 @@ extern "C" int clearmoe_route_noalloc(const void* x, int64_t T, int32_t d, int32
     a.inv = nullptr;
     a.counts = counts;
     a.offsets = offsets;
-    a.cta_words = reinterpret_cast<unsigned long long*>(scratch + kHistOffset);
-    a.epoch = reinterpret_cast<unsigned long long*>(scratch);
-    a.arrivals = (unsigned int)grid;
+    a.cta_counts = scratch + kHistOffset;
+    a.tinfo = idx;  // packed words in idx; route_finalize_kernel unpacks them
+    a.debug_skip = -1;
     a.wait_limit_ns = 1000000000LL;
     a.status = status ? status : scratch + 2;
-    const cudaError_t e = cm::launch_route(a, grid, chunk, s);
+    cudaError_t e = cm::launch_route(a, grid, chunk, s);
+    if (e == cudaSuccess) e = cm::launch_route_finalize(a, grid, chunk, s);
     if (e != cudaSuccess) {
         (void)cudaGetLastError();
         return CLEARMOE_ECUDA;

@@ -1,18 +1,18 @@
-// Fused routing kernel of the CLEAR-MoE FFN (Algorithm 3, steps 3-4):
+// Routing of the CLEAR-MoE FFN (Algorithm 3, steps 3-4):
 //   logits = W_g x + b_g (linear router), a = argmax (lowest index on ties),
 //   per-expert histogram, exclusive prefix sum, and the stable permutation perm[slot] = token.
 //
-// One cooperative launch of co-resident CTAs; CTA b owns a contiguous range of `chunk` tokens.
-//   phase 1: stream x once from HBM, router logits and argmax per token, local histogram.
+// route_kernel: CTA b owns a contiguous range of `chunk` tokens and never waits for another CTA.
+//   phase 1: stream x once from HBM, router logits and argmax per token, the range's histogram.
 //            bf16: one CTA per SM; a producer thread copies the CTA's rows, 16 at a time, into a
 //            ring of shared-memory stages with 1-D bulk copies (mbarrier-tracked, so the bytes in
 //            flight cost no registers) and eight consumer warps take one 16-row stage each;
-//   exchange: each CTA publishes its histogram as 64-bit words (launch tag << 32 | count), ranks
-//            its rows locally, then polls every CTA's row (one row per thread) until all carry
-//            this launch's tag, which is both the grid-wide wait (bounded) and the load of the
-//            counts;
-//   phase 2: each CTA sums the histograms of the CTAs before it and writes its tokens' slots in
-//            token order (local ranks from warp match masks), which makes the sort stable.
+//   then:    the histogram row goes to cta_counts, and each token's rank among the range's
+//            earlier tokens of its expert (warp match masks) to tinfo, packed with the expert.
+// The slot of token t in range c is offsets[e] + (tokens of e in ranges before c) + its rank, in
+// token order within each expert, which makes the sort stable. It is formed by the consumer of
+// the routing: the fc1 epilogue of the 2-SM GEMM (which then stores z rows at their slots and
+// writes perm), or route_finalize_kernel (perm and inv ahead of the other paths).
 // bf16 tokens: the d x E contraction runs on the legacy warp MMA (m16n8k16, fp32 accumulate):
 // x fragments from the shared-memory stage, W_g fragments staged once in shared memory (reading
 // them through L1 in the inner loop was measured slower), and the K order of each fragment is
@@ -75,7 +75,7 @@ __host__ __device__ inline size_t frag_bytes(int dtype, int d, int E) {
 // phase right after the one it last consumed (a parity wait cannot tell phases two apart).
 constexpr size_t RT_SMEM_MAX = 220 * 1024;
 struct RouteLayout {
-    size_t ring, bars, sidx, total;
+    size_t ring, bars, sidx, scnt, total;
     int S, stage_bytes;
     bool sidx_in_smem;
 };
@@ -90,8 +90,12 @@ __host__ __device__ inline RouteLayout route_layout(int dtype, int d, int E, int
     L.bars = (L.ring + (size_t)L.S * L.stage_bytes + 15) & ~(size_t)15;
     L.sidx = L.bars + (size_t)(2 * L.S + 1) * 8;  // bf16: ring barriers + the W_g barrier
     // expert ids of the CTA's rows: in shared memory when they fit, else read back from idx
-    L.sidx_in_smem = L.sidx + (size_t)chunk * 4 <= RT_SMEM_MAX;
-    L.total = L.sidx + (L.sidx_in_smem ? (size_t)chunk * 4 : 0);
+    // per row a 4-byte word; bf16 also keeps each 16-row stage's per-expert counts (2 bytes each)
+    const size_t rows_bytes =
+        (size_t)chunk * 4 + (dtype == CLEARMOE_BF16 ? (size_t)((chunk + 15) / 16) * CM_MAX_E * 2 : 0);
+    L.scnt = L.sidx + (size_t)chunk * 4;
+    L.sidx_in_smem = L.sidx + rows_bytes <= RT_SMEM_MAX;
+    L.total = L.sidx + (L.sidx_in_smem ? rows_bytes : 0);
     return L;
 }
 static size_t route_smem(int dtype, int d, int E, int chunk) { return route_layout(dtype, d, E, chunk).total; }
@@ -113,14 +117,11 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     constexpr int NCONS_MAX = 8;  // warps computing logits (bf16: the first S warps)
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ int s_count[CM_MAX_E];
-    __shared__ int s_base[CM_MAX_E];
     __shared__ int s_run[CM_MAX_E];
     __shared__ int s_wc[RT_MAX_WARPS][CM_MAX_E];
-    __shared__ int s_part[RT_MAX_WARPS][CM_MAX_E];
     __shared__ int s_abort;
-    __shared__ uint32_t s_tag;
 
-    pdl_launch_dependents();  // the GEMM that follows may set itself up meanwhile
+    pdl_launch_dependents();  // the kernel that follows may set itself up meanwhile
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int E = a.E, d = a.d;
     const int64_t row0 = (int64_t)blockIdx.x * chunk;
@@ -128,26 +129,20 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     const int nchunk = d / 32;
     const int NT = (E + 7) / 8;
     const RouteLayout lay = route_layout(BF16 ? CLEARMOE_BF16 : CLEARMOE_F32, d, E, chunk);
-    // per-row word: the expert after phase 1, expert | local rank << 8 after the local ranking
+    // per-row expert after phase 1: in shared memory when it fits, else read back from idx
     uint32_t* sinfo = lay.sidx_in_smem ? reinterpret_cast<uint32_t*>(smem + lay.sidx) : nullptr;
     auto info_of = [&](int i) -> uint32_t { return sinfo ? sinfo[i] : (uint32_t)__ldcg(a.idx + row0 + i); };
-    auto set_info = [&](int i, uint32_t v) {
-        if (sinfo)
-            sinfo[i] = v;
-        else
-            a.idx[row0 + i] = (int32_t)v;
-    };
-    auto record = [&](int i, int e) {  // phase 1 result of row i: idx, the row's word, histogram
+    // bf16 with the words in shared memory: ranks within 16-row stages during phase 1 (scnt holds
+    // each stage's per-expert counts), so that only a scan over stages remains afterwards
+    uint16_t* scnt = (BF16 && sinfo) ? reinterpret_cast<uint16_t*>(smem + lay.scnt) : nullptr;
+    auto record = [&](int i, int e, int rank) {  // phase 1 result of row i: idx, its word, histogram
         a.idx[row0 + i] = e;
-        if (sinfo) sinfo[i] = (uint32_t)e;
+        if (sinfo) sinfo[i] = (uint32_t)e | ((uint32_t)rank << 8);
         atomicAdd(&s_count[e], 1);
     };
 
     if (tid < CM_MAX_E) s_count[tid] = 0;
     if (tid == 0) s_abort = 0;
-    // the launch epoch, read now and used after phase 1 (the load's latency hides behind it)
-    unsigned long long ep0 = 0;
-    if (tid == 0) asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(ep0) : "l"(a.epoch) : "memory");
 
     // ---------------- phase 1: router logits + argmax for this CTA's rows
     if constexpr (BF16) {
@@ -178,6 +173,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
             const unsigned char* Wb = static_cast<const unsigned char*>(a.Wg);
             for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(smem) + e * WRB, Wb + (size_t)e * d * 2, d * 2, wbar);
         }
+        pdl_wait();  // from here on the previous kernel's results (x) are read and outputs written
         if (warp == NCONS_MAX) {
             if (producer) {
                 const unsigned char* xb = static_cast<const unsigned char*>(a.x) + row0 * d * 2;
@@ -186,6 +182,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                     const int s = k % S;
                     if (!mbar_wait(empty_bar(s), ((k / S) & 1) ^ 1, abort_flag, a.status, (uint64_t)a.wait_limit_ns))
                         break;
+                    if (k == a.debug_skip && blockIdx.x == 0) continue;  // fault injection: withhold a stage
                     const int rows = min(RT_STAGE_ROWS, nrows - k * RT_STAGE_ROWS);
                     const uint32_t bytes = (uint32_t)rows * d * 2;
                     mbar_arrive_expect_tx(full_bar(s), bytes);
@@ -298,10 +295,29 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 }
                 if (eA > E - 1) eA = 0;  // only reachable with non-finite logits
                 if (eB > E - 1) eB = 0;
+                int rankA = 0, rankB = 0;
+                if (scnt) {
+                    // rank of each row among the stage's earlier rows of its expert, from one ballot
+                    // per expert over the lanes holding rows 0-7 (eA) and rows 8-15 (eB)
+                    unsigned selAA = 0, selBA = 0, selBB = 0;
+                    for (int e = 0; e < E; ++e) {
+                        const unsigned mA = __ballot_sync(0xffffffffu, tig == 0 && vA && eA == e);
+                        const unsigned mB = __ballot_sync(0xffffffffu, tig == 0 && vB && eB == e);
+                        if (eA == e) selAA = mA;
+                        if (eB == e) {
+                            selBA = mA;
+                            selBB = mB;
+                        }
+                        if (lane == 0) scnt[k * CM_MAX_E + e] = (uint16_t)(__popc(mA) + __popc(mB));
+                    }
+                    const unsigned below = (1u << (4 * g)) - 1u;  // lanes of rows before row g
+                    rankA = __popc(selAA & below);
+                    rankB = __popc(selBA) + __popc(selBB & below);
+                }
                 if (tig == 0) {
                     const int iA = k * RT_STAGE_ROWS + g, iB = iA + 8;
-                    if (vA) record(iA, eA);
-                    if (vB) record(iB, eB);
+                    if (vA) record(iA, eA, rankA);
+                    if (vB) record(iB, eB, rankB);
                 }
             }
         }
@@ -309,6 +325,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         float* Wf = reinterpret_cast<float*>(smem);
         const float* W = static_cast<const float*>(a.Wg);
         for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = W[i];
+        pdl_wait();
         __syncthreads();
         const float* bgp = static_cast<const float*>(a.bg);
         const float* X = static_cast<const float*>(a.x);
@@ -335,32 +352,44 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 }
             }
             if (be > E - 1) be = 0;
-            if (lane == 0) record(i, be);
+            if (lane == 0) record(i, be, 0);
         }
     }
     __syncthreads();
 
-    // ---------------- exchange of the histograms. The launch tag is the low word of epoch + 1,
-    // where *a.epoch only grows (the last launch's tag, raised at the end of every launch, also
-    // one that timed out), so no row left by an earlier launch carries this launch's tag and
-    // nothing is reset between launches. Each 8-byte word is written and read whole, so a word
-    // with the right tag holds this launch's count.
-    if (tid == 0) s_tag = (uint32_t)(ep0 + 1);
-    __syncthreads();
-    const uint32_t tag = s_tag;
-    if (tid < E) {
-        const unsigned long long w = ((unsigned long long)tag << 32) | (uint32_t)s_count[tid];
-        asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(a.cta_words + (size_t)blockIdx.x * CM_MAX_E + tid),
-                     "l"(w)
-                     : "memory");
+    // ---------------- this CTA's histogram, and each row's rank among the CTA's earlier rows of
+    // its expert (warp match masks, then a per-expert prefix over warps and over passes), which
+    // makes the final order stable. The slots themselves are assigned by the consumer of the
+    // routing (the fc1 epilogue, or route_finalize_kernel): no CTA ever waits for another.
+    if (tid < E) a.cta_counts[(size_t)blockIdx.x * CM_MAX_E + tid] = s_count[tid];
+    if (scnt) {
+        // per expert, an exclusive scan of the stage counts (one warp per expert, 32 stages a
+        // step), then rank = the stage's prefix + the rank within the stage
+        const int nst = (nrows + RT_STAGE_ROWS - 1) / RT_STAGE_ROWS;
+        for (int e = warp; e < E; e += NWARPS) {
+            int carry = 0;
+            for (int k0 = 0; k0 < nst; k0 += 32) {
+                const int k = k0 + lane;
+                const int v = k < nst ? scnt[k * CM_MAX_E + e] : 0;
+                int incl = v;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const int o = __shfl_up_sync(0xffffffffu, incl, off);
+                    if (lane >= off) incl += o;
+                }
+                if (k < nst) scnt[k * CM_MAX_E + e] = (uint16_t)(carry + incl - v);
+                carry += __shfl_sync(0xffffffffu, incl, 31);
+            }
+        }
+        __syncthreads();
+        for (int i = tid; i < nrows; i += NTHREADS) {
+            const uint32_t w = sinfo[i];
+            int e = (int)(w & 0xffu);
+            if (e >= E) e = 0;  // rows a launch that gave up never routed: keep indices in range
+            a.tinfo[row0 + i] = e | ((scnt[(i / RT_STAGE_ROWS) * CM_MAX_E + e] + (int)((w >> 8) & 0xffu)) << 8);
+        }
+        return;
     }
-
-    // ---------------- local ranks: row i's rank among this CTA's earlier rows of the same expert
-    // (warp match masks, then a per-expert prefix over warps and over passes), which makes the
-    // final order stable. Done while the other CTAs publish.
-    // Per pass of NTHREADS rows: each warp's count per expert goes to s_wc; then lane e of every
-    // warp adds the counts of the warps before it (independent loads, no serial chain) to the
-    // running count of earlier passes, s_run; the last warp advances s_run.
     const unsigned lt = (1u << lane) - 1u;
     if (tid < CM_MAX_E) s_run[tid] = 0;
     for (int i0 = 0; i0 < nrows; i0 += NTHREADS) {
@@ -368,7 +397,8 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         __syncthreads();
         const int i = i0 + tid;
         const bool valid = i < nrows;
-        const int e = valid ? (int)(info_of(i) & 0xffu) : CM_MAX_E + 1;
+        int e = valid ? (int)(info_of(i) & 0xffu) : CM_MAX_E + 1;
+        if (valid && e >= E) e = 0;  // rows a launch that gave up never routed: keep indices in range
         const unsigned same = __match_any_sync(0xffffffffu, e);
         const int rank = __popc(same & lt);
         if (valid && rank == 0) s_wc[warp][e] = __popc(same);
@@ -380,115 +410,87 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
             own = s_wc[warp][lane];
         }
         const int base_e = __shfl_sync(0xffffffffu, pre, valid ? e : 0);
-        if (valid) set_info(i, (uint32_t)e | ((uint32_t)(base_e + rank) << 8));
+        if (valid) a.tinfo[row0 + i] = e | ((base_e + rank) << 8);
         __syncthreads();  // every warp has read s_run and s_wc
         if (warp == NWARPS - 1 && lane < E) s_run[lane] = pre + own;
     }
+}
 
-    // ---------------- bounded wait for every CTA's row. Thread t takes rows t, t + NTHREADS, ...;
-    // a row is read with 16-byte loads (its words issued together: one round trip), added to
-    // the sums over the CTAs before this one and over all CTAs once all its words carry this
-    // launch's tag, and not read again, so later polls touch only the rows still missing.
-    // `arrivals` rows are awaited (more than the grid only in fault tests).
-    int before[CM_MAX_E], total[CM_MAX_E];
+// Slots of one routing range (the same ranges as route_kernel: CTA b owns rows [b chunk, +chunk)):
+// the per-expert sums of the G ranges' histograms before this one and over all (thread b reads row
+// b), offsets by a scan over experts, then slot = offsets[e] + before + local rank for every row.
+// Writes perm, inv (if set), counts and offsets (range 0), and unpacks idx when it carried the
+// packed words.
+__global__ void __launch_bounds__(256) route_finalize_kernel(const RouteArgs a, const int chunk, const int G) {
+    __shared__ int s_wb[8][CM_MAX_E], s_wt[8][CM_MAX_E], s_base[CM_MAX_E];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, E = a.E;
+    const int64_t row0 = (int64_t)blockIdx.x * chunk;
+    const int nrows = (int)max((int64_t)0, min((int64_t)chunk, a.T - row0));
+    pdl_wait();  // everything below reads the routing kernel's output
+    pdl_launch_dependents();
+    int bef[CM_MAX_E], tot[CM_MAX_E];
 #pragma unroll
-    for (int e = 0; e < CM_MAX_E; ++e) before[e] = total[e] = 0;
-    {
-        const uint64_t t0 = globaltimer();
-        uint32_t done = 0;  // bit j: row tid + j * NTHREADS has been added
-        while (true) {
-            int ok = 1;
-            for (int j = 0, b = tid; b < (int)a.arrivals; ++j, b += NTHREADS) {
-                if ((done >> j) & 1u) continue;
-                const unsigned long long* row = a.cta_words + (size_t)b * CM_MAX_E;
-                unsigned long long w[CM_MAX_E];
+    for (int e = 0; e < CM_MAX_E; ++e) bef[e] = tot[e] = 0;
+    for (int b = tid; b < G; b += 256) {
+        const int4* row = reinterpret_cast<const int4*>(a.cta_counts + (size_t)b * CM_MAX_E);
 #pragma unroll
-                for (int q = 0; q < CM_MAX_E / 2; ++q)
-                    if (2 * q < E)
-                        asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];"
-                                     : "=l"(w[2 * q]), "=l"(w[2 * q + 1])
-                                     : "l"(row + 2 * q)
-                                     : "memory");
-                bool valid = true;
+        for (int q = 0; q < CM_MAX_E / 4; ++q) {
+            if (4 * q < E) {
+                const int4 v = __ldcg(row + q);
+                const int c4[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-                for (int e = 0; e < CM_MAX_E; ++e)
-                    if (e < E && (uint32_t)(w[e] >> 32) != tag) valid = false;
-                if (!valid) {
-                    ok = 0;
-                    continue;
-                }
-                done |= 1u << j;
-#pragma unroll
-                for (int e = 0; e < CM_MAX_E; ++e) {
-                    if (e < E) {
-                        const int c = (int)(uint32_t)w[e];
-                        total[e] += c;
-                        if (b < (int)blockIdx.x) before[e] += c;
-                    }
+                for (int j = 0; j < 4; ++j) {
+                    tot[4 * q + j] += c4[j];
+                    if (b < (int)blockIdx.x) bef[4 * q + j] += c4[j];
                 }
             }
-            if (__syncthreads_and(ok)) break;
-            if (tid == 0 && globaltimer() - t0 > (uint64_t)a.wait_limit_ns) s_abort = 1;
-            __syncthreads();
-            if (s_abort) {
-                if (tid == 0) {
-                    set_status(a.status, CLEARMOE_ETIMEOUT);
-                    atomicMax(a.epoch, ep0 + 1);  // this launch's tag is spent
-                }
-                return;
-            }
-            __nanosleep(64);
         }
     }
-    if (blockIdx.x == 0 && tid == 0) atomicMax(a.epoch, ep0 + 1);  // every CTA has read the epoch
-    if (s_abort) return;  // a wait of phase 1 gave up (status already set)
-
-    // ---------------- phase 2: global offsets, then this CTA's slots in token order. Sums by warp
-    // shuffles, per-warp partials in shared memory, then warp 0 lane e adds expert e's partials
-    // and scans the totals over experts.
 #pragma unroll
     for (int e = 0; e < CM_MAX_E; ++e) {
         if (e < E) {
-            const int vb = __reduce_add_sync(0xffffffffu, before[e]);
-            const int vt = __reduce_add_sync(0xffffffffu, total[e]);
+            const int vb = __reduce_add_sync(0xffffffffu, bef[e]);
+            const int vt = __reduce_add_sync(0xffffffffu, tot[e]);
             if (lane == 0) {
-                s_wc[warp][e] = vb;
-                s_part[warp][e] = vt;
+                s_wb[warp][e] = vb;
+                s_wt[warp][e] = vt;
             }
         }
     }
     __syncthreads();
     if (warp == 0) {
-        int bef = 0, tot = 0;
-        if (lane < E) {
-            for (int w = 0; w < NWARPS; ++w) {
-                bef += s_wc[w][lane];
-                tot += s_part[w][lane];
+        int b = 0, t = 0;
+        if (lane < E)
+            for (int w = 0; w < 8; ++w) {
+                b += s_wb[w][lane];
+                t += s_wt[w][lane];
             }
-        }
-        int incl = tot;  // inclusive scan of the totals over experts (lanes)
+        int incl = t;  // inclusive scan of the totals over experts (lanes)
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
             const int v = __shfl_up_sync(0xffffffffu, incl, off);
             if (lane >= off) incl += v;
         }
         if (lane < E) {
-            s_base[lane] = incl - tot + bef;
+            s_base[lane] = incl - t + b;
             if (blockIdx.x == 0) {
-                a.counts[lane] = tot;
-                a.offsets[lane] = incl - tot;
+                a.counts[lane] = t;
+                a.offsets[lane] = incl - t;
                 if (lane == E - 1) a.offsets[E] = incl;
             }
         }
     }
     __syncthreads();
-    for (int i = tid; i < nrows; i += NTHREADS) {
-        const uint32_t v = info_of(i);  // this thread's own word from the ranking pass
-        const int e = (int)(v & 0xffu);
-        const int slot = s_base[e] + (int)(v >> 8);
+    const bool unpack = a.tinfo == a.idx;
+    for (int i = tid; i < nrows; i += 256) {
+        const uint32_t w = (uint32_t)a.tinfo[row0 + i];
+        const int e = (int)(w & 0xffu);
+        if (e >= E) continue;  // only a routing launch that gave up leaves such words
+        const int64_t slot = (int64_t)s_base[e] + (int)(w >> 8);
+        if (slot >= a.T) continue;
         a.perm[slot] = (int32_t)(row0 + i);
-        if (a.inv) a.inv[row0 + i] = slot;
-        if (!sinfo) a.idx[row0 + i] = e;
+        if (a.inv) a.inv[row0 + i] = (int32_t)slot;
+        if (unpack) a.idx[row0 + i] = e;
     }
 }
 
@@ -499,7 +501,8 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
     const bool bf16 = dtype == CLEARMOE_BF16;
     int occ = 0;
     int64_t want = (int64_t)num_sms * (bf16 ? 1 : 2);  // bf16: one CTA per SM owns the ring
-    int64_t ch = ((T + want - 1) / want + 15) / 16 * 16;
+    // equal ranges over all CTAs (a range's last 16-row stage may be partial)
+    int64_t ch = (T + want - 1) / want;
     static std::mutex mu;
     std::lock_guard<std::mutex> lock(mu);
     static bool attr_set = false;
@@ -534,7 +537,7 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
         const int64_t maxg = (int64_t)occ * num_sms;
         if (want <= maxg) break;
         want = maxg;
-        ch = ((T + want - 1) / want + 15) / 16 * 16;
+        ch = (T + want - 1) / want;
     }
     if (ch < 16) ch = 16;
     if (ch >= ((int64_t)1 << 24)) return -2;  // a row's local rank must fit in 24 bits
@@ -552,13 +555,26 @@ cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = 1;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     if (!bf16) return cudaLaunchKernelEx(&cfg, route_kernel<false, false>, a, chunk);
     if (route_wreg(a.dtype, a.d, a.E)) return cudaLaunchKernelEx(&cfg, route_kernel<true, true>, a, chunk);
     return cudaLaunchKernelEx(&cfg, route_kernel<true, false>, a, chunk);
+}
+
+cudaError_t launch_route_finalize(const RouteArgs& a, int grid, int chunk, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, route_finalize_kernel, a, chunk, grid);
 }
 
 }  // namespace cm

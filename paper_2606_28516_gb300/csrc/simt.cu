@@ -66,7 +66,7 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
                 float v = 0.f;
                 if (m < m_hi && k0 + kk < K) {
                     const int64_t ar = (seg == 0 && a.a_rows) ? (int64_t)a.a_rows[m] : m;
-                    v = A[ar * lda + k0 + kk];
+                    if ((uint64_t)ar < (uint64_t)a.M) v = A[ar * lda + k0 + kk];
                 }
                 As[kk][r] = v;
                 const int n = n0 + r;
@@ -95,6 +95,7 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
         const int64_t m = m_lo + ty * 4 + i;
         if (m >= m_hi) continue;
         const int64_t orow = a.c_rows ? (int64_t)a.c_rows[m] : m;
+        if ((uint64_t)orow >= (uint64_t)a.M) continue;  // only a launch that gave up leaves such rows
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int n = n0 + tx * 4 + j;

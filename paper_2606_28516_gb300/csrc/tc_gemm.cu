@@ -200,6 +200,7 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
             for (int i = 0; i < 8; ++i) {
                 const int r = rsub + 16 * i;
                 src[i] = (r < t.rows) ? (int64_t)a.rows[t.m0 + r] : -1;
+                if ((uint64_t)src[i] >= (uint64_t)a.M) src[i] = -1;  // only a launch that gave up leaves such rows
             }
             for (int kb = 0; kb < nkb; ++kb) {
                 if (!mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim)) {
@@ -287,6 +288,7 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
             const int r = q * 32 + lane;
             int64_t orow = -1;
             if (r < t.rows) orow = (a.epi == TC_EPI_SCATTER) ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
+            if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;
             for (int c = c_lo; c < c_lo + C::HALF; c += C::CW) {
                 uint32_t v[32];
                 const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;

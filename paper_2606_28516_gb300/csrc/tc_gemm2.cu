@@ -40,8 +40,10 @@ struct T2 {
     static constexpr int STG_ROW = SW * 2;
     static constexpr int STG_BYTES = NUM_EPI * 32 * STG_ROW;
     static constexpr int BIAS_CAP = TC2_BIAS_CAP;         // fp32 bias / scale staged in shared memory
+    static constexpr int TAB_CAP = TC2_TAB_CAP;           // routing prefix table (fused fc1)
     static constexpr int NBARS = 2 * STAGES + 5;
-    static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + BIAS_CAP * 4 + NBARS * 8 + 128;
+    static constexpr int SMEM =
+        1024 + STAGES * STAGE_BYTES + STG_BYTES + BIAS_CAP * 4 + (TAB_CAP + CM_MAX_E) * 4 + NBARS * 8 + 128;
     static constexpr int TMEM_COLS = 2 * BN;              // two accumulators
 };
 
@@ -127,7 +129,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
     unsigned char* sm = smem_raw + ((1024 - (raw_addr & 1023)) & 1023);
     unsigned char* stg = sm + STAGES * STAGE_BYTES;
     float* s_bias = reinterpret_cast<float*>(stg + STG_BYTES);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(s_bias + BIAS_CAP);
+    int* s_tab = reinterpret_cast<int*>(s_bias + BIAS_CAP);  // [range][expert] tokens before
+    int* s_off = s_tab + C::TAB_CAP;                           // [expert] offsets
+    uint64_t* bars = reinterpret_cast<uint64_t*>(s_off + CM_MAX_E);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NBARS);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* s_prefix = reinterpret_cast<int*>(tmem_slot + 4);  // [CM_MAX_E + 1]
@@ -183,6 +187,69 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
     tc_fence_after();
     // everything above overlaps the predecessor kernel; from here on its results are read
     pdl_wait();
+    if (MODE == TC_DENSE && a.rt_info && warp < NUM_EPI) {
+        // Routing prefix table, by the epilogue warps while the producer and MMA warps start:
+        // thread c holds routing range c's counts; per expert, an exclusive scan over ranges (warp
+        // scans, warp totals in the staging area, named barrier 1 among the epilogue warps).
+        int* s_wt = reinterpret_cast<int*>(stg);  // [NUM_EPI][CM_MAX_E], before the staging is used
+        const int c = threadIdx.x;
+        const int E = a.rt_E;
+        int cnt[CM_MAX_E], incl[CM_MAX_E];
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e) cnt[e] = 0;
+        if (c < a.rt_ctas) {
+            const int4* row = reinterpret_cast<const int4*>(a.rt_counts + (size_t)c * CM_MAX_E);
+#pragma unroll
+            for (int q = 0; q < CM_MAX_E / 4; ++q) {
+                if (4 * q < E) {
+                    const int4 v = __ldcg(row + q);
+                    cnt[4 * q] = v.x;
+                    cnt[4 * q + 1] = v.y;
+                    cnt[4 * q + 2] = v.z;
+                    cnt[4 * q + 3] = v.w;
+                }
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e) {
+            incl[e] = cnt[e];
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, incl[e], off);
+                if (lane >= off) incl[e] += v;
+            }
+            if (lane == 31 && e < E) s_wt[warp * CM_MAX_E + e] = incl[e];
+        }
+        asm volatile("bar.sync 1, %0;" ::"n"(NUM_EPI * 32) : "memory");
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e) {
+            if (e < E) {
+                int before = incl[e] - cnt[e];
+                for (int w = 0; w < warp; ++w) before += s_wt[w * CM_MAX_E + e];
+                if (c < a.rt_ctas) s_tab[c * E + e] = before;
+            }
+        }
+        if (warp == 0) {  // lane e: expert totals, offsets by a scan over experts
+            int tot = 0;
+            if (lane < E)
+                for (int w = 0; w < NUM_EPI; ++w) tot += s_wt[w * CM_MAX_E + lane];
+            int sc = tot;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, sc, off);
+                if (lane >= off) sc += v;
+            }
+            if (lane < E) {
+                s_off[lane] = sc - tot;
+                if (blockIdx.x == 0) {
+                    a.rt_out_counts[lane] = tot;
+                    a.rt_out_offsets[lane] = sc - tot;
+                    if (lane == E - 1) a.rt_out_offsets[E] = sc;
+                }
+            }
+        }
+        asm volatile("bar.sync 1, %0;" ::"n"(NUM_EPI * 32) : "memory");
+    }
     if (MODE == TC_GROUPED) {
         if (threadIdx.x == 0) {
             int acc = 0;
@@ -320,11 +387,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         uint32_t aph = 0;
         for (int u = cid; u < num_units; u += ncl) {
             const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
+            const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
+            // the token's routing word, loaded before the accumulator wait so that the wait hides it
+            const uint32_t rtw = (MODE == TC_DENSE && a.rt_info && mrow < t.hi) ? (uint32_t)a.rt_info[mrow] : 0u;
             if (!mbar_wait(tfull_bar(acc), aph, abort_flag, a.status, lim)) break;
             tc_fence_after();
-            const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
             int64_t orow = -1;
-            if (mrow < t.hi) orow = a.rows ? (int64_t)a.rows[mrow] : mrow;
+            if (mrow < t.hi) {
+                if (MODE == TC_DENSE && a.rt_info) {  // the token's routing slot
+                    const uint32_t w = rtw;
+                    const int e = (int)(w & 0xffu);
+                    const int rc = (int)((uint32_t)mrow / (uint32_t)a.rt_chunk);  // T < 2^31
+                    if (e < a.rt_E) orow = (int64_t)s_off[e] + s_tab[rc * a.rt_E + e] + (int)(w >> 8);
+                    if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
+                    if (orow >= 0 && t.n0 == 0 && c_lo == 0) a.rt_perm[orow] = (int32_t)mrow;  // once per token
+                } else {
+                    orow = a.rows ? (int64_t)a.rows[mrow] : mrow;
+                    if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
+                }
+            }
             // this lane stores rows p * RPP + lane / LPR of the warp's 32 (p < LPR), 16-byte chunk
             // lane % LPR: their destinations, once per tile
             uint16_t* dst_row[LPR];
