@@ -36,18 +36,18 @@ METRIC = ("CLEAR-MoE FFN tokens/sec/layer (1×GB300) + % HBM peak (dispatch), "
           "% tensor peak (GEMMs)")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 STAGES = ("route", "fc1_gelu", "basis", "grouped")
-KERNEL_OF_STAGE = {"route": "cm::route_kernel<1>",
-                   "fc1_gelu": "cm::tc_gemm2_kernel<0> (2-SM dense, rows stored at inv[token])",
-                   "basis": "cm::tc_gemm_kernel<128, 0>",
-                   "grouped": "cm::tc_gemm2_kernel<2> (2-SM grouped, rows stored at perm[slot])"}
+KERNEL_OF_STAGE = {"route": "cm::route_kernel<1, 1>",
+                   "fc1_gelu": "cm::tc_gemm2_kernel<256, 0> (2-SM dense, rows stored at their routing slots)",
+                   "basis": "cm::tc_gemm2_kernel<128, 0> (2-SM dense, column scale)",
+                   "grouped": "cm::tc_gemm2_kernel<256, 2> (2-SM grouped, rows stored at perm[slot])"}
 # DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from the committed ncu
 # capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel sources
 # it was taken on; a different hash means the kernels changed and the figure is void.
 TRAFFIC = {
-    "route": {"bytes": 78.336768e6, "src": "5d42463a6e4f5296"},
-    "fc1_gelu": {"bytes": 337.993216e6, "src": "5d42463a6e4f5296"},
-    "basis": {"bytes": 321.057536e6, "src": "5d42463a6e4f5296"},
-    "grouped": {"bytes": 426.601728e6, "src": "5d42463a6e4f5296"},
+    "route": {"bytes": 78.329088e6, "src": "9ca6561f62a624ec"},
+    "fc1_gelu": {"bytes": 338.367744e6, "src": "9ca6561f62a624ec"},
+    "basis": {"bytes": 320.252672e6, "src": "9ca6561f62a624ec"},
+    "grouped": {"bytes": 426.128640e6, "src": "9ca6561f62a624ec"},
 }
 
 
