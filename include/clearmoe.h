@@ -90,10 +90,11 @@ int clearmoe_route(clearmoe_layer* layer, const void* x, int64_t T, const clearm
                    int32_t E, void* stream);
 
 /* The CLEAR-MoE FFN forward (Eq. 2 with Algorithm 3): routes (as clearmoe_route), computes
- * z = GELU(W1 x + b1) for every token in expert-sorted order (the gather by perm is folded into
- * the fc1 operand loads), the shared basis through its factors, t = diag(S_r) Vh_r z, and then,
- * per expert sub-batch, out[perm[slot]] = U_r t + residual_e[e] z (the scatter and the sum of
- * the shared and residual terms are folded into the epilogue; each row is written once).
+ * z = GELU(W1 x + b1) for every token in expert-sorted order (fc1 reads x in token order and its
+ * epilogue stores each row at the token's slot), the shared basis through its factors,
+ * t = diag(S_r) Vh_r z, and then, per expert sub-batch, out[perm[slot]] = U_r t + residual_e[e] z
+ * (the scatter and the sum of the shared and residual terms are folded into the epilogue; each
+ * row is written once).
  * residual_e is a HOST array of E device pointers, each to a [d x H] matrix.
  * 1 <= T <= max_tokens, 1 <= E <= max_E, 1 <= r <= min(max_r, d, H). out [T x d] must not
  * alias any input. */
@@ -101,6 +102,23 @@ int clearmoe_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const 
                          const void* b1, const void* U_r, const float* S_r, const void* Vh_r,
                          const void* const* residual_e, const clearmoe_router* router,
                          int32_t E, int32_t r, void* out, void* stream);
+
+/* The shared basis folded into the experts (Eq. 2 regrouped; the paper materialises W_shared in
+ * Phase 3): W_comb[e] = U_r diag(S_r) Vh_r + residual_e[e] for e < E, so that the layer output is
+ * y_t = W_comb[a_t] GELU(W1 x_t + b1). W_shared is formed in fp32 (products in fp32, summed over
+ * k ascending) and each sum is rounded once to the layer dtype. W_comb is a HOST array of E
+ * caller-owned device buffers, each [d x H] row-major like residual_e; computed once per weight
+ * set, it replaces the basis step of every later forward. Arguments as clearmoe_ffn_forward. */
+int clearmoe_fold_basis(clearmoe_layer* layer, const void* U_r, const float* S_r, const void* Vh_r,
+                        const void* const* residual_e, int32_t E, int32_t r, void* const* W_comb,
+                        void* stream);
+
+/* The CLEAR-MoE FFN forward on folded weights: routing and fc1 as clearmoe_ffn_forward, then per
+ * expert sub-batch out[perm[slot]] = W_comb[e] z in one grouped GEMM (no basis step: the dense
+ * FFN's arithmetic plus the routing). Same limits and errors as clearmoe_ffn_forward. */
+int clearmoe_ffn_forward_folded(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                                const void* b1, const void* const* W_comb,
+                                const clearmoe_router* router, int32_t E, void* out, void* stream);
 
 /* The dense FFN the layer was converted from, on the same device: out = W2 GELU(W1 x + b1)
  * (the comparison path; no bias on fc2, as in Eq. 2). 1 <= T <= max_tokens. */

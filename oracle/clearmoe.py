@@ -127,6 +127,23 @@ def ffn_forward(x, W1, b1, U, S, Vh, residuals, Wg=None, bg=None, a=None,
     return experts_forward(z, shared_weight(U, S, Vh), residuals, a)
 
 
+def fold_basis(U, S, Vh, residuals) -> np.ndarray:
+    """W_e^comb = W_shared + W_e^res for every expert e: Eq. 2 regrouped, since both terms act
+    on the same hidden state, y = W_shared z + W_a^res z = (W_shared + W_a^res) z."""
+    W_sh = shared_weight(U, S, Vh)
+    return np.stack([W_sh + f64(R) for R in residuals])
+
+
+def ffn_forward_folded(x, W1, b1, W_comb, Wg=None, bg=None, a=None,
+                       z_bf16: bool = False) -> np.ndarray:
+    """y = W_comb[a] z, z = GELU(fc1(x)): Algorithm 3 on folded weights (no shared step 2;
+    steps 4-6 with W_comb in place of the residuals)."""
+    if a is None:
+        a = route(x, Wg, bg)["a"]
+    z = fc1_gelu(x, W1, b1, z_bf16)
+    return experts_forward(z, np.zeros((f64(W_comb[0]).shape[0], z.shape[1])), W_comb, a)
+
+
 def dense_ffn(x, W1, b1, W2, z_bf16: bool = False) -> np.ndarray:
     """The unconverted layer: y = W2 GELU(W1 x + b1) (the dense FFN, D0)."""
     return fc1_gelu(x, W1, b1, z_bf16) @ f64(W2).T

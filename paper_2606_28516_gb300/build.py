@@ -11,7 +11,7 @@ PKG = pathlib.Path(__file__).resolve().parent
 CSRC = PKG / "csrc"
 OUT = PKG / "libclearmoe.so"
 BUILD = PKG / "_build"
-SOURCES = ("api.cu", "route.cu", "simt.cu", "tc_gemm.cu", "tc_gemm2.cu", "noalloc.cu")
+SOURCES = ("api.cu", "route.cu", "simt.cu", "tc_gemm.cu", "tc_gemm2.cu", "noalloc.cu", "fold.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr"]
 

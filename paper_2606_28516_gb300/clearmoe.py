@@ -45,6 +45,10 @@ _SIGS = {
     "clearmoe_layer_status": [_P],
     "clearmoe_debug_set_wait": [_P, _I64, _I32],
     "clearmoe_set_profile_events": [_P, ctypes.POINTER(ctypes.c_void_p), _I32],
+    "clearmoe_fold_basis": [_P, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p), _I32, _I32,
+                            ctypes.POINTER(ctypes.c_void_p), _P],
+    "clearmoe_ffn_forward_folded": [_P, _P, _I64, _P, _P, ctypes.POINTER(ctypes.c_void_p),
+                                    ctypes.POINTER(clearmoe_router), _I32, _P, _P],
     "clearmoe_route_noalloc": [_P, _I64, _I32, _I32, ctypes.POINTER(clearmoe_router), _I32, _P, _P,
                                _P, _P, _P, _P],
     "clearmoe_strerror": [ctypes.c_int],
@@ -130,6 +134,24 @@ def clearmoe_ffn_forward(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, 
                                       _ptr(S_r), _ptr(Vh_r), res, ctypes.byref(r), E,
                                       S_r.shape[0], _ptr(out), _stream(stream)),
            "clearmoe_ffn_forward")
+
+
+def clearmoe_fold_basis(layer: int, U_r, S_r, Vh_r, residual_e, W_comb, stream=None) -> None:
+    """residual_e, W_comb: sequences of E [d x H] tensors, or [E x d x H] tensors."""
+    E = len(residual_e)
+    res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
+    comb = (ctypes.c_void_p * E)(*[_ptr(W_comb[e]) for e in range(E)])
+    _check(lib().clearmoe_fold_basis(layer, _ptr(U_r), _ptr(S_r), _ptr(Vh_r), res, E, S_r.shape[0],
+                                     comb, _stream(stream)), "clearmoe_fold_basis")
+
+
+def clearmoe_ffn_forward_folded(layer: int, x, W1, b1, W_comb, Wg, bg, out, stream=None) -> None:
+    E = Wg.shape[0]
+    comb = (ctypes.c_void_p * E)(*[_ptr(W_comb[e]) for e in range(E)])
+    r = _router(Wg, bg)
+    _check(lib().clearmoe_ffn_forward_folded(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), comb,
+                                             ctypes.byref(r), E, _ptr(out), _stream(stream)),
+           "clearmoe_ffn_forward_folded")
 
 
 def clearmoe_dense_ffn_forward(layer: int, x, W1, b1, W2, out, stream=None) -> None:

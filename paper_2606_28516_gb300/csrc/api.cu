@@ -199,25 +199,14 @@ int clearmoe_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_r
     return do_finalize(L, s);
 }
 
-int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
-                         const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
-                         const clearmoe_router* router, int32_t E, int32_t r, void* out, void* stream) {
-    int rc = check_common(L, x, T);
-    if (rc) return rc;
-    if ((rc = check_router(L, router, E))) return rc;
-    if (!W1 || !b1 || !U_r || !S_r || !Vh_r || !residual_e || !out) return CLEARMOE_EINVAL;
+static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                    const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
+                    const clearmoe_router* router, int E, int r, void* out, cudaStream_t s) {
+    // U_r == nullptr: the folded forward, residual_e holds W_comb (no basis step, no t segment)
+    const bool folded = U_r == nullptr;
     const int d = L->desc.d, H = L->desc.hidden;
-    if (r < 1 || r > L->desc.max_r || r > d || r > H) return CLEARMOE_EINVAL;
-    for (int e = 0; e < E; ++e)
-        if (!residual_e[e] || misaligned(residual_e[e])) return CLEARMOE_EINVAL;
-    if (misaligned(W1) || misaligned(b1) || misaligned(U_r) || misaligned(S_r) || misaligned(Vh_r) ||
-        misaligned(out))
-        return CLEARMOE_EINVAL;
     const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
-    if (bf16 && r % 16) return CLEARMOE_EUNSUPPORTED;
-    if (!bf16 && r % 4) return CLEARMOE_EUNSUPPORTED;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-
+    int rc;
     mark(L, 0, s);
     if ((rc = do_route(L, x, T, router, E, s))) return rc;
     // bf16 with the 2-SM fc1: the fc1 epilogue assigns the slots itself (no finalize launch)
@@ -243,25 +232,28 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
         g.ldc = H;
         if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
         mark(L, 2, s);
-        // t = diag(S_r) Vh_r z
-        std::memset(&g, 0, sizeof(g));
-        g.A0 = static_cast<const float*>(L->z);
-        g.lda0 = H;
-        g.K0 = H;
-        g.B0 = static_cast<const float*>(Vh_r);
-        g.M = T;
-        g.N = r;
-        g.scale = S_r;
-        g.C = static_cast<float*>(L->t);
-        g.ldc = r;
-        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        if (!folded) {  // t = diag(S_r) Vh_r z
+            std::memset(&g, 0, sizeof(g));
+            g.A0 = static_cast<const float*>(L->z);
+            g.lda0 = H;
+            g.K0 = H;
+            g.B0 = static_cast<const float*>(Vh_r);
+            g.M = T;
+            g.N = r;
+            g.scale = S_r;
+            g.C = static_cast<float*>(L->t);
+            g.ldc = r;
+            if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        }
         mark(L, 3, s);
-        // out[perm[slot]] = U_r t + W_e^res z per expert sub-batch
+        // out[perm[slot]] = U_r t + W_e^res z per expert sub-batch (folded: W_e^comb z)
         std::memset(&g, 0, sizeof(g));
-        g.A0 = static_cast<const float*>(L->t);
-        g.lda0 = r;
-        g.K0 = r;
-        g.B0 = static_cast<const float*>(U_r);
+        if (!folded) {
+            g.A0 = static_cast<const float*>(L->t);
+            g.lda0 = r;
+            g.K0 = r;
+            g.B0 = static_cast<const float*>(U_r);
+        }
         g.A1 = static_cast<const float*>(L->z);
         g.lda1 = H;
         g.K1 = H;
@@ -280,7 +272,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
 
     // ---- bf16: tcgen05 GEMMs
     const int bn1 = cm::tc_pick_bn(cm::TC_GATHER, H);
-    const int bn2 = cm::tc_pick_bn(cm::TC_DENSE, r);
+    const int bn2 = folded ? 1 : cm::tc_pick_bn(cm::TC_DENSE, r);
     const int bn3 = cm::tc_pick_bn(cm::TC_GROUPED, d);
     if (!bn1 || !bn2 || !bn3) return CLEARMOE_EUNSUPPORTED;
     cm::TcGemmArgs g;
@@ -324,24 +316,26 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     }
     if (rc) return rc;
     mark(L, 2, s);
-    // t = diag(S_r) Vh_r z (the 2-SM kernel when r is a multiple of 128: more of z in flight per SM)
-    cm::TcGemmArgs g2;
-    std::memset(&g2, 0, sizeof(g2));
-    g2.status = L->status;
-    g2.wait_limit_ns = L->wait_limit_ns;
-    const int p2 = cm::tc2_pick_bn(cm::TC_DENSE, r);
-    if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, Vh_r, r, H, p2 ? p2 / 2 : bn2))
-        return CLEARMOE_ECUDA;
-    g2.mode = cm::TC_DENSE;
-    g2.epi = cm::TC_EPI_SCALE;
-    g2.M = T;
-    g2.N = r;
-    g2.K0 = H;
-    g2.scale = S_r;
-    g2.C = L->t;
-    g2.ldc = r;
-    rc = cuda_fail(p2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
-    if (rc) return rc;
+    if (!folded) {  // t = diag(S_r) Vh_r z (2-SM kernel when r is a multiple of 128)
+        cm::TcGemmArgs g2;
+        std::memset(&g2, 0, sizeof(g2));
+        g2.status = L->status;
+        g2.wait_limit_ns = L->wait_limit_ns;
+        const int p2 = cm::tc2_pick_bn(cm::TC_DENSE, r);
+        if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) ||
+            encode_tmap_bf16(&g2.tmB0, Vh_r, r, H, p2 ? p2 / 2 : bn2))
+            return CLEARMOE_ECUDA;
+        g2.mode = cm::TC_DENSE;
+        g2.epi = cm::TC_EPI_SCALE;
+        g2.M = T;
+        g2.N = r;
+        g2.K0 = H;
+        g2.scale = S_r;
+        g2.C = L->t;
+        g2.ldc = r;
+        rc = cuda_fail(p2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
+        if (rc) return rc;
+    }
     mark(L, 3, s);
     // out[perm[slot]] = [t | z] [U_r | W_e^res]^T per expert sub-batch
     cm::TcGemmArgs g3;
@@ -351,7 +345,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     // The 2-SM kernel loads half of each pair tile's B rows per CTA: boxes of p3 / 2 rows.
     const int p3 = cm::tc2_pick_bn(cm::TC_GROUPED, d);
     const int box3 = p3 ? p3 / 2 : bn3;
-    if (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, box3) ||
+    if ((!folded && (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, box3))) ||
         encode_tmap_bf16(&g3.tmA1, L->z, T, H, 128))
         return CLEARMOE_ECUDA;
     for (int e = 0; e < E; ++e)
@@ -360,7 +354,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     g3.epi = cm::TC_EPI_SCATTER;
     g3.M = T;
     g3.N = d;
-    g3.K0 = r;
+    g3.K0 = folded ? 0 : r;  // folded: the K chain is z x W_e^comb alone
     g3.K1 = H;
     g3.offsets = L->offsets;
     g3.E = E;
@@ -370,6 +364,64 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     rc = cuda_fail(p3 ? cm::launch_tc_gemm2(g3, L->num_sms, s) : cm::launch_tc_gemm(g3, L->num_sms, s));
     mark(L, 4, s);
     return rc;
+}
+
+int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                         const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
+                         const clearmoe_router* router, int32_t E, int32_t r, void* out, void* stream) {
+    int rc = check_common(L, x, T);
+    if (rc) return rc;
+    if ((rc = check_router(L, router, E))) return rc;
+    if (!W1 || !b1 || !U_r || !S_r || !Vh_r || !residual_e || !out) return CLEARMOE_EINVAL;
+    const int d = L->desc.d, H = L->desc.hidden;
+    if (r < 1 || r > L->desc.max_r || r > d || r > H) return CLEARMOE_EINVAL;
+    for (int e = 0; e < E; ++e)
+        if (!residual_e[e] || misaligned(residual_e[e])) return CLEARMOE_EINVAL;
+    if (misaligned(W1) || misaligned(b1) || misaligned(U_r) || misaligned(S_r) || misaligned(Vh_r) ||
+        misaligned(out))
+        return CLEARMOE_EINVAL;
+    const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
+    if (bf16 && r % 16) return CLEARMOE_EUNSUPPORTED;
+    if (!bf16 && r % 4) return CLEARMOE_EUNSUPPORTED;
+    return ffn_impl(L, x, T, W1, b1, U_r, S_r, Vh_r, residual_e, router, E, r, out,
+                    static_cast<cudaStream_t>(stream));
+}
+
+int clearmoe_ffn_forward_folded(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                                const void* const* W_comb, const clearmoe_router* router, int32_t E, void* out,
+                                void* stream) {
+    int rc = check_common(L, x, T);
+    if (rc) return rc;
+    if ((rc = check_router(L, router, E))) return rc;
+    if (!W1 || !b1 || !W_comb || !out) return CLEARMOE_EINVAL;
+    for (int e = 0; e < E; ++e)
+        if (!W_comb[e] || misaligned(W_comb[e])) return CLEARMOE_EINVAL;
+    if (misaligned(W1) || misaligned(b1) || misaligned(out)) return CLEARMOE_EINVAL;
+    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, W_comb, router, E, 0, out,
+                    static_cast<cudaStream_t>(stream));
+}
+
+int clearmoe_fold_basis(clearmoe_layer* L, const void* U_r, const float* S_r, const void* Vh_r,
+                        const void* const* residual_e, int32_t E, int32_t r, void* const* W_comb, void* stream) {
+    if (!L || !U_r || !S_r || !Vh_r || !residual_e || !W_comb) return CLEARMOE_EINVAL;
+    const int d = L->desc.d, H = L->desc.hidden;
+    if (E < 1 || E > L->desc.max_E) return CLEARMOE_EINVAL;
+    if (r < 1 || r > L->desc.max_r || r > d || r > H) return CLEARMOE_EINVAL;
+    cm::FoldArgs f;
+    std::memset(&f, 0, sizeof(f));
+    f.U = U_r;
+    f.S = S_r;
+    f.Vh = Vh_r;
+    for (int e = 0; e < E; ++e) {
+        if (!residual_e[e] || !W_comb[e]) return CLEARMOE_EINVAL;
+        f.res[e] = residual_e[e];
+        f.out[e] = W_comb[e];
+    }
+    f.d = d;
+    f.H = H;
+    f.r = r;
+    f.E = E;
+    return cuda_fail(cm::launch_fold_basis(f, L->desc.dtype, static_cast<cudaStream_t>(stream)));
 }
 
 int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,

@@ -33,6 +33,11 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);  // round to nearest even
     return *reinterpret_cast<uint32_t*>(&p);
 }
+__device__ __forceinline__ float bf16_to_f32(uint16_t v) { return __uint_as_float((uint32_t)v << 16); }
+__device__ __forceinline__ uint16_t f32_to_bf16(float v) {
+    const __nv_bfloat16 b = __float2bfloat16_rn(v);  // round to nearest even
+    return *reinterpret_cast<const uint16_t*>(&b);
+}
 
 __device__ __forceinline__ float gelu_erf(float u) {
     // GELU(u) = u * Phi(u) = u * (1 + erf(u / sqrt 2)) / 2, with CUDA's erff.

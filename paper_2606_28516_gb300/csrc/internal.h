@@ -37,6 +37,17 @@ cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s
 // tinfo == idx. Same grid and chunk as the routing launch.
 cudaError_t launch_route_finalize(const RouteArgs& a, int grid, int chunk, cudaStream_t s);
 
+// ---- folding the shared basis into the experts: out[e] = U diag(S) Vh + res[e] ----
+struct FoldArgs {
+    const void* U;      // [d x r] layer dtype
+    const float* S;     // [r]
+    const void* Vh;     // [r x H] layer dtype
+    const void* res[16];
+    void* out[16];      // [d x H] each, layer dtype
+    int d, H, r, E;
+};
+cudaError_t launch_fold_basis(const FoldArgs& a, int dtype, cudaStream_t s);
+
 // ---- exact-fp32 SIMT GEMMs (fp32 layer) ----
 struct SimtGemmArgs {
     // C[m, n] = epi(sum_k A0[rowA(m), k] B0[n, k] + sum_k A1[m, k] B1_e[n, k])

@@ -136,6 +136,36 @@ def test_scalar_residual_form():
     assert check_scalar_residual()
 
 
+def check_fold_d3(seed=4):
+    """Residuals W2 - W_shared (D3) fold to W2 itself for every expert."""
+    rng = np.random.default_rng(seed)
+    d, H, E, r = 9, 30, 3, 5
+    L = rand_layer(rng, 8, d, H, E, r)
+    D = L["W2"] - O.shared_weight(L["U"], L["S"], L["Vh"])
+    W = O.fold_basis(L["U"], L["S"], L["Vh"], np.stack([D] * E))
+    return all(np.max(np.abs(W[e] - L["W2"])) <= 1e-12 for e in range(E))
+
+
+def check_folded_brute(seed=5, T=19, d=16, H=64, E=3, r=6):
+    """The folded forward against the factorised brute force (which never forms W_shared)."""
+    rng = np.random.default_rng(seed)
+    L = rand_layer(rng, T, d, H, E, r)
+    a_b, y_b = B.layer(L["x"].tolist(), L["W1"].tolist(), L["b1"].tolist(), L["U"].tolist(),
+                       L["S"].tolist(), L["Vh"].tolist(), L["residuals"].tolist(),
+                       L["Wg"].tolist(), L["bg"].tolist())
+    W = O.fold_basis(L["U"], L["S"], L["Vh"], L["residuals"])
+    y = O.ffn_forward_folded(L["x"], L["W1"], L["b1"], W, a=np.array(a_b))
+    return rel_err(y, np.array(y_b)) <= 1e-12
+
+
+def test_fold_d3_gives_w2():
+    assert check_fold_d3()
+
+
+def test_folded_forward_brute_force():
+    assert check_folded_brute()
+
+
 # ------------------------------------------------------------------ brute force
 def check_brute(seed, T=23, d=16, H=64, E=4, r=16):
     rng = np.random.default_rng(seed)
@@ -264,6 +294,8 @@ MUTATIONS = {
         z, W_sh, res, np.zeros_like(np.asarray(a)))),
     "Sigma applied as 1/S": ("shared_weight", lambda U, S, Vh: O.f64(U) @ np.diag(
         1 / O.f64(S)) @ O.f64(Vh)),
+    "fold drops the shared term": ("fold_basis", lambda U, S, Vh, res: np.stack(
+        [O.f64(R) for R in res])),
     "unsorted sub-batches": ("sort_by_expert", lambda a, E: dict(
         a=np.asarray(a), counts=np.bincount(a, minlength=E),
         offsets=np.concatenate([[0], np.cumsum(np.bincount(a, minlength=E))]),
@@ -276,7 +308,8 @@ def test_pins_catch_planted_mistakes(name, monkeypatch):
     attr, fake = MUTATIONS[name]
     monkeypatch.setattr(O, attr, fake)
     checks = [check_gelu_table, check_worked_example, check_dense_reduction,
-              check_d3_identity, check_scalar_residual, lambda: check_brute(0)]
+              check_d3_identity, check_scalar_residual, lambda: check_brute(0), check_fold_d3,
+              check_folded_brute]
     results = []
     for c in checks:
         try:
