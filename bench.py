@@ -305,6 +305,28 @@ def main():
         total_ms = float(t.item())
     value = world * s.T * K / (total_ms / 1e3)
 
+    # The folded variant (the shared basis folded into the experts once; same routing and fc1,
+    # one grouped GEMM over z), same timing rules. Reported beside the headline, not as it.
+    W_comb = torch.empty_like(D["residuals"]) if s.dtype == "bf16" else None
+    folded = None
+    if W_comb is not None:
+        cm.clearmoe_fold_basis(h, D["U"], D["S"], D["Vh"], D["residuals"], W_comb)
+        fev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(min(K, 300))]
+        for k in range(len(fev) + args.warmup):
+            flush.zero_()
+            if k >= args.warmup:
+                fev[k - args.warmup][0].record(stream)
+            cm.clearmoe_ffn_forward_folded(h, D["x"], D["W1"], D["b1"], W_comb, D["Wg"], D["bg"], out)
+            if k >= args.warmup:
+                fev[k - args.warmup][1].record(stream)
+        torch.cuda.synchronize()
+        assert cm.clearmoe_layer_status(h) == 0
+        f_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in fev)
+        folded = {"value": world * s.T / (f_ms / 1e3), "unit": "tokens/s", "ms_per_step": f_ms,
+                  "note": "W_e^comb = U_r diag(S_r) V_r^T + W_e^res formed once (clearmoe_fold_basis); "
+                          "forward = routing, fc1, one grouped GEMM over z"}
+        del W_comb
+
     # same-GPU dense FFN, same timing rules (events around each forward only)
     dout = torch.empty_like(out)
     dev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(min(K, 300))]
@@ -438,6 +460,7 @@ def main():
         "layer_roofline_frac": layer_roofline_s(s, pk) / (mean_step / 1e3),
         "dense_ffn": {"value": dense_value, "unit": "tokens/s",
                       "ms_per_step": statistics.mean(dense_ms)},
+        "folded": folded,
         "wall_s_timed": wall,
     }
     if rank == 0:
