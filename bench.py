@@ -54,7 +54,7 @@ TRAFFIC = {
 def workloads():
     import synth
     return {"deit_base_bf16": synth.DEIT_BASE_BF16, "deit_small_bf16": synth.DEIT_SMALL_BF16,
-            "deit_tiny_fp32": synth.DEIT_TINY_FP32}
+            "deit_tiny_fp32": synth.DEIT_TINY_FP32, "vit_base_stack12": synth.VIT_BASE_STACK12}
 
 
 def peaks():
@@ -207,6 +207,142 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_stack(args):
+    """The 12-sublayer ViT-B stack (odd sublayers CLEAR-MoE, x_{l+1} = LN(y_l)), end to end on one
+    stream: value = tokens / time of one pass through all 12 sublayers. The pass's input (155 MB)
+    and weights exceed L2, so no flush is needed between passes."""
+    import numpy as np
+    import torch
+
+    import synth
+    import __graft_entry__
+    from paper_2606_28516_gb300 import clearmoe as cm
+    from oracle import clearmoe as O
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    if rank == 0:
+        __graft_entry__.build()
+    if dist:
+        dist.barrier()
+    cm.lib()
+    sh = synth.VIT_BASE_STACK12
+    S = synth.make_stack(sh)
+    T = S["T"]
+    dev = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to("cuda", torch.bfloat16)
+    layers = []
+    for L in S["layers"]:
+        G = dict(moe=L["moe"], W1=dev(L["W1"]), b1=dev(L["b1"]))
+        if L["moe"]:
+            G.update(U=dev(L["U"]), S=torch.from_numpy(L["S"].astype(np.float32)).cuda(), Vh=dev(L["Vh"]),
+                     residuals=dev(L["residuals"]), Wg=dev(L["Wg"]), bg=dev(L["bg"]))
+        else:
+            G["W2"] = dev(L["W2"])
+        layers.append(G)
+    h = cm.clearmoe_layer_create(T, sh.d, sh.H, sh.E, sh.r, cm.BF16)
+    x0 = dev(S["x"])
+    buf = [torch.empty_like(x0) for _ in range(2)]
+    y = torch.empty_like(x0)
+
+    def stack_pass(x_in, folded=False):
+        x = x_in
+        for l, G in enumerate(layers):
+            if G["moe"] and folded:
+                cm.clearmoe_ffn_forward_folded(h, x, G["W1"], G["b1"], G["W_comb"], G["Wg"], G["bg"], y)
+            elif G["moe"]:
+                cm.clearmoe_ffn_forward(h, x, G["W1"], G["b1"], G["U"], G["S"], G["Vh"], G["residuals"],
+                                        G["Wg"], G["bg"], y)
+            else:
+                cm.clearmoe_dense_ffn_forward(h, x, G["W1"], G["b1"], G["W2"], y)
+            x = buf[l & 1]
+            cm.clearmoe_layer_norm(h, y, x)
+        return x
+
+    def timed(K, folded=False):
+        for _ in range(args.warmup):
+            stack_pass(x0, folded)
+        torch.cuda.synchronize()
+        assert cm.clearmoe_layer_status(h) == 0
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        for k in range(K):
+            ev[k][0].record()
+            stack_pass(x0, folded)
+            ev[k][1].record()
+        torch.cuda.synchronize()
+        assert cm.clearmoe_layer_status(h) == 0
+        ms = float(sum(e[0].elapsed_time(e[1]) for e in ev))
+        if dist:
+            t = torch.tensor([ms], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms = float(t.item())
+        return ms / K
+
+    K = max(1, min(args.steps, 50))
+    with ClockSampler(local) as clk:
+        ms = timed(K)
+    value = world * T / (ms / 1e3)
+    # folded variant of the same stack (each converted sublayer's basis folded once)
+    for G in layers:
+        if G["moe"]:
+            G["W_comb"] = torch.empty_like(G["residuals"])
+            cm.clearmoe_fold_basis(h, G["U"], G["S"], G["Vh"], G["residuals"], G["W_comb"])
+    ms_f = timed(K, folded=True)
+    # end to end: the tokens copied in from pinned host memory, the last output copied back
+    xh = x0.cpu().pin_memory()
+    outh = torch.empty(x0.shape, dtype=x0.dtype).pin_memory()
+    xd = torch.empty_like(x0)
+    Ke = max(1, min(K, 10))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(Ke):
+        xd.copy_(xh, non_blocking=True)
+        outh.copy_(stack_pass(xd), non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_value = world * T * Ke / (e0.elapsed_time(e1) / 1e3)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n = 2048
+        t0 = time.perf_counter()
+        xs = S["x"][:n].astype(np.float64)
+        for L in S["layers"]:
+            xs = O.stack_next_input(O.stack_layer(xs, L))
+        el = time.perf_counter() - t0
+        cpu = {"value": n / el, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle",
+               "sample": f"the first {n} tokens through all 12 sublayers ({el:.1f} s; float64 oracle)"}
+    cm.clearmoe_layer_destroy(h)
+    line = {
+        "metric": "ViT-B 12-sublayer FFN stack tokens/sec (6 CLEAR-MoE + 6 dense sublayers, LayerNorm between)",
+        "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": sh.name, "T": T, "d": sh.d, "H": sh.H, "E": sh.E, "r": sh.r,
+                   "layers": sh.layers, "moe_layers": list(sh.moe_layers),
+                   "l2": "no flush: each pass reads 155 MB of tokens and ~100 MB of weights (> L2)",
+                   "parallelism": f"replicas{world}"},
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": int(x0.numel() * 2),
+                "d2h_bytes_per_step": int(x0.numel() * 2), "note": "copies not overlapped with compute"},
+        "gpu_launches": 6 * 4 + 6 * 2 + 12,
+        "cpu_baseline": cpu,
+        "clocks": clk.summary(),
+        "folded": {"value": world * T / (ms_f / 1e3), "unit": "tokens/s", "ms_per_step": ms_f},
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -220,6 +356,8 @@ def main():
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "vit_base_stack12":
+        return run_stack(args)
 
     import numpy as np
     import torch
