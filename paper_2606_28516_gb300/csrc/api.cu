@@ -333,6 +333,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         g2.scale = S_r;
         g2.C = L->t;
         g2.ldc = r;
+        g2.a_evict_first = 1;  // z is streamed once here; its rows still in L2 from fc1 stay there
         rc = cuda_fail(p2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
         if (rc) return rc;
     }

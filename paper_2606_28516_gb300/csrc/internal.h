@@ -110,6 +110,9 @@ struct TcGemmArgs {
     int32_t* rt_perm;
     int32_t* rt_out_counts;
     int32_t* rt_out_offsets;
+    // 2-SM kernel: A tiles loaded with the L2 evict-first policy (a stream read once), so that they
+    // displace one another rather than lines the next reads are still to find in L2
+    int a_evict_first;
 };
 int tc_pick_bn(int mode, int N);
 // 2-SM (cta_group::2) variant for the dense and grouped modes: 256 x BN tiles per CTA pair, BN =

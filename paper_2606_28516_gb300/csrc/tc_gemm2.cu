@@ -68,6 +68,19 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar_cluster)
         : "memory");
 }
+__device__ __forceinline__ void tma_load_2d_pair_hint(uint32_t dst, const CUtensorMap* map, int32_t c0, int32_t c1,
+                                                      uint32_t bar_cluster, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2.L2::cache_hint"
+        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar_cluster), "l"(policy)
+        : "memory");
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
 __device__ __forceinline__ void umma2_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                            uint32_t accumulate) {
     asm volatile(
@@ -280,6 +293,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         // ------------------------------------------------ producers (both CTAs)
         if (lane == 0) {
             const uint32_t full_leader0 = map_to_rank(full_bar(0), 0);
+            const uint64_t pol_a = l2_policy_evict_first();
             int stage = 0;
             uint32_t ph = 0;
             bool ok = true;
@@ -312,7 +326,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                         mB = &a.tmB0;
                         kk = (kb - nk1) * BK;
                     }
-                    tma_load_2d_pair(sA, mA, kk, am, fb);
+                    if (a.a_evict_first)
+                        tma_load_2d_pair_hint(sA, mA, kk, am, fb, pol_a);
+                    else
+                        tma_load_2d_pair(sA, mA, kk, am, fb);
                     tma_load_2d_pair(sB, mB, kk, bn, fb);
                     if (++stage == STAGES) {
                         stage = 0;
