@@ -50,6 +50,33 @@ def token_forward(x_t, W1, b1, U, S, Vh, residuals, e: int):
     return y
 
 
+def dense_token(x_t, W1, b1, W2):
+    """y_i = sum_j W2[i][j] GELU(W1 x_t + b1)_j: the unconverted layer on one token."""
+    z = []
+    for j in range(len(W1)):
+        u = float(b1[j])
+        for k in range(len(x_t)):
+            u += float(W1[j][k]) * float(x_t[k])
+        z.append(_gelu(u))
+    return [sum(float(W2[i][j]) * z[j] for j in range(len(z))) for i in range(len(W2))]
+
+
+def layer_ex(x, W1, b1, U, S, Vh, residuals, Wg, bg, W2, b2, cls_stride):
+    """Tokens t with t % cls_stride == 0 (cls_stride > 0) take the dense layer and the group
+    index len(residuals); the others as in `layer`; b2 (or None) is added to every output."""
+    a, y = [], []
+    for t, x_t in enumerate(x):
+        if cls_stride > 0 and t % cls_stride == 0:
+            e = len(residuals)
+            row = dense_token(x_t, W1, b1, W2)
+        else:
+            e = token_expert(x_t, Wg, bg)
+            row = token_forward(x_t, W1, b1, U, S, Vh, residuals, e)
+        a.append(e)
+        y.append([v + (float(b2[i]) if b2 is not None else 0.0) for i, v in enumerate(row)])
+    return a, y
+
+
 def layer(x, W1, b1, U, S, Vh, residuals, Wg, bg):
     """Returns (expert per token, output rows) for every token of x."""
     a, y = [], []

@@ -144,9 +144,51 @@ def ffn_forward_folded(x, W1, b1, W_comb, Wg=None, bg=None, a=None,
     return experts_forward(z, np.zeros((f64(W_comb[0]).shape[0], z.shape[1])), W_comb, a)
 
 
-def dense_ffn(x, W1, b1, W2, z_bf16: bool = False) -> np.ndarray:
-    """The unconverted layer: y = W2 GELU(W1 x + b1) (the dense FFN, D0)."""
-    return fc1_gelu(x, W1, b1, z_bf16) @ f64(W2).T
+def dense_ffn(x, W1, b1, W2, z_bf16: bool = False, b2=None) -> np.ndarray:
+    """The unconverted layer: y = W2 GELU(W1 x + b1) (the dense FFN, D0), + b2 when given."""
+    return fc2_bias(fc1_gelu(x, W1, b1, z_bf16) @ f64(W2).T, b2)
+
+
+# ---------------------------------------------------------------- deployment: fc2 bias, class tokens
+def fc2_bias(y, b2) -> np.ndarray:
+    """y + b2 on every row: the fc2 bias of the pretrained layer, which Eq. 2 leaves out (a bias
+    is unchanged by the SVD split of W2, so it is added once per token, outside both terms)."""
+    return f64(y) if b2 is None else f64(y) + f64(b2)
+
+
+def class_mask(T: int, cls_stride: int) -> np.ndarray:
+    """Class tokens among T: token t with t % cls_stride == 0 (the class token leads each image's
+    cls_stride tokens, 197 for a ViT at 224 px, patch 16); none when cls_stride is 0."""
+    t = np.arange(T)
+    return t % cls_stride == 0 if cls_stride > 0 else np.zeros(T, dtype=bool)
+
+
+def route_ex(x, Wg, bg, cls_stride: int = 0) -> dict:
+    """Routing with the class token kept out of expert dispatch and run on the dense path (the
+    dispatch micro-benchmark table, appendix "Dispatch Benchmark and Parallel Scaling", excludes
+    it from dispatch and processes it on the dense path): class tokens skip the router and
+    form group E, placed after every expert's group, in token order (counts: E + 1 entries,
+    offsets: E + 2)."""
+    E = np.asarray(Wg).shape[0]
+    rt = route(x, Wg, bg)
+    cls = class_mask(len(rt["a"]), cls_stride)
+    a = np.where(cls, E, rt["a"])
+    return sort_by_expert(a, E + (1 if cls_stride > 0 else 0)) | dict(near_tie=rt["near_tie"] & ~cls)
+
+
+def ffn_forward_ex(x, W1, b1, U, S, Vh, residuals, Wg=None, bg=None, a=None, W2=None, b2=None,
+                   cls_stride: int = 0, z_bf16: bool = False) -> np.ndarray:
+    """Eq. 2 as deployed: a routed token gets y_t = W_shared z_t + W_{a_t}^res z_t + b2, a class
+    token y_t = W2 z_t + b2 (the unconverted fc2, the dense path). `a` as in ffn_forward (its
+    entries for class tokens are not used)."""
+    if a is None:
+        a = route(x, Wg, bg)["a"]
+    z = fc1_gelu(x, W1, b1, z_bf16)
+    cls = class_mask(z.shape[0], cls_stride)
+    y = experts_forward(z, shared_weight(U, S, Vh), residuals, np.where(cls, 0, a))
+    if cls.any():
+        y[cls] = z[cls] @ f64(W2).T
+    return fc2_bias(y, b2)
 
 
 # ---------------------------------------------------------------- the 12-sublayer stack

@@ -166,6 +166,76 @@ def test_folded_forward_brute_force():
     assert check_folded_brute()
 
 
+# ------------------------------------------------------------------ fc2 bias and class tokens
+def check_cls_all_dense(seed=6):
+    """cls_stride = 1: every token is a class token, so the layer is the unconverted FFN (+ b2)
+    whatever the residuals and the router say."""
+    rng = np.random.default_rng(seed)
+    L = rand_layer(rng, 30, 12, 40, 3, 5)
+    b2 = rng.standard_normal(12)
+    y = O.ffn_forward_ex(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], L["residuals"],
+                         L["Wg"], L["bg"], W2=L["W2"], b2=b2, cls_stride=1)
+    want = O.dense_ffn(L["x"], L["W1"], L["b1"], L["W2"]) + b2
+    return rel_err(y, want) <= 1e-12
+
+
+def check_cls_brute(seed=7, T=23, d=16, H=64, E=3, r=6, stride=5):
+    """Class tokens and b2 against the pure-Python per-token loops (dense layer for t % 5 == 0)."""
+    rng = np.random.default_rng(seed)
+    L = rand_layer(rng, T, d, H, E, r)
+    b2 = rng.standard_normal(d)
+    a_b, y_b = B.layer_ex(L["x"].tolist(), L["W1"].tolist(), L["b1"].tolist(), L["U"].tolist(),
+                          L["S"].tolist(), L["Vh"].tolist(), L["residuals"].tolist(),
+                          L["Wg"].tolist(), L["bg"].tolist(), L["W2"].tolist(), b2.tolist(), stride)
+    rt = O.route_ex(L["x"], L["Wg"], L["bg"], stride)
+    y = O.ffn_forward_ex(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], L["residuals"],
+                         a=np.array(a_b), W2=L["W2"], b2=b2, cls_stride=stride)
+    free = ~rt["near_tie"]
+    a_b = np.array(a_b)
+    # slots: experts' tokens in (expert, id) order, then the class tokens in id order
+    want_perm = np.array(sorted(range(T), key=lambda t: (a_b[t], t)))
+    return (np.array_equal(rt["a"][free], a_b[free]) and np.array_equal(rt["perm"], want_perm)
+            and rt["counts"][E] == len(range(0, T, stride)) and rel_err(y, np.array(y_b)) <= 1e-12)
+
+
+def check_cls_keeps_routed_rows(seed=8):
+    """Rows of routed tokens are those of Eq. 2 (ffn_forward) shifted by b2; class rows differ."""
+    rng = np.random.default_rng(seed)
+    L = rand_layer(rng, 40, 10, 36, 4, 4)
+    b2 = rng.standard_normal(10)
+    args = (L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], L["residuals"], L["Wg"], L["bg"])
+    y0 = O.ffn_forward(*args)
+    y = O.ffn_forward_ex(*args, W2=L["W2"], b2=b2, cls_stride=7)
+    cls = np.arange(40) % 7 == 0
+    return (np.max(np.abs(y[~cls] - b2 - y0[~cls])) <= 1e-12
+            and np.min(np.abs(y[cls] - b2 - y0[cls]).max(axis=1)) > 1e-6)
+
+
+def test_class_tokens_all_dense():
+    assert check_cls_all_dense()
+
+
+def test_class_tokens_and_b2_brute_force():
+    assert check_cls_brute()
+    assert check_cls_brute(seed=9, T=9, stride=1)   # all class tokens
+    assert check_cls_brute(seed=10, T=5, stride=8)  # one class token, T < stride
+
+
+def test_class_tokens_keep_routed_rows():
+    assert check_cls_keeps_routed_rows()
+
+
+def test_routing_with_class_tokens_invariants():
+    rng = np.random.default_rng(11)
+    L = rand_layer(rng, 197 * 3, 8, 16, 5, 2)
+    rt = O.route_ex(L["x"], L["Wg"], L["bg"], 197)
+    T = 197 * 3
+    assert np.array_equal(rt["a"][[0, 197, 394]], [5, 5, 5]) and rt["counts"][5] == 3
+    assert rt["offsets"][5] == T - 3 and rt["offsets"][6] == T
+    assert np.array_equal(rt["perm"][T - 3:], [0, 197, 394])
+    assert np.array_equal(np.sort(rt["perm"]), np.arange(T))
+
+
 # ------------------------------------------------------------------ brute force
 def check_brute(seed, T=23, d=16, H=64, E=4, r=16):
     rng = np.random.default_rng(seed)
@@ -296,6 +366,10 @@ MUTATIONS = {
         1 / O.f64(S)) @ O.f64(Vh)),
     "fold drops the shared term": ("fold_basis", lambda U, S, Vh, res: np.stack(
         [O.f64(R) for R in res])),
+    "class tokens routed to experts": ("class_mask", lambda T, s: np.zeros(T, dtype=bool)),
+    "fc2 bias added twice": ("fc2_bias", lambda y, b2: O.f64(y) if b2 is None else O.f64(y) + 2 * O.f64(b2)),
+    "class token is every token after the first": ("class_mask", lambda T, s: (
+        np.arange(T) % s != 0) if s > 0 else np.zeros(T, dtype=bool)),
     "unsorted sub-batches": ("sort_by_expert", lambda a, E: dict(
         a=np.asarray(a), counts=np.bincount(a, minlength=E),
         offsets=np.concatenate([[0], np.cumsum(np.bincount(a, minlength=E))]),
@@ -309,7 +383,7 @@ def test_pins_catch_planted_mistakes(name, monkeypatch):
     monkeypatch.setattr(O, attr, fake)
     checks = [check_gelu_table, check_worked_example, check_dense_reduction,
               check_d3_identity, check_scalar_residual, lambda: check_brute(0), check_fold_d3,
-              check_folded_brute]
+              check_folded_brute, check_cls_all_dense, check_cls_brute, check_cls_keeps_routed_rows]
     results = []
     for c in checks:
         try:
