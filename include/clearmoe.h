@@ -103,6 +103,32 @@ int clearmoe_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const 
                          const void* const* residual_e, const clearmoe_router* router,
                          int32_t E, int32_t r, void* out, void* stream);
 
+/* Deployment options of clearmoe_ffn_forward_ex (zero-initialise, then set the fields used).
+ *  b2          fc2's bias [d] in the layer dtype (device), added once to every output row; NULL:
+ *              none (Eq. 2 as printed has no fc2 bias; a pretrained ViT layer has one).
+ *  cls_stride  > 0: token t with t % cls_stride == 0 is a class token (cls_stride = tokens per
+ *              image, 197 for a 224 px ViT at patch 16, the class token first): it skips the router
+ *              and takes the dense path out_t = W2 z_t (+ b2), as the dispatch benchmark keeps the
+ *              class token out of expert dispatch. The class tokens form group E after the experts:
+ *              idx = E, counts[E] = n_cls = ceil(T / cls_stride), slots [T - n_cls, T) in token
+ *              order. Requires W2 and E + 1 <= 16 (EUNSUPPORTED otherwise). 0: every token routed.
+ *  W2          the layer's dense fc2 [d x H] row-major (device), read for class tokens only. */
+typedef struct {
+    const void* b2;
+    int64_t cls_stride;
+    const void* W2;
+} clearmoe_ffn_options;
+
+/* clearmoe_ffn_forward with deployment options (opt may be NULL: then identical to it). With
+ * class tokens the basis step covers the routed slots only and the grouped GEMM has E + 1 groups,
+ * the last one z x W2^T alone. EINVAL for cls_stride < 0 or > 2^30, a misaligned b2 or W2, or a
+ * NULL W2 with cls_stride > 0. */
+int clearmoe_ffn_forward_ex(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                            const void* b1, const void* U_r, const float* S_r, const void* Vh_r,
+                            const void* const* residual_e, const clearmoe_router* router,
+                            int32_t E, int32_t r, const clearmoe_ffn_options* opt, void* out,
+                            void* stream);
+
 /* The shared basis folded into the experts (Eq. 2 regrouped; the paper materialises W_shared in
  * Phase 3): W_comb[e] = U_r diag(S_r) Vh_r + residual_e[e] for e < E, so that the layer output is
  * y_t = W_comb[a_t] GELU(W1 x_t + b1). W_shared is formed in fp32 (products in fp32, summed over
@@ -125,6 +151,12 @@ int clearmoe_ffn_forward_folded(clearmoe_layer* layer, const void* x, int64_t T,
 int clearmoe_dense_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
                                const void* b1, const void* W2, void* out, void* stream);
 
+/* The dense FFN with fc2's bias: out = W2 GELU(W1 x + b1) + b2, b2 [d] in the layer dtype
+ * (NULL: as clearmoe_dense_ffn_forward). */
+int clearmoe_dense_ffn_forward_ex(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                                  const void* b1, const void* W2, const void* b2, void* out,
+                                  void* stream);
+
 /* Per-token LayerNorm without affine between stacked sublayers: x_out = (y - mean(y)) /
  * sqrt(var(y) + 1e-6), biased variance, fp32 statistics; y and x_out [T x d] in the layer's
  * dtype (they may alias). 1 <= T <= max_tokens. */
@@ -132,8 +164,9 @@ int clearmoe_layer_norm(clearmoe_layer* layer, const void* y, int64_t T, void* x
                         void* stream);
 
 /* Copies (device to device, on `stream`) the routing of the last clearmoe_route /
- * clearmoe_ffn_forward on this handle: idx [T], counts [E], offsets [E + 1], perm [T], all
- * int32 device pointers; any may be NULL to skip it. EINVAL if no forward has run yet. */
+ * clearmoe_ffn_forward on this handle: idx [T], counts [G], offsets [G + 1], perm [T], all
+ * int32 device pointers, G = E (E + 1 when that forward had class tokens: group E is theirs);
+ * any may be NULL to skip it. EINVAL if no forward has run yet. */
 int clearmoe_get_routing(clearmoe_layer* layer, int32_t* idx, int32_t* counts, int32_t* offsets,
                          int32_t* perm, void* stream);
 

@@ -32,6 +32,10 @@ class clearmoe_router(ctypes.Structure):
     _fields_ = [("W", ctypes.c_void_p), ("b", ctypes.c_void_p)]
 
 
+class clearmoe_ffn_options(ctypes.Structure):
+    _fields_ = [("b2", ctypes.c_void_p), ("cls_stride", ctypes.c_int64), ("W2", ctypes.c_void_p)]
+
+
 _P, _I64, _I32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
 _SIGS = {
     "clearmoe_layer_create": [ctypes.POINTER(clearmoe_layer_desc), ctypes.POINTER(ctypes.c_void_p)],
@@ -39,7 +43,11 @@ _SIGS = {
     "clearmoe_route": [_P, _P, _I64, ctypes.POINTER(clearmoe_router), _I32, _P],
     "clearmoe_ffn_forward": [_P, _P, _I64, _P, _P, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
                              ctypes.POINTER(clearmoe_router), _I32, _I32, _P, _P],
+    "clearmoe_ffn_forward_ex": [_P, _P, _I64, _P, _P, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
+                                ctypes.POINTER(clearmoe_router), _I32, _I32,
+                                ctypes.POINTER(clearmoe_ffn_options), _P, _P],
     "clearmoe_dense_ffn_forward": [_P, _P, _I64, _P, _P, _P, _P, _P],
+    "clearmoe_dense_ffn_forward_ex": [_P, _P, _I64, _P, _P, _P, _P, _P, _P],
     "clearmoe_layer_norm": [_P, _P, _I64, _P, _P],
     "clearmoe_get_routing": [_P, _P, _P, _P, _P, _P],
     "clearmoe_layer_status": [_P],
@@ -136,6 +144,20 @@ def clearmoe_ffn_forward(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, 
            "clearmoe_ffn_forward")
 
 
+def clearmoe_ffn_forward_ex(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, bg, out,
+                            b2=None, W2=None, cls_stride: int = 0, stream=None) -> None:
+    """clearmoe_ffn_forward with fc2's bias b2 and class tokens (every cls_stride-th token from
+    token 0) on the dense path W2."""
+    E = Wg.shape[0]
+    res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
+    r = _router(Wg, bg)
+    opt = clearmoe_ffn_options(_ptr(b2), int(cls_stride), _ptr(W2))
+    _check(lib().clearmoe_ffn_forward_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), _ptr(U_r),
+                                         _ptr(S_r), _ptr(Vh_r), res, ctypes.byref(r), E,
+                                         S_r.shape[0], ctypes.byref(opt), _ptr(out),
+                                         _stream(stream)), "clearmoe_ffn_forward_ex")
+
+
 def clearmoe_fold_basis(layer: int, U_r, S_r, Vh_r, residual_e, W_comb, stream=None) -> None:
     """residual_e, W_comb: sequences of E [d x H] tensors, or [E x d x H] tensors."""
     E = len(residual_e)
@@ -158,6 +180,12 @@ def clearmoe_dense_ffn_forward(layer: int, x, W1, b1, W2, out, stream=None) -> N
     _check(lib().clearmoe_dense_ffn_forward(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
                                             _ptr(W2), _ptr(out), _stream(stream)),
            "clearmoe_dense_ffn_forward")
+
+
+def clearmoe_dense_ffn_forward_ex(layer: int, x, W1, b1, W2, b2, out, stream=None) -> None:
+    _check(lib().clearmoe_dense_ffn_forward_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
+                                               _ptr(W2), _ptr(b2), _ptr(out), _stream(stream)),
+           "clearmoe_dense_ffn_forward_ex")
 
 
 def clearmoe_layer_norm(layer: int, y, x_out, stream=None) -> None:

@@ -29,6 +29,7 @@ struct clearmoe_layer {
     int rt_grid, rt_chunk;
     int64_t last_T;
     int32_t last_E;
+    int32_t last_groups;  // last_E, + 1 when class tokens formed the dense path's group
     cudaEvent_t prof[8];
     int32_t prof_n;
 };
@@ -59,7 +60,7 @@ int check_common(const clearmoe_layer* L, const void* x, int64_t T) {
 }
 
 int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router, int E,
-             cudaStream_t s) {
+             int64_t cls_stride, cudaStream_t s) {
     int grid = 0, chunk = 0;
     const int g = cm::route_grid(T, L->desc.d, E, L->desc.dtype, L->num_sms, &grid, &chunk);
     if (g) return g == -2 ? CLEARMOE_EUNSUPPORTED : CLEARMOE_ECUDA;
@@ -83,12 +84,14 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
     a.debug_skip = L->phantom > 0 ? 0 : -1;
     a.wait_limit_ns = L->wait_limit_ns;
     a.status = L->status;
+    a.cls_stride = cls_stride;
     L->rt_grid = grid;
     L->rt_chunk = chunk;
     const int rc = cuda_fail(cm::launch_route(a, grid, chunk, s));
     if (rc == CLEARMOE_OK) {
         L->last_T = T;
         L->last_E = E;
+        L->last_groups = E + (cls_stride > 0 ? 1 : 0);
     }
     return rc;
 }
@@ -195,20 +198,26 @@ int clearmoe_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_r
     if (rc) return rc;
     if ((rc = check_router(L, router, E))) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if ((rc = do_route(L, x, T, router, E, s))) return rc;
+    if ((rc = do_route(L, x, T, router, E, 0, s))) return rc;
     return do_finalize(L, s);
 }
 
 static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
                     const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
-                    const clearmoe_router* router, int E, int r, void* out, cudaStream_t s) {
+                    const clearmoe_router* router, int E, int r, const clearmoe_ffn_options* opt, void* out,
+                    cudaStream_t s) {
     // U_r == nullptr: the folded forward, residual_e holds W_comb (no basis step, no t segment)
     const bool folded = U_r == nullptr;
     const int d = L->desc.d, H = L->desc.hidden;
     const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
+    // class tokens: group E after the experts (slots [T - n_cls, T)), K chain z x W2 alone
+    const int64_t cls_stride = opt ? opt->cls_stride : 0;
+    const int64_t n_cls = cm::n_class_tokens(T, cls_stride);
+    const int G = E + (cls_stride > 0 ? 1 : 0);  // groups of the grouped GEMM
+    const void* b2 = opt ? opt->b2 : nullptr;
     int rc;
     mark(L, 0, s);
-    if ((rc = do_route(L, x, T, router, E, s))) return rc;
+    if ((rc = do_route(L, x, T, router, E, cls_stride, s))) return rc;
     // bf16 with the 2-SM fc1: the fc1 epilogue assigns the slots itself (no finalize launch)
     const int p1 = bf16 && H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;
     const bool fused = p1 && L->rt_grid <= 256 && L->rt_grid * E <= cm::TC2_TAB_CAP;
@@ -238,7 +247,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
             g.lda0 = H;
             g.K0 = H;
             g.B0 = static_cast<const float*>(Vh_r);
-            g.M = T;
+            g.M = T - n_cls;  // the routed slots (class tokens' follow them)
             g.N = r;
             g.scale = S_r;
             g.C = static_cast<float*>(L->t);
@@ -258,13 +267,18 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         g.lda1 = H;
         g.K1 = H;
         for (int e = 0; e < E; ++e) g.B1[e] = static_cast<const float*>(residual_e[e]);
+        if (n_cls > 0) {
+            g.B1[E] = static_cast<const float*>(opt->W2);
+            g.dense_last = 1;
+        }
+        g.bias = static_cast<const float*>(b2);
         g.M = T;
         g.N = d;
         g.C = static_cast<float*>(out);
         g.ldc = d;
         g.c_rows = L->perm;
         g.offsets = L->offsets;
-        g.E = E;
+        g.E = G;
         rc = cuda_fail(cm::launch_simt_gemm(g, s));
         mark(L, 4, s);
         return rc;
@@ -302,6 +316,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
             g.rt_perm = L->perm;
             g.rt_out_counts = L->counts;
             g.rt_out_offsets = L->offsets;
+            g.rt_cls_stride = cls_stride;
         } else {
             g.rows = L->inv;
         }
@@ -327,7 +342,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
             return CLEARMOE_ECUDA;
         g2.mode = cm::TC_DENSE;
         g2.epi = cm::TC_EPI_SCALE;
-        g2.M = T;
+        g2.M = T - n_cls;  // the routed slots (class tokens' follow them)
         g2.N = r;
         g2.K0 = H;
         g2.scale = S_r;
@@ -351,6 +366,11 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         return CLEARMOE_ECUDA;
     for (int e = 0; e < E; ++e)
         if (encode_tmap_bf16(&g3.tmB1[e], residual_e[e], d, H, box3)) return CLEARMOE_ECUDA;
+    if (n_cls > 0) {  // the dense path's group: W2
+        if (encode_tmap_bf16(&g3.tmB1[E], opt->W2, d, H, box3)) return CLEARMOE_ECUDA;
+        g3.dense_last = 1;
+    }
+    g3.out_bias = b2;
     g3.mode = cm::TC_GROUPED;
     g3.epi = cm::TC_EPI_SCATTER;
     g3.M = T;
@@ -358,7 +378,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     g3.K0 = folded ? 0 : r;  // folded: the K chain is z x W_e^comb alone
     g3.K1 = H;
     g3.offsets = L->offsets;
-    g3.E = E;
+    g3.E = G;
     g3.rows = L->perm;
     g3.C = out;
     g3.ldc = d;
@@ -370,9 +390,24 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
 int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
                          const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
                          const clearmoe_router* router, int32_t E, int32_t r, void* out, void* stream) {
+    return clearmoe_ffn_forward_ex(L, x, T, W1, b1, U_r, S_r, Vh_r, residual_e, router, E, r, nullptr, out, stream);
+}
+
+int clearmoe_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                            const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
+                            const clearmoe_router* router, int32_t E, int32_t r, const clearmoe_ffn_options* opt,
+                            void* out, void* stream) {
     int rc = check_common(L, x, T);
     if (rc) return rc;
     if ((rc = check_router(L, router, E))) return rc;
+    if (opt) {
+        if (opt->cls_stride < 0 || opt->cls_stride > ((int64_t)1 << 30)) return CLEARMOE_EINVAL;
+        if (opt->b2 && misaligned(opt->b2)) return CLEARMOE_EINVAL;
+        if (opt->cls_stride > 0) {
+            if (!opt->W2 || misaligned(opt->W2)) return CLEARMOE_EINVAL;
+            if (E + 1 > CM_MAX_E) return CLEARMOE_EUNSUPPORTED;  // the dense path takes a group
+        }
+    }
     if (!W1 || !b1 || !U_r || !S_r || !Vh_r || !residual_e || !out) return CLEARMOE_EINVAL;
     const int d = L->desc.d, H = L->desc.hidden;
     if (r < 1 || r > L->desc.max_r || r > d || r > H) return CLEARMOE_EINVAL;
@@ -384,7 +419,7 @@ int clearmoe_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void
     const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
     if (bf16 && r % 16) return CLEARMOE_EUNSUPPORTED;
     if (!bf16 && r % 4) return CLEARMOE_EUNSUPPORTED;
-    return ffn_impl(L, x, T, W1, b1, U_r, S_r, Vh_r, residual_e, router, E, r, out,
+    return ffn_impl(L, x, T, W1, b1, U_r, S_r, Vh_r, residual_e, router, E, r, opt, out,
                     static_cast<cudaStream_t>(stream));
 }
 
@@ -398,7 +433,7 @@ int clearmoe_ffn_forward_folded(clearmoe_layer* L, const void* x, int64_t T, con
     for (int e = 0; e < E; ++e)
         if (!W_comb[e] || misaligned(W_comb[e])) return CLEARMOE_EINVAL;
     if (misaligned(W1) || misaligned(b1) || misaligned(out)) return CLEARMOE_EINVAL;
-    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, W_comb, router, E, 0, out,
+    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, W_comb, router, E, 0, nullptr, out,
                     static_cast<cudaStream_t>(stream));
 }
 
@@ -427,10 +462,16 @@ int clearmoe_fold_basis(clearmoe_layer* L, const void* U_r, const float* S_r, co
 
 int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
                                const void* W2, void* out, void* stream) {
+    return clearmoe_dense_ffn_forward_ex(L, x, T, W1, b1, W2, nullptr, out, stream);
+}
+
+int clearmoe_dense_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                                  const void* W2, const void* b2, void* out, void* stream) {
     int rc = check_common(L, x, T);
     if (rc) return rc;
     if (!W1 || !b1 || !W2 || !out) return CLEARMOE_EINVAL;
-    if (misaligned(W1) || misaligned(b1) || misaligned(W2) || misaligned(out)) return CLEARMOE_EINVAL;
+    if (misaligned(W1) || misaligned(b1) || misaligned(W2) || misaligned(out) || misaligned(b2))
+        return CLEARMOE_EINVAL;
     const int d = L->desc.d, H = L->desc.hidden;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     mark(L, 0, s);
@@ -454,6 +495,7 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
         g.lda0 = H;
         g.K0 = H;
         g.B0 = static_cast<const float*>(W2);
+        g.bias = static_cast<const float*>(b2);
         g.M = T;
         g.N = d;
         g.C = static_cast<float*>(out);
@@ -491,6 +533,7 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
         return CLEARMOE_ECUDA;
     g2.mode = cm::TC_DENSE;
     g2.epi = cm::TC_EPI_STORE;
+    g2.out_bias = b2;
     g2.M = T;
     g2.N = d;
     g2.K0 = H;
@@ -513,7 +556,7 @@ int clearmoe_get_routing(clearmoe_layer* L, int32_t* idx, int32_t* counts, int32
     if (!L) return CLEARMOE_EINVAL;
     if (L->last_T < 1) return CLEARMOE_EINVAL;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const size_t T = (size_t)L->last_T, E = (size_t)L->last_E;
+    const size_t T = (size_t)L->last_T, E = (size_t)L->last_groups;
     cudaError_t e = cudaSuccess;
     if (idx && e == cudaSuccess) e = cudaMemcpyAsync(idx, L->idx, T * 4, cudaMemcpyDeviceToDevice, s);
     if (counts && e == cudaSuccess) e = cudaMemcpyAsync(counts, L->counts, E * 4, cudaMemcpyDeviceToDevice, s);

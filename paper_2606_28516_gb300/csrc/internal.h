@@ -25,7 +25,14 @@ struct RouteArgs {
     int debug_skip;                // fault injection: CTA 0 withholds this stage (-1: none)
     int64_t wait_limit_ns;
     int32_t* status;
+    // > 0: token t with t % cls_stride == 0 is a class token: it skips the router and forms group
+    // E (idx = E), the dense path, whose slots follow every expert's: T - n_cls + t / cls_stride
+    int64_t cls_stride;
 };
+// Class tokens of T: every cls_stride-th from token 0 (none when cls_stride is 0).
+__host__ __device__ inline int64_t n_class_tokens(int64_t T, int64_t cls_stride) {
+    return cls_stride > 0 ? (T + cls_stride - 1) / cls_stride : 0;
+}
 
 // Grid of the routing kernel for T tokens (one or two CTAs per SM); chunk = rows per CTA (a
 // routing range). Returns 0, -1 on a CUDA error, -2 when no launch shape fits.
@@ -70,6 +77,7 @@ struct SimtGemmArgs {
     const int32_t* c_rows;   // scatter rows of C (nullable)
     const int32_t* offsets;  // grouped: expert boundaries [E + 1] (nullable = not grouped)
     int E;
+    int dense_last;          // grouped: the last group (the dense path) has no first K segment
 };
 cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s);
 
@@ -110,6 +118,14 @@ struct TcGemmArgs {
     int32_t* rt_perm;
     int32_t* rt_out_counts;
     int32_t* rt_out_offsets;
+    // store / scatter epilogues: + out_bias[n] (bf16 [N], nullable; the 2-SM kernel stages it in
+    // shared memory, N <= TC2_BIAS_CAP)
+    const void* out_bias;
+    // grouped: the last of the E groups is the dense path (class tokens), whose K chain is the
+    // z x B1 segment alone
+    int dense_last;
+    // fused fc1: class tokens (t % rt_cls_stride == 0) go to slot M - n_cls + t / rt_cls_stride
+    int64_t rt_cls_stride;
     // 2-SM kernel: A tiles loaded with the L2 evict-first policy (a stream read once), so that they
     // displace one another rather than lines the next reads are still to find in L2
     int a_evict_first;

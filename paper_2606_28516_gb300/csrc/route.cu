@@ -18,6 +18,8 @@
 // them through L1 in the inner loop was measured slower), and the K order of each fragment is
 // permuted identically for x and W_g, which leaves every dot product unchanged.
 // fp32 tokens: fp32 FMA on the CUDA cores (an fp32 router decision needs fp32 products).
+// Class tokens (cls_stride > 0, t % cls_stride == 0) skip the router: idx = E, no histogram entry
+// and no rank; their slots T - n_cls + t / cls_stride follow the experts' (the dense path).
 #include <mutex>
 
 #include "common.cuh"
@@ -138,7 +140,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     auto record = [&](int i, int e, int rank) {  // phase 1 result of row i: idx, its word, histogram
         a.idx[row0 + i] = e;
         if (sinfo) sinfo[i] = (uint32_t)e | ((uint32_t)rank << 8);
-        atomicAdd(&s_count[e], 1);
+        if (e < E) atomicAdd(&s_count[e], 1);  // e == E: a class token
     };
 
     if (tid < CM_MAX_E) s_count[tid] = 0;
@@ -295,6 +297,11 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 }
                 if (eA > E - 1) eA = 0;  // only reachable with non-finite logits
                 if (eB > E - 1) eB = 0;
+                if (a.cls_stride > 0) {  // class tokens: group E, outside every expert's ballot
+                    const int64_t tA = row0 + (int64_t)k * RT_STAGE_ROWS + g;
+                    if (tA % a.cls_stride == 0) eA = E;
+                    if ((tA + 8) % a.cls_stride == 0) eB = E;
+                }
                 int rankA = 0, rankB = 0;
                 if (scnt) {
                     // rank of each row among the stage's earlier rows of its expert, from one ballot
@@ -352,6 +359,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 }
             }
             if (be > E - 1) be = 0;
+            if (a.cls_stride > 0 && (row0 + i) % a.cls_stride == 0) be = E;  // a class token
             if (lane == 0) record(i, be, 0);
         }
     }
@@ -384,9 +392,10 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         __syncthreads();
         for (int i = tid; i < nrows; i += NTHREADS) {
             const uint32_t w = sinfo[i];
-            int e = (int)(w & 0xffu);
-            if (e >= E) e = 0;  // rows a launch that gave up never routed: keep indices in range
-            a.tinfo[row0 + i] = e | ((scnt[(i / RT_STAGE_ROWS) * CM_MAX_E + e] + (int)((w >> 8) & 0xffu)) << 8);
+            const int e = (int)(w & 0xffu);
+            // class tokens (e == E) and rows a launch that gave up never routed take no slot here
+            a.tinfo[row0 + i] =
+                e < E ? e | ((scnt[(i / RT_STAGE_ROWS) * CM_MAX_E + e] + (int)((w >> 8) & 0xffu)) << 8) : E;
         }
         return;
     }
@@ -398,10 +407,12 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         const int i = i0 + tid;
         const bool valid = i < nrows;
         int e = valid ? (int)(info_of(i) & 0xffu) : CM_MAX_E + 1;
-        if (valid && e >= E) e = 0;  // rows a launch that gave up never routed: keep indices in range
+        // class tokens (e == E) and rows a launch that gave up never routed take no rank
+        const bool ranked = valid && e < E;
+        if (!ranked) e = CM_MAX_E + 1;
         const unsigned same = __match_any_sync(0xffffffffu, e);
         const int rank = __popc(same & lt);
-        if (valid && rank == 0) s_wc[warp][e] = __popc(same);
+        if (ranked && rank == 0) s_wc[warp][e] = __popc(same);
         __syncthreads();
         int pre = 0, own = 0;  // lane l < E: expert l's rows in this CTA before this warp's rows
         if (lane < E) {
@@ -409,8 +420,11 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
             for (int w = 0; w < warp; ++w) pre += s_wc[w][lane];
             own = s_wc[warp][lane];
         }
-        const int base_e = __shfl_sync(0xffffffffu, pre, valid ? e : 0);
-        if (valid) a.tinfo[row0 + i] = e | ((base_e + rank) << 8);
+        const int base_e = __shfl_sync(0xffffffffu, pre, ranked ? e : 0);
+        if (ranked)
+            a.tinfo[row0 + i] = e | ((base_e + rank) << 8);
+        else if (valid)
+            a.tinfo[row0 + i] = E;
         __syncthreads();  // every warp has read s_run and s_wc
         if (warp == NWARPS - 1 && lane < E) s_run[lane] = pre + own;
     }
@@ -420,12 +434,14 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
 // the per-expert sums of the G ranges' histograms before this one and over all (thread b reads row
 // b), offsets by a scan over experts, then slot = offsets[e] + before + local rank for every row.
 // Writes perm, inv (if set), counts and offsets (range 0), and unpacks idx when it carried the
-// packed words.
+// packed words. Class tokens take slot T - n_cls + t / cls_stride; counts[E] = n_cls and
+// offsets[E + 1] = T then describe their group.
 __global__ void __launch_bounds__(256) route_finalize_kernel(const RouteArgs a, const int chunk, const int G) {
     __shared__ int s_wb[8][CM_MAX_E], s_wt[8][CM_MAX_E], s_base[CM_MAX_E];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, E = a.E;
     const int64_t row0 = (int64_t)blockIdx.x * chunk;
     const int nrows = (int)max((int64_t)0, min((int64_t)chunk, a.T - row0));
+    const int64_t n_cls = n_class_tokens(a.T, a.cls_stride);
     pdl_wait();  // everything below reads the routing kernel's output
     pdl_launch_dependents();
     int bef[CM_MAX_E], tot[CM_MAX_E];
@@ -476,13 +492,27 @@ __global__ void __launch_bounds__(256) route_finalize_kernel(const RouteArgs a, 
             if (blockIdx.x == 0) {
                 a.counts[lane] = t;
                 a.offsets[lane] = incl - t;
-                if (lane == E - 1) a.offsets[E] = incl;
+                if (lane == E - 1) {
+                    a.offsets[E] = incl;
+                    if (n_cls > 0) {  // the dense path's group
+                        a.counts[E] = (int32_t)n_cls;
+                        a.offsets[E + 1] = incl + (int32_t)n_cls;
+                    }
+                }
             }
         }
     }
     __syncthreads();
     const bool unpack = a.tinfo == a.idx;
     for (int i = tid; i < nrows; i += 256) {
+        const int64_t tok = row0 + i;
+        if (a.cls_stride > 0 && tok % a.cls_stride == 0) {  // a class token: the dense path's slots
+            const int64_t slot = a.T - n_cls + tok / a.cls_stride;
+            a.perm[slot] = (int32_t)tok;
+            if (a.inv) a.inv[tok] = (int32_t)slot;
+            if (unpack) a.idx[tok] = E;
+            continue;
+        }
         const uint32_t w = (uint32_t)a.tinfo[row0 + i];
         const int e = (int)(w & 0xffu);
         if (e >= E) continue;  // only a routing launch that gave up leaves such words

@@ -5,7 +5,8 @@
 // on the CUDA cores. One tiled kernel covers every product of the layer:
 //   C[m, n] = epi( sum_k A0[rowA(m), k] B0[n, k]  +  sum_k A1[m, k] B1_e[n, k] )
 // with an optional row gather of A0 (fc1 on tokens in expert order), an optional second K
-// segment with a per-expert B (the grouped residual GEMM, Algorithm 3 step 5), an epilogue of
+// segment with a per-expert B (the grouped residual GEMM, Algorithm 3 step 5; with dense_last the
+// last group is the class tokens' dense path, second segment only), an epilogue of
 // bias, GELU and per-column scale, and an optional row scatter of C (the unshuffle, step 6).
 #include "common.cuh"
 #include "internal.h"
@@ -57,6 +58,7 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
         const int K = seg == 0 ? a.K0 : a.K1;
         const int64_t lda = seg == 0 ? a.lda0 : a.lda1;
         if (A == nullptr || K == 0) continue;
+        if (seg == 0 && a.offsets && a.dense_last && e == a.E - 1) continue;  // the dense path: z x W2 alone
         for (int k0 = 0; k0 < K; k0 += SG_K) {
 #pragma unroll
             for (int i = 0; i < 4; ++i) {

@@ -155,7 +155,9 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
             bool ok = true;
             for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
                 const TileInfo t = decode_tile(a, tile, n_tiles, s_prefix, BN);
-                for (int kb = 0; kb < nkb; ++kb) {
+                // the dense path's group (class tokens): the z x W2 segment alone
+                const int kb0 = (MODE == TC_GROUPED && a.dense_last && t.e == a.E - 1) ? nk0 : 0;
+                for (int kb = kb0; kb < nkb; ++kb) {
                     if (!mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim)) {
                         ok = false;
                         break;
@@ -242,7 +244,11 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
                 if (!mbar_wait(tempty_bar(acc), aph ^ 1, abort_flag, a.status, lim)) break;
                 tc_fence_after();
                 const uint32_t dtm = tmem_base + acc * BN;
-                for (int kb = 0; kb < nkb; ++kb) {
+                const int kb0 = (MODE == TC_GROUPED && a.dense_last &&
+                                 decode_tile(a, tile, n_tiles, s_prefix, BN).e == a.E - 1)
+                                    ? nk0
+                                    : 0;
+                for (int kb = kb0; kb < nkb; ++kb) {
                     if (!mbar_wait(full_bar(stage), ph, abort_flag, a.status, lim)) {
                         ok = false;
                         break;
@@ -256,7 +262,7 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
                     const int steps = kvalid >> 4;
                     for (int k = 0; k < steps; ++k)
                         umma_bf16(dtm, sdesc_kmajor_sw128(sA + k * 32), sdesc_kmajor_sw128(sB + k * 32),
-                                  idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                                  idesc, (kb > kb0 || k > 0) ? 1u : 0u);
                     umma_commit(empty_bar(stage));
                     if (++stage == C::STAGES) {
                         stage = 0;
@@ -316,6 +322,18 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
                                            make_float2(bf16_lo(bw[h]), bf16_hi(bw[h]))));
                             f[j8 * 8 + 2 * h] = g.x;
                             f[j8 * 8 + 2 * h + 1] = g.y;
+                        }
+                    }
+                } else if (a.out_bias) {
+                    const uint4* bp = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.out_bias) + nb);
+#pragma unroll
+                    for (int j8 = 0; j8 < C::CW / 8; ++j8) {
+                        const uint4 b = __ldg(bp + j8);
+                        const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+                        for (int h = 0; h < 4; ++h) {
+                            f[j8 * 8 + 2 * h] += bf16_lo(bw[h]);
+                            f[j8 * 8 + 2 * h + 1] += bf16_hi(bw[h]);
                         }
                     }
                 } else if (a.epi == TC_EPI_SCALE) {

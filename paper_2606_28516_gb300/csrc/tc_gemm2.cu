@@ -11,7 +11,9 @@
 // name it through the cluster); the even CTA's MMA commits arrive on both CTAs' empty / tfull
 // barriers (multicast); the epilogue warps of both CTAs arrive on the even CTA's tempty barrier.
 // Modes: dense (one K segment, epilogue bias+GELU / plain store) and grouped (the residual
-// experts: tile pairs never straddle an expert, K chain [z | t] x [W_e | U_r]). With a.rows set,
+// experts: tile pairs never straddle an expert, K chain [z | t] x [W_e | U_r]; with dense_last
+// the last group is the class tokens' dense path, K chain z x W2 alone). Store epilogues may add
+// an output bias (fc2's b2). With a.rows set,
 // output row m goes to C[a.rows[m]] (fc1: inv[token] = slot; grouped: perm[slot] = token).
 // Every wait is bounded; both CTAs always reach the closing cluster barrier.
 #include "common.cuh"
@@ -185,6 +187,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = __uint_as_float((uint32_t)b[n] << 16);
     } else if (MODE == TC_DENSE && a.epi == TC_EPI_SCALE && warp < NUM_EPI) {
         for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = a.scale[n];
+    } else if (a.out_bias && warp < NUM_EPI) {
+        const uint16_t* b = static_cast<const uint16_t*>(a.out_bias);
+        for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = __uint_as_float((uint32_t)b[n] << 16);
     }
     // Tensor memory for the pair: allocated collectively by one warp of each CTA. The two CTAs
     // must see the same base (the even CTA's MMAs name it for both); a mismatch aborts cleanly.
@@ -257,7 +262,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                 if (blockIdx.x == 0) {
                     a.rt_out_counts[lane] = tot;
                     a.rt_out_offsets[lane] = sc - tot;
-                    if (lane == E - 1) a.rt_out_offsets[E] = sc;
+                    if (lane == E - 1) {
+                        a.rt_out_offsets[E] = sc;
+                        const int64_t n_cls = n_class_tokens(a.M, a.rt_cls_stride);
+                        if (n_cls > 0) {  // the class tokens' group (the dense path)
+                            a.rt_out_counts[E] = (int32_t)n_cls;
+                            a.rt_out_offsets[E + 1] = sc + (int32_t)n_cls;
+                        }
+                    }
                 }
             }
         }
@@ -301,7 +313,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                 const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
                 const int am = (int)(t.m0 + (int64_t)rank * BM);
                 const int bn = t.n0 + (int)rank * BH;
-                for (int kb = 0; kb < nkb; ++kb) {
+                const int nkb_t = (MODE == TC_GROUPED && a.dense_last && t.e == a.E - 1) ? nk1 : nkb;
+                for (int kb = 0; kb < nkb_t; ++kb) {
                     if (!mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim)) {
                         ok = false;
                         break;
@@ -354,7 +367,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                 if (!mbar_wait(tempty_bar(acc), aph ^ 1, abort_flag, a.status, lim)) break;
                 tc_fence_after();
                 const uint32_t dtm = tmem_base + acc * BN;
-                for (int kb = 0; kb < nkb; ++kb) {
+                int nkb_t = nkb;  // the dense path's group: the z x W2 segment alone
+                if (MODE == TC_GROUPED && a.dense_last && decode_pair<BN>(a, u, n_tiles, s_prefix).e == a.E - 1)
+                    nkb_t = nk1;
+                for (int kb = 0; kb < nkb_t; ++kb) {
                     if (!mbar_wait(full_bar(stage), ph, abort_flag, a.status, lim)) {
                         ok = false;
                         break;
@@ -415,7 +431,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                     const uint32_t w = rtw;
                     const int e = (int)(w & 0xffu);
                     const int rc = (int)((uint32_t)mrow / (uint32_t)a.rt_chunk);  // T < 2^31
-                    if (e < a.rt_E) orow = (int64_t)s_off[e] + s_tab[rc * a.rt_E + e] + (int)(w >> 8);
+                    if (a.rt_cls_stride > 0 && (uint32_t)mrow % (uint32_t)a.rt_cls_stride == 0)  // class token
+                        orow = a.M - n_class_tokens(a.M, a.rt_cls_stride) + (uint32_t)mrow / (uint32_t)a.rt_cls_stride;
+                    else if (e < a.rt_E)
+                        orow = (int64_t)s_off[e] + s_tab[rc * a.rt_E + e] + (int)(w >> 8);
                     if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
                     if (orow >= 0 && t.n0 == 0 && c_lo == 0) a.rt_perm[orow] = (int32_t)mrow;  // once per token
                 } else {
@@ -454,6 +473,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                         f[4 * j4 + 1] = g0.y;
                         f[4 * j4 + 2] = g1.x;
                         f[4 * j4 + 3] = g1.y;
+                    }
+                } else if (a.out_bias) {
+                    const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
+#pragma unroll
+                    for (int j4 = 0; j4 < CW / 4; ++j4) {
+                        const float4 b = bp[j4];
+                        const float2 p0 = __fadd2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), make_float2(b.x, b.y));
+                        const float2 p1 = __fadd2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), make_float2(b.z, b.w));
+                        f[4 * j4] = p0.x;
+                        f[4 * j4 + 1] = p0.y;
+                        f[4 * j4 + 2] = p1.x;
+                        f[4 * j4 + 3] = p1.y;
                     }
                 } else if (a.epi == TC_EPI_SCALE) {
                     const float4* sp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
@@ -550,6 +581,7 @@ cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     const int bn = tc2_pick_bn(a.mode, a.N);
     const bool staged = a.epi == TC_EPI_BIAS_GELU || a.epi == TC_EPI_SCALE;  // fp32 vector in shared memory
     if (!bn || (staged && (a.mode != TC_DENSE || a.N > TC2_BIAS_CAP))) return cudaErrorInvalidValue;
+    if (a.out_bias && (staged || a.N > TC2_BIAS_CAP)) return cudaErrorInvalidValue;
     return bn == 256 ? launch2<256>(a, num_sms, s) : launch2<128>(a, num_sms, s);
 }
 
