@@ -443,27 +443,44 @@ def main():
         total_ms = float(t.item())
     value = world * s.T * K / (total_ms / 1e3)
 
-    # The folded variant (the shared basis folded into the experts once; same routing and fc1,
-    # one grouped GEMM over z), same timing rules. Reported beside the headline, not as it.
-    W_comb = torch.empty_like(D["residuals"]) if s.dtype == "bf16" else None
-    folded = None
-    if W_comb is not None:
-        cm.clearmoe_fold_basis(h, D["U"], D["S"], D["Vh"], D["residuals"], W_comb)
-        fev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(min(K, 300))]
-        for k in range(len(fev) + args.warmup):
+    # Variants of the same layer, same timing rules (events around each forward only, L2 flushed
+    # before each). Reported beside the headline, not as it.
+    def time_variant(fn, note):
+        vev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(min(K, 300))]
+        for k in range(len(vev) + args.warmup):
             flush.zero_()
             if k >= args.warmup:
-                fev[k - args.warmup][0].record(stream)
-            cm.clearmoe_ffn_forward_folded(h, D["x"], D["W1"], D["b1"], W_comb, D["Wg"], D["bg"], out)
+                vev[k - args.warmup][0].record(stream)
+            fn()
             if k >= args.warmup:
-                fev[k - args.warmup][1].record(stream)
+                vev[k - args.warmup][1].record(stream)
         torch.cuda.synchronize()
         assert cm.clearmoe_layer_status(h) == 0
-        f_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in fev)
-        folded = {"value": world * s.T / (f_ms / 1e3), "unit": "tokens/s", "ms_per_step": f_ms,
-                  "note": "W_e^comb = U_r diag(S_r) V_r^T + W_e^res formed once (clearmoe_fold_basis); "
-                          "forward = routing, fc1, one grouped GEMM over z"}
+        v_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in vev)
+        return {"value": world * s.T / (v_ms / 1e3), "unit": "tokens/s", "ms_per_step": v_ms, "note": note}
+
+    folded = materialized = class_tokens = None
+    if s.dtype == "bf16":
+        W_comb = torch.empty_like(D["residuals"])
+        cm.clearmoe_fold_basis(h, D["U"], D["S"], D["Vh"], D["residuals"], W_comb)
+        folded = time_variant(
+            lambda: cm.clearmoe_ffn_forward_folded(h, D["x"], D["W1"], D["b1"], W_comb, D["Wg"], D["bg"], out),
+            "W_e^comb = U_r diag(S_r) V_r^T + W_e^res formed once (clearmoe_fold_basis); "
+            "forward = routing, fc1, one grouped GEMM over z")
         del W_comb
+        W_sh = torch.empty(s.d, s.H, device="cuda", dtype=D["x"].dtype)
+        cm.clearmoe_materialize_basis(h, D["U"], D["S"], D["Vh"], W_sh)
+        materialized = time_variant(
+            lambda: cm.clearmoe_ffn_forward_materialized(h, D["x"], D["W1"], D["b1"], W_sh, D["residuals"],
+                                                         D["Wg"], D["bg"], out),
+            "the paper's materialised W_shared (clearmoe_materialize_basis once); grouped K chain "
+            "[z | z] x [W_e^res | W_shared]")
+        del W_sh
+        class_tokens = time_variant(
+            lambda: cm.clearmoe_ffn_forward_ex(h, D["x"], D["W1"], D["b1"], D["U"], D["S"], D["Vh"],
+                                               D["residuals"], D["Wg"], D["bg"], out, b2=D["b2"], W2=D["W2"],
+                                               cls_stride=197),
+            "class token of each 197-token image on the dense path (W2), fc2 bias b2 added")
 
     # same-GPU dense FFN, same timing rules (events around each forward only)
     dout = torch.empty_like(out)
@@ -599,6 +616,8 @@ def main():
         "dense_ffn": {"value": dense_value, "unit": "tokens/s",
                       "ms_per_step": statistics.mean(dense_ms)},
         "folded": folded,
+        "materialized": materialized,
+        "class_tokens": class_tokens,
         "wall_s_timed": wall,
     }
     if rank == 0:

@@ -146,6 +146,22 @@ int clearmoe_ffn_forward_folded(clearmoe_layer* layer, const void* x, int64_t T,
                                 const void* b1, const void* const* W_comb,
                                 const clearmoe_router* router, int32_t E, void* out, void* stream);
 
+/* The paper's own form of the shared basis (Phase 3 text: W_shared materialised before
+ * inference): W_sh = U_r diag(S_r) Vh_r as one [d x H] row-major matrix in the layer dtype, formed
+ * in fp32 (products in fp32, summed over k ascending) and rounded once. W_sh is a caller-owned
+ * device buffer. 1 <= r <= min(max_r, d, H). */
+int clearmoe_materialize_basis(clearmoe_layer* layer, const void* U_r, const float* S_r, const void* Vh_r,
+                               int32_t r, void* W_sh, void* stream);
+
+/* The CLEAR-MoE FFN forward with the materialised basis (Eq. 2 as the paper computes it):
+ * routing and fc1 as clearmoe_ffn_forward, then per expert sub-batch out[perm[slot]] =
+ * W_sh z + residual_e[e] z in one grouped GEMM whose K chain is [z | z] x [W_e^res | W_sh]
+ * (2 d H multiply-adds per token there, against d (H + r) + r H factorised). Same limits and
+ * errors as clearmoe_ffn_forward_folded. */
+int clearmoe_ffn_forward_materialized(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                                      const void* b1, const void* W_sh, const void* const* residual_e,
+                                      const clearmoe_router* router, int32_t E, void* out, void* stream);
+
 /* The dense FFN the layer was converted from, on the same device: out = W2 GELU(W1 x + b1)
  * (the comparison path; no bias on fc2, as in Eq. 2). 1 <= T <= max_tokens. */
 int clearmoe_dense_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,

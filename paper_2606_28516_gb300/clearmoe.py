@@ -46,6 +46,9 @@ _SIGS = {
     "clearmoe_ffn_forward_ex": [_P, _P, _I64, _P, _P, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
                                 ctypes.POINTER(clearmoe_router), _I32, _I32,
                                 ctypes.POINTER(clearmoe_ffn_options), _P, _P],
+    "clearmoe_materialize_basis": [_P, _P, _P, _P, _I32, _P, _P],
+    "clearmoe_ffn_forward_materialized": [_P, _P, _I64, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
+                                          ctypes.POINTER(clearmoe_router), _I32, _P, _P],
     "clearmoe_dense_ffn_forward": [_P, _P, _I64, _P, _P, _P, _P, _P],
     "clearmoe_dense_ffn_forward_ex": [_P, _P, _I64, _P, _P, _P, _P, _P, _P],
     "clearmoe_layer_norm": [_P, _P, _I64, _P, _P],
@@ -174,6 +177,21 @@ def clearmoe_ffn_forward_folded(layer: int, x, W1, b1, W_comb, Wg, bg, out, stre
     _check(lib().clearmoe_ffn_forward_folded(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), comb,
                                              ctypes.byref(r), E, _ptr(out), _stream(stream)),
            "clearmoe_ffn_forward_folded")
+
+
+def clearmoe_materialize_basis(layer: int, U_r, S_r, Vh_r, W_sh, stream=None) -> None:
+    _check(lib().clearmoe_materialize_basis(layer, _ptr(U_r), _ptr(S_r), _ptr(Vh_r), S_r.shape[0],
+                                            _ptr(W_sh), _stream(stream)), "clearmoe_materialize_basis")
+
+
+def clearmoe_ffn_forward_materialized(layer: int, x, W1, b1, W_sh, residual_e, Wg, bg, out,
+                                      stream=None) -> None:
+    E = Wg.shape[0]
+    res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
+    r = _router(Wg, bg)
+    _check(lib().clearmoe_ffn_forward_materialized(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
+                                                   _ptr(W_sh), res, ctypes.byref(r), E, _ptr(out),
+                                                   _stream(stream)), "clearmoe_ffn_forward_materialized")
 
 
 def clearmoe_dense_ffn_forward(layer: int, x, W1, b1, W2, out, stream=None) -> None:

@@ -203,11 +203,14 @@ int clearmoe_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_r
 }
 
 static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
-                    const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
-                    const clearmoe_router* router, int E, int r, const clearmoe_ffn_options* opt, void* out,
-                    cudaStream_t s) {
-    // U_r == nullptr: the folded forward, residual_e holds W_comb (no basis step, no t segment)
-    const bool folded = U_r == nullptr;
+                    const void* U_r, const float* S_r, const void* Vh_r, const void* W_sh,
+                    const void* const* residual_e, const clearmoe_router* router, int E, int r,
+                    const clearmoe_ffn_options* opt, void* out, cudaStream_t s) {
+    // Basis forms: factorised (U_r set: t = diag(S_r) Vh_r z, then U_r t), materialised (W_sh
+    // set: the K chain [z | z] x [W_e^res | W_sh]), folded (neither: residual_e holds W_comb, no
+    // basis step, no first K segment).
+    const bool factored = U_r != nullptr;
+    const bool materialized = !factored && W_sh != nullptr;
     const int d = L->desc.d, H = L->desc.hidden;
     const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
     // class tokens: group E after the experts (slots [T - n_cls, T)), K chain z x W2 alone
@@ -241,7 +244,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         g.ldc = H;
         if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
         mark(L, 2, s);
-        if (!folded) {  // t = diag(S_r) Vh_r z
+        if (factored) {  // t = diag(S_r) Vh_r z
             std::memset(&g, 0, sizeof(g));
             g.A0 = static_cast<const float*>(L->z);
             g.lda0 = H;
@@ -257,11 +260,16 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         mark(L, 3, s);
         // out[perm[slot]] = U_r t + W_e^res z per expert sub-batch (folded: W_e^comb z)
         std::memset(&g, 0, sizeof(g));
-        if (!folded) {
+        if (factored) {
             g.A0 = static_cast<const float*>(L->t);
             g.lda0 = r;
             g.K0 = r;
             g.B0 = static_cast<const float*>(U_r);
+        } else if (materialized) {
+            g.A0 = static_cast<const float*>(L->z);
+            g.lda0 = H;
+            g.K0 = H;
+            g.B0 = static_cast<const float*>(W_sh);
         }
         g.A1 = static_cast<const float*>(L->z);
         g.lda1 = H;
@@ -286,7 +294,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
 
     // ---- bf16: tcgen05 GEMMs
     const int bn1 = cm::tc_pick_bn(cm::TC_GATHER, H);
-    const int bn2 = folded ? 1 : cm::tc_pick_bn(cm::TC_DENSE, r);
+    const int bn2 = factored ? cm::tc_pick_bn(cm::TC_DENSE, r) : 1;
     const int bn3 = cm::tc_pick_bn(cm::TC_GROUPED, d);
     if (!bn1 || !bn2 || !bn3) return CLEARMOE_EUNSUPPORTED;
     cm::TcGemmArgs g;
@@ -331,7 +339,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     }
     if (rc) return rc;
     mark(L, 2, s);
-    if (!folded) {  // t = diag(S_r) Vh_r z (2-SM kernel when r is a multiple of 128)
+    if (factored) {  // t = diag(S_r) Vh_r z (2-SM kernel when r is a multiple of 128)
         cm::TcGemmArgs g2;
         std::memset(&g2, 0, sizeof(g2));
         g2.status = L->status;
@@ -361,7 +369,9 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     // The 2-SM kernel loads half of each pair tile's B rows per CTA: boxes of p3 / 2 rows.
     const int p3 = cm::tc2_pick_bn(cm::TC_GROUPED, d);
     const int box3 = p3 ? p3 / 2 : bn3;
-    if ((!folded && (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, box3))) ||
+    if ((factored && (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, box3))) ||
+        (materialized &&
+         (encode_tmap_bf16(&g3.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g3.tmB0, W_sh, d, H, box3))) ||
         encode_tmap_bf16(&g3.tmA1, L->z, T, H, 128))
         return CLEARMOE_ECUDA;
     for (int e = 0; e < E; ++e)
@@ -375,7 +385,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     g3.epi = cm::TC_EPI_SCATTER;
     g3.M = T;
     g3.N = d;
-    g3.K0 = folded ? 0 : r;  // folded: the K chain is z x W_e^comb alone
+    g3.K0 = factored ? r : materialized ? H : 0;  // folded: the K chain is z x W_e^comb alone
     g3.K1 = H;
     g3.offsets = L->offsets;
     g3.E = G;
@@ -419,7 +429,7 @@ int clearmoe_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, const v
     const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
     if (bf16 && r % 16) return CLEARMOE_EUNSUPPORTED;
     if (!bf16 && r % 4) return CLEARMOE_EUNSUPPORTED;
-    return ffn_impl(L, x, T, W1, b1, U_r, S_r, Vh_r, residual_e, router, E, r, opt, out,
+    return ffn_impl(L, x, T, W1, b1, U_r, S_r, Vh_r, nullptr, residual_e, router, E, r, opt, out,
                     static_cast<cudaStream_t>(stream));
 }
 
@@ -433,8 +443,40 @@ int clearmoe_ffn_forward_folded(clearmoe_layer* L, const void* x, int64_t T, con
     for (int e = 0; e < E; ++e)
         if (!W_comb[e] || misaligned(W_comb[e])) return CLEARMOE_EINVAL;
     if (misaligned(W1) || misaligned(b1) || misaligned(out)) return CLEARMOE_EINVAL;
-    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, W_comb, router, E, 0, nullptr, out,
+    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, nullptr, W_comb, router, E, 0, nullptr, out,
                     static_cast<cudaStream_t>(stream));
+}
+
+int clearmoe_ffn_forward_materialized(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                                      const void* W_sh, const void* const* residual_e, const clearmoe_router* router,
+                                      int32_t E, void* out, void* stream) {
+    int rc = check_common(L, x, T);
+    if (rc) return rc;
+    if ((rc = check_router(L, router, E))) return rc;
+    if (!W1 || !b1 || !W_sh || !residual_e || !out) return CLEARMOE_EINVAL;
+    for (int e = 0; e < E; ++e)
+        if (!residual_e[e] || misaligned(residual_e[e])) return CLEARMOE_EINVAL;
+    if (misaligned(W1) || misaligned(b1) || misaligned(W_sh) || misaligned(out)) return CLEARMOE_EINVAL;
+    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, W_sh, residual_e, router, E, 0, nullptr, out,
+                    static_cast<cudaStream_t>(stream));
+}
+
+int clearmoe_materialize_basis(clearmoe_layer* L, const void* U_r, const float* S_r, const void* Vh_r, int32_t r,
+                               void* W_sh, void* stream) {
+    if (!L || !U_r || !S_r || !Vh_r || !W_sh) return CLEARMOE_EINVAL;
+    const int d = L->desc.d, H = L->desc.hidden;
+    if (r < 1 || r > L->desc.max_r || r > d || r > H) return CLEARMOE_EINVAL;
+    cm::FoldArgs f;
+    std::memset(&f, 0, sizeof(f));
+    f.U = U_r;
+    f.S = S_r;
+    f.Vh = Vh_r;
+    f.out[0] = W_sh;  // res[0] == nullptr: W_shared alone
+    f.d = d;
+    f.H = H;
+    f.r = r;
+    f.E = 1;
+    return cuda_fail(cm::launch_fold_basis(f, L->desc.dtype, static_cast<cudaStream_t>(stream)));
 }
 
 int clearmoe_fold_basis(clearmoe_layer* L, const void* U_r, const float* S_r, const void* Vh_r,

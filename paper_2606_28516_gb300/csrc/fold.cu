@@ -5,7 +5,8 @@
 // GEMM over z (the dense FFN's arithmetic) with no basis step. This kernel forms the combined
 // weights once per weight set: each CTA computes a 64 x 64 tile of W_shared = U_r diag(S_r) Vh_r in
 // fp32 (products S_r[k] Vh_r[k][h] in fp32, fma over k ascending), then adds it to the same tile of
-// every expert's residual and rounds once to the layer dtype.
+// every expert's residual (none when res[e] is null: W_shared materialised alone) and rounds once
+// to the layer dtype.
 #include "common.cuh"
 #include "internal.h"
 
@@ -70,7 +71,7 @@ __global__ void __launch_bounds__(256) fold_basis_kernel(const FoldArgs a) {
                 const int col = h0 + tx * 4 + j;
                 if (col >= a.H) continue;
                 const int64_t off = (int64_t)row * a.H + col;
-                const float v = acc[i][j] + load_elem<BF16>(a.res[e], off);
+                const float v = a.res[e] ? acc[i][j] + load_elem<BF16>(a.res[e], off) : acc[i][j];
                 if constexpr (BF16)
                     static_cast<uint16_t*>(a.out[e])[off] = f32_to_bf16(v);
                 else
