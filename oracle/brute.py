@@ -24,6 +24,17 @@ def token_expert(x_t, Wg, bg) -> int:
     return best_e
 
 
+def mlp_token_expert(x_t, W_in, b_in, W_out, b_out, act: str) -> int:
+    """Expert of one token under the MLP router W_out act(W_in x + b_in) + b_out."""
+    h = []
+    for j in range(len(W_in)):
+        u = float(b_in[j])
+        for k in range(len(x_t)):
+            u += float(W_in[j][k]) * float(x_t[k])
+        h.append(max(u, 0.0) if act == "relu" else _gelu(u))
+    return token_expert(h, W_out, b_out)
+
+
 def token_forward(x_t, W1, b1, U, S, Vh, residuals, e: int):
     H, d, r = len(W1), len(x_t), len(S)
     z = []

@@ -43,6 +43,37 @@ def router_logits(x, Wg, bg, precision=np.float64) -> np.ndarray:
     return x @ Wg.T + bg
 
 
+def relu(u) -> np.ndarray:
+    return np.maximum(f64(u), 0.0)
+
+
+ROUTER_ACTS = {"relu": lambda u: relu(u), "gelu": lambda u: gelu(u)}
+
+
+def mlp_hidden(x, W_in, b_in, act: str) -> np.ndarray:
+    """The MLP router's hidden layer act(W_in x + b_in), float64."""
+    return ROUTER_ACTS[act](f64(x) @ f64(W_in).T + f64(b_in))
+
+
+def mlp_router_logits(x, W_in, b_in, W_out, b_out, act: str = "relu", precision=np.float64):
+    """MLP router g(x) = W_out act(W_in x + b_in) + b_out (Phase 4, "MLP": one hidden layer of d/6
+    units; the paper does not name the activation, both ReLU and GELU are offered). With
+    precision float32 the hidden layer is formed in float64, stored in float32, and the output
+    layer is evaluated in float32 (the precision of the decision)."""
+    h = mlp_hidden(x, W_in, b_in, act)
+    h, W_out, b_out = (np.asarray(a, dtype=precision) for a in (h, W_out, b_out))
+    return h @ W_out.T + b_out
+
+
+def route_mlp(x, W_in, b_in, W_out, b_out, act: str = "relu") -> dict:
+    """Algorithm 3 steps 3-4 with the MLP router: the decision on float32 logits, near ties
+    flagged from float64 logits as for the linear router."""
+    E = np.asarray(W_out).shape[0]
+    a = argmax_lowest(mlp_router_logits(x, W_in, b_in, W_out, b_out, act, precision=np.float32))
+    lg = mlp_router_logits(x, W_in, b_in, W_out, b_out, act)
+    return sort_by_expert(a, E) | dict(near_tie=_near_tie_logits(lg))
+
+
 def argmax_lowest(logits) -> np.ndarray:
     """a_t = min{e : logit_{t,e} = max_e logit_{t,e}} (Algorithm 3, "a <- argmax g(x)"; the
     paper leaves ties open, the lowest index wins here)."""
@@ -51,7 +82,10 @@ def argmax_lowest(logits) -> np.ndarray:
 
 def near_ties(x, Wg, bg, rel=NEAR_TIE_REL) -> np.ndarray:
     """Tokens whose top-2 router logits (float64) differ by less than rel * max(|l1|, |l2|)."""
-    lg = router_logits(x, Wg, bg)
+    return _near_tie_logits(router_logits(x, Wg, bg), rel)
+
+
+def _near_tie_logits(lg, rel=NEAR_TIE_REL) -> np.ndarray:
     if lg.shape[1] < 2:
         return np.zeros(lg.shape[0], dtype=bool)
     top = np.sort(lg, axis=1)[:, -2:]

@@ -295,6 +295,37 @@ def make_stack(shape: StackShape = VIT_BASE_STACK12, T: int | None = None) -> di
     return dict(shape=shape, dtype="bf16", x=round_bf16(x), layers=layers, T=T)
 
 
+def mlp_router(layer: dict, hidden: int | None = None, act: str = "relu") -> dict:
+    """Weights of an MLP router d -> hidden -> E (Phase 4 "MLP", hidden = d / 6 by default) built
+    from the layer's linear router, so that it routes the mixture as sensibly without training.
+
+    P (rows) is an orthonormal basis of the span of W_g's rows; hidden units 0..E-1 read P x and
+    units E..2E-1 read -P x, and since act(u) - act(-u) = u for ReLU and for GELU, output weights
+    [W_g P^T, -W_g P^T] reproduce W_g P^T P x = W_g x. The remaining units get random input
+    weights and small random output weights, which perturb the decisions near cluster borders.
+    Values are rounded to the layer dtype like every other weight."""
+    Wg = np.asarray(layer["Wg"], np.float64)
+    bg = np.asarray(layer["bg"], np.float64)
+    E, d = Wg.shape
+    hidden = hidden or d // 6
+    if hidden < 2 * E:
+        raise ValueError("the MLP router needs at least 2 E hidden units")
+    P = np.linalg.qr(Wg.T)[0].T  # E x d, orthonormal rows
+    rng = np.random.default_rng(layer["shape"].seed + 3)
+    W_in = np.zeros((hidden, d))
+    W_in[:E], W_in[E:2 * E] = P, -P
+    W_in[2 * E:] = rng.standard_normal((hidden - 2 * E, d)) / np.sqrt(d)
+    b_in = np.zeros(hidden)
+    b_in[2 * E:] = 0.1 * rng.standard_normal(hidden - 2 * E)
+    G = Wg @ P.T
+    W_out = np.zeros((E, hidden))
+    W_out[:, :E], W_out[:, E:2 * E] = G, -G
+    W_out[:, 2 * E:] = 0.05 * np.abs(G).mean() * rng.standard_normal((E, hidden - 2 * E))
+    dt = layer["dtype"]
+    return dict(W_in=to_dtype(W_in, dt), b_in=to_dtype(b_in, dt), W_out=to_dtype(W_out, dt),
+                b_out=to_dtype(bg, dt), hidden=hidden, act=act)
+
+
 def to_torch(layer: dict, device="cuda") -> dict:
     """Device copies of a layer's arrays in its dtype (bf16 values convert exactly); S_r and
     the integer metadata keep their types."""
@@ -302,7 +333,8 @@ def to_torch(layer: dict, device="cuda") -> dict:
 
     tdt = torch.bfloat16 if layer.get("dtype", "bf16") == "bf16" else torch.float32
     out = {}
-    for k in ("x", "W1", "b1", "W2", "b2", "U", "Vh", "residuals", "Wg", "bg"):
+    for k in ("x", "W1", "b1", "W2", "b2", "U", "Vh", "residuals", "Wg", "bg", "W_in", "b_in", "W_out",
+              "b_out"):
         if k in layer:
             out[k] = torch.from_numpy(np.ascontiguousarray(layer[k], dtype=np.float32)).to(
                 device=device, dtype=tdt).contiguous()

@@ -236,6 +236,54 @@ def test_routing_with_class_tokens_invariants():
     assert np.array_equal(np.sort(rt["perm"]), np.arange(T))
 
 
+# ------------------------------------------------------------------ MLP router
+def check_mlp_identity(seed=12):
+    """W_in = [I; -I], b_in = 0, W_out = [W_g, -W_g], b_out = b_g: since act(u) - act(-u) = u for
+    ReLU and for GELU, the MLP router's logits are the linear router's."""
+    rng = np.random.default_rng(seed)
+    L = rand_layer(rng, 40, 9, 20, 5, 3)
+    d = 9
+    W_in = np.concatenate([np.eye(d), -np.eye(d)])
+    W_out = np.concatenate([L["Wg"], -L["Wg"]], axis=1)
+    want = O.router_logits(L["x"], L["Wg"], L["bg"])
+    return all(rel_err(O.mlp_router_logits(L["x"], W_in, np.zeros(2 * d), W_out, L["bg"], act), want)
+               <= 1e-12 for act in ("relu", "gelu"))
+
+
+def check_mlp_brute(seed=13, T=40, d=12, hidden=6, E=4):
+    """route_mlp against the pure-Python per-token loops, both activations."""
+    rng = np.random.default_rng(seed)
+    x = rng.standard_normal((T, d))
+    W_in, b_in = rng.standard_normal((hidden, d)), rng.standard_normal(hidden)
+    W_out, b_out = rng.standard_normal((E, hidden)), rng.standard_normal(E)
+    ok = True
+    for act in ("relu", "gelu"):
+        rt = O.route_mlp(x, W_in, b_in, W_out, b_out, act)
+        a_b = np.array([B.mlp_token_expert(x[t].tolist(), W_in.tolist(), b_in.tolist(), W_out.tolist(),
+                                           b_out.tolist(), act) for t in range(T)])
+        free = ~rt["near_tie"]
+        ok = ok and np.array_equal(rt["a"][free], a_b[free]) and free.sum() >= T - 2
+    return ok
+
+
+def test_mlp_router_reduces_to_linear():
+    assert check_mlp_identity()
+
+
+def test_mlp_router_brute_force():
+    assert check_mlp_brute()
+    assert check_mlp_brute(seed=14, T=64, d=16, hidden=16, E=7)
+
+
+def test_mlp_router_generator_routes_like_linear():
+    import synth
+    L = synth.make_layer(synth.DEIT_TINY_FP32.with_(T=600, n_cal=2000))
+    M = synth.mlp_router(L)
+    a_lin = O.route(L["x"], L["Wg"], L["bg"])["a"]
+    a_mlp = O.route_mlp(L["x"], M["W_in"], M["b_in"], M["W_out"], M["b_out"])["a"]
+    assert M["hidden"] == 32 and np.mean(a_lin == a_mlp) > 0.9
+
+
 # ------------------------------------------------------------------ brute force
 def check_brute(seed, T=23, d=16, H=64, E=4, r=16):
     rng = np.random.default_rng(seed)
@@ -366,6 +414,9 @@ MUTATIONS = {
         1 / O.f64(S)) @ O.f64(Vh)),
     "fold drops the shared term": ("fold_basis", lambda U, S, Vh, res: np.stack(
         [O.f64(R) for R in res])),
+    "router hidden activation dropped": ("relu", lambda u: O.f64(u)),
+    "router hidden bias dropped": ("mlp_hidden", lambda x, W_in, b_in, act: O.ROUTER_ACTS[act](
+        O.f64(x) @ O.f64(W_in).T)),
     "class tokens routed to experts": ("class_mask", lambda T, s: np.zeros(T, dtype=bool)),
     "fc2 bias added twice": ("fc2_bias", lambda y, b2: O.f64(y) if b2 is None else O.f64(y) + 2 * O.f64(b2)),
     "class token is every token after the first": ("class_mask", lambda T, s: (
@@ -383,7 +434,8 @@ def test_pins_catch_planted_mistakes(name, monkeypatch):
     monkeypatch.setattr(O, attr, fake)
     checks = [check_gelu_table, check_worked_example, check_dense_reduction,
               check_d3_identity, check_scalar_residual, lambda: check_brute(0), check_fold_d3,
-              check_folded_brute, check_cls_all_dense, check_cls_brute, check_cls_keeps_routed_rows]
+              check_folded_brute, check_cls_all_dense, check_cls_brute, check_cls_keeps_routed_rows,
+              check_mlp_identity, check_mlp_brute]
     results = []
     for c in checks:
         try:
