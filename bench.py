@@ -459,7 +459,7 @@ def main():
         v_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in vev)
         return {"value": world * s.T / (v_ms / 1e3), "unit": "tokens/s", "ms_per_step": v_ms, "note": note}
 
-    folded = materialized = class_tokens = None
+    folded = materialized = class_tokens = mlp_router = None
     if s.dtype == "bf16":
         W_comb = torch.empty_like(D["residuals"])
         cm.clearmoe_fold_basis(h, D["U"], D["S"], D["Vh"], D["residuals"], W_comb)
@@ -481,6 +481,12 @@ def main():
                                                D["residuals"], D["Wg"], D["bg"], out, b2=D["b2"], W2=D["W2"],
                                                cls_stride=197),
             "class token of each 197-token image on the dense path (W2), fc2 bias b2 added")
+        M = synth.to_torch(synth.mlp_router(L, act="gelu") | {"dtype": s.dtype})
+        mlp = cm.mlp_router(M["W_in"], M["b_in"], M["W_out"], M["b_out"], "gelu")
+        mlp_router = time_variant(
+            lambda: cm.clearmoe_ffn_forward_ex(h, D["x"], D["W1"], D["b1"], D["U"], D["S"], D["Vh"],
+                                               D["residuals"], None, None, out, mlp=mlp, E=s.E),
+            f"MLP router d -> {s.d // 6} -> E (GELU) in place of the linear router")
 
     # same-GPU dense FFN, same timing rules (events around each forward only)
     dout = torch.empty_like(out)
@@ -618,6 +624,7 @@ def main():
         "folded": folded,
         "materialized": materialized,
         "class_tokens": class_tokens,
+        "mlp_router": mlp_router,
         "wall_s_timed": wall,
     }
     if rank == 0:

@@ -68,6 +68,23 @@ typedef struct {
     const void* b;
 } clearmoe_router;
 
+/* MLP router (Phase 4, "MLP": one hidden layer of d/6 units; the paper does not name its
+ * activation, so both are offered): logits = W_out act(W_in x + b_in) + b_out with W_in
+ * [hidden x d], b_in [hidden], W_out [E x hidden], b_out [E], device pointers in the layer's dtype.
+ * The hidden layer runs on the tensor-core GEMM (fp32 on the fp32 layer) and is kept in fp32; the
+ * output layer and the argmax run in fp32 on the routing kernel, so the decision is taken on fp32
+ * logits as for the linear router. hidden: a multiple of 16 (bf16) or 4 (fp32), at most H / 2
+ * (bf16) or H (fp32): the hidden layer lives in the hidden-state workspace before fc1 runs. */
+typedef enum { CLEARMOE_ACT_RELU = 0, CLEARMOE_ACT_GELU = 1 } clearmoe_act;
+typedef struct {
+    const void* W_in;
+    const void* b_in;
+    const void* W_out;
+    const void* b_out;
+    int32_t hidden;
+    int32_t act; /* clearmoe_act */
+} clearmoe_mlp_router;
+
 typedef struct clearmoe_layer clearmoe_layer;
 
 /* Allocates the handle and its device workspace on the current device (hidden states
@@ -88,6 +105,13 @@ int clearmoe_layer_destroy(clearmoe_layer* layer);
  * 1 <= T <= max_tokens, 1 <= E <= max_E. */
 int clearmoe_route(clearmoe_layer* layer, const void* x, int64_t T, const clearmoe_router* router,
                    int32_t E, void* stream);
+
+/* Routing only with the MLP router: its hidden layer (one GEMM launch), then the routing kernel on
+ * the fp32 hidden layer with W_out, b_out as the router, then the slot kernel. Same outputs and
+ * errors as clearmoe_route; EINVAL for a NULL or misaligned weight, an unknown act or a hidden
+ * width outside the limits above. */
+int clearmoe_route_mlp(clearmoe_layer* layer, const void* x, int64_t T, const clearmoe_mlp_router* mlp,
+                       int32_t E, void* stream);
 
 /* The CLEAR-MoE FFN forward (Eq. 2 with Algorithm 3): routes (as clearmoe_route), computes
  * z = GELU(W1 x + b1) for every token in expert-sorted order (fc1 reads x in token order and its
@@ -112,11 +136,13 @@ int clearmoe_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const 
  *              class token out of expert dispatch. The class tokens form group E after the experts:
  *              idx = E, counts[E] = n_cls = ceil(T / cls_stride), slots [T - n_cls, T) in token
  *              order. Requires W2 and E + 1 <= 16 (EUNSUPPORTED otherwise). 0: every token routed.
- *  W2          the layer's dense fc2 [d x H] row-major (device), read for class tokens only. */
+ *  W2          the layer's dense fc2 [d x H] row-major (device), read for class tokens only.
+ *  mlp_router  the MLP router in place of the linear one (see clearmoe_mlp_router). */
 typedef struct {
     const void* b2;
     int64_t cls_stride;
     const void* W2;
+    const clearmoe_mlp_router* mlp_router; /* non-NULL: routes with it (router may then be NULL) */
 } clearmoe_ffn_options;
 
 /* clearmoe_ffn_forward with deployment options (opt may be NULL: then identical to it). With

@@ -32,8 +32,23 @@ class clearmoe_router(ctypes.Structure):
     _fields_ = [("W", ctypes.c_void_p), ("b", ctypes.c_void_p)]
 
 
+class clearmoe_mlp_router(ctypes.Structure):
+    _fields_ = [("W_in", ctypes.c_void_p), ("b_in", ctypes.c_void_p), ("W_out", ctypes.c_void_p),
+                ("b_out", ctypes.c_void_p), ("hidden", ctypes.c_int32), ("act", ctypes.c_int32)]
+
+
 class clearmoe_ffn_options(ctypes.Structure):
-    _fields_ = [("b2", ctypes.c_void_p), ("cls_stride", ctypes.c_int64), ("W2", ctypes.c_void_p)]
+    _fields_ = [("b2", ctypes.c_void_p), ("cls_stride", ctypes.c_int64), ("W2", ctypes.c_void_p),
+                ("mlp_router", ctypes.POINTER(clearmoe_mlp_router))]
+
+
+ACT_RELU, ACT_GELU = 0, 1
+
+
+def mlp_router(W_in, b_in, W_out, b_out, act: str = "relu") -> clearmoe_mlp_router:
+    """The MLP router's weights as the C struct (act: "relu" or "gelu")."""
+    return clearmoe_mlp_router(_ptr(W_in), _ptr(b_in), _ptr(W_out), _ptr(b_out), W_in.shape[0],
+                               {"relu": ACT_RELU, "gelu": ACT_GELU}[act])
 
 
 _P, _I64, _I32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
@@ -41,6 +56,7 @@ _SIGS = {
     "clearmoe_layer_create": [ctypes.POINTER(clearmoe_layer_desc), ctypes.POINTER(ctypes.c_void_p)],
     "clearmoe_layer_destroy": [_P],
     "clearmoe_route": [_P, _P, _I64, ctypes.POINTER(clearmoe_router), _I32, _P],
+    "clearmoe_route_mlp": [_P, _P, _I64, ctypes.POINTER(clearmoe_mlp_router), _I32, _P],
     "clearmoe_ffn_forward": [_P, _P, _I64, _P, _P, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
                              ctypes.POINTER(clearmoe_router), _I32, _I32, _P, _P],
     "clearmoe_ffn_forward_ex": [_P, _P, _I64, _P, _P, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
@@ -135,6 +151,11 @@ def clearmoe_route(layer: int, x, Wg, bg, stream=None) -> None:
                                 _stream(stream)), "clearmoe_route")
 
 
+def clearmoe_route_mlp(layer: int, x, mlp: clearmoe_mlp_router, E: int, stream=None) -> None:
+    _check(lib().clearmoe_route_mlp(layer, _ptr(x), x.shape[0], ctypes.byref(mlp), E, _stream(stream)),
+           "clearmoe_route_mlp")
+
+
 def clearmoe_ffn_forward(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, bg, out,
                          stream=None) -> None:
     """residual_e: a sequence of E [d x H] tensors, or one [E x d x H] tensor."""
@@ -148,15 +169,17 @@ def clearmoe_ffn_forward(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, 
 
 
 def clearmoe_ffn_forward_ex(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, bg, out,
-                            b2=None, W2=None, cls_stride: int = 0, stream=None) -> None:
-    """clearmoe_ffn_forward with fc2's bias b2 and class tokens (every cls_stride-th token from
-    token 0) on the dense path W2."""
-    E = Wg.shape[0]
+                            b2=None, W2=None, cls_stride: int = 0, mlp: clearmoe_mlp_router | None = None,
+                            E: int | None = None, stream=None) -> None:
+    """clearmoe_ffn_forward with fc2's bias b2, class tokens (every cls_stride-th token from token 0)
+    on the dense path W2, and the MLP router `mlp` (then Wg, bg may be None and E is given)."""
+    E = Wg.shape[0] if E is None else E
     res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
-    r = _router(Wg, bg)
-    opt = clearmoe_ffn_options(_ptr(b2), int(cls_stride), _ptr(W2))
+    r = _router(Wg, bg) if Wg is not None else None
+    opt = clearmoe_ffn_options(_ptr(b2), int(cls_stride), _ptr(W2),
+                               ctypes.pointer(mlp) if mlp is not None else None)
     _check(lib().clearmoe_ffn_forward_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), _ptr(U_r),
-                                         _ptr(S_r), _ptr(Vh_r), res, ctypes.byref(r), E,
+                                         _ptr(S_r), _ptr(Vh_r), res, ctypes.byref(r) if r else None, E,
                                          S_r.shape[0], ctypes.byref(opt), _ptr(out),
                                          _stream(stream)), "clearmoe_ffn_forward_ex")
 

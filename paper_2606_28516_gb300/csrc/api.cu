@@ -59,21 +59,82 @@ int check_common(const clearmoe_layer* L, const void* x, int64_t T) {
     return CLEARMOE_OK;
 }
 
-int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router, int E,
-             int64_t cls_stride, cudaStream_t s) {
+// The MLP router's hidden layer h = act(W_in x + b_in) [T x hidden], fp32, into the hidden-state
+// workspace (free until fc1 runs): the tensor-core GEMM with an fp32-store epilogue, or the fp32
+// SIMT GEMM on the fp32 layer.
+int mlp_hidden(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_mlp_router* m, cudaStream_t s) {
+    const int d = L->desc.d, nh = m->hidden;
+    if (L->desc.dtype == CLEARMOE_F32) {
+        cm::SimtGemmArgs g;
+        std::memset(&g, 0, sizeof(g));
+        g.A0 = static_cast<const float*>(x);
+        g.lda0 = d;
+        g.K0 = d;
+        g.B0 = static_cast<const float*>(m->W_in);
+        g.M = T;
+        g.N = nh;
+        g.bias = static_cast<const float*>(m->b_in);
+        g.gelu = m->act == CLEARMOE_ACT_GELU;
+        g.relu = m->act == CLEARMOE_ACT_RELU;
+        g.C = static_cast<float*>(L->z);
+        g.ldc = nh;
+        return cuda_fail(cm::launch_simt_gemm(g, s));
+    }
+    cm::TcGemmArgs g;
+    std::memset(&g, 0, sizeof(g));
+    g.status = L->status;
+    g.wait_limit_ns = L->wait_limit_ns;
+    const int p = nh <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, nh) : 0;
+    const int bn = cm::tc_pick_bn(cm::TC_DENSE, nh);
+    if (!p && !bn) return CLEARMOE_EUNSUPPORTED;
+    if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, m->W_in, nh, d, p ? p / 2 : bn))
+        return CLEARMOE_ECUDA;
+    g.mode = cm::TC_DENSE;
+    g.epi = m->act == CLEARMOE_ACT_GELU ? cm::TC_EPI_BIAS_GELU : cm::TC_EPI_BIAS_RELU;
+    g.M = T;
+    g.N = nh;
+    g.K0 = d;
+    g.bias = m->b_in;
+    g.C = L->z;
+    g.ldc = nh;
+    g.c_f32 = 1;
+    return cuda_fail(p ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s));
+}
+
+int check_mlp(const clearmoe_layer* L, const clearmoe_mlp_router* m, int E) {
+    if (!m || !m->W_in || !m->b_in || !m->W_out || !m->b_out) return CLEARMOE_EINVAL;
+    if (misaligned(m->W_in) || misaligned(m->b_in) || misaligned(m->W_out)) return CLEARMOE_EINVAL;
+    if (m->act != CLEARMOE_ACT_RELU && m->act != CLEARMOE_ACT_GELU) return CLEARMOE_EINVAL;
+    if (E < 1 || E > L->desc.max_E) return CLEARMOE_EINVAL;
+    const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
+    if (m->hidden < 1 || m->hidden % (bf16 ? 16 : 4)) return CLEARMOE_EINVAL;
+    if ((int64_t)m->hidden * 4 > (int64_t)L->esz * L->desc.hidden) return CLEARMOE_EINVAL;  // fits in z
+    return CLEARMOE_OK;
+}
+
+int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router,
+             const clearmoe_mlp_router* mlp, int E, int64_t cls_stride, cudaStream_t s) {
+    // the MLP router: its hidden layer first, then the routing kernel on it (fp32 tokens)
+    const int rd = mlp ? mlp->hidden : L->desc.d;
+    const int rdtype = mlp ? CLEARMOE_F32 : L->desc.dtype;
     int grid = 0, chunk = 0;
-    const int g = cm::route_grid(T, L->desc.d, E, L->desc.dtype, L->num_sms, &grid, &chunk);
+    const int g = cm::route_grid(T, rd, E, rdtype, L->num_sms, &grid, &chunk);
     if (g) return g == -2 ? CLEARMOE_EUNSUPPORTED : CLEARMOE_ECUDA;
-    if (grid > cm::route_max_ctas(L->num_sms, L->desc.dtype, L->desc.d, E)) return CLEARMOE_EUNSUPPORTED;
+    if (grid > cm::route_max_ctas(L->num_sms, rdtype, rd, E)) return CLEARMOE_EUNSUPPORTED;
+    if (mlp) {
+        const int rc = mlp_hidden(L, x, T, mlp, s);
+        if (rc) return rc;
+    }
     cm::RouteArgs& a = L->rt;
     std::memset(&a, 0, sizeof(a));
-    a.x = x;
+    a.x = mlp ? L->z : x;
     a.T = T;
-    a.d = L->desc.d;
+    a.d = rd;
     a.E = E;
-    a.dtype = L->desc.dtype;
-    a.Wg = router->W;
-    a.bg = router->b;
+    a.dtype = rdtype;
+    a.Wg = mlp ? mlp->W_out : router->W;
+    a.bg = mlp ? mlp->b_out : router->b;
+    a.w_bf16 = mlp && L->desc.dtype == CLEARMOE_BF16;
     a.idx = L->idx;
     a.perm = L->perm;
     a.inv = L->inv;
@@ -198,7 +259,17 @@ int clearmoe_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_r
     if (rc) return rc;
     if ((rc = check_router(L, router, E))) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if ((rc = do_route(L, x, T, router, E, 0, s))) return rc;
+    if ((rc = do_route(L, x, T, router, nullptr, E, 0, s))) return rc;
+    return do_finalize(L, s);
+}
+
+int clearmoe_route_mlp(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_mlp_router* mlp, int32_t E,
+                       void* stream) {
+    int rc = check_common(L, x, T);
+    if (rc) return rc;
+    if ((rc = check_mlp(L, mlp, E))) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((rc = do_route(L, x, T, nullptr, mlp, E, 0, s))) return rc;
     return do_finalize(L, s);
 }
 
@@ -220,7 +291,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     const void* b2 = opt ? opt->b2 : nullptr;
     int rc;
     mark(L, 0, s);
-    if ((rc = do_route(L, x, T, router, E, cls_stride, s))) return rc;
+    if ((rc = do_route(L, x, T, router, opt ? opt->mlp_router : nullptr, E, cls_stride, s))) return rc;
     // bf16 with the 2-SM fc1: the fc1 epilogue assigns the slots itself (no finalize launch)
     const int p1 = bf16 && H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;
     const bool fused = p1 && L->rt_grid <= 256 && L->rt_grid * E <= cm::TC2_TAB_CAP;
@@ -409,7 +480,11 @@ int clearmoe_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, const v
                             void* out, void* stream) {
     int rc = check_common(L, x, T);
     if (rc) return rc;
-    if ((rc = check_router(L, router, E))) return rc;
+    if (opt && opt->mlp_router)
+        rc = check_mlp(L, opt->mlp_router, E);
+    else
+        rc = check_router(L, router, E);
+    if (rc) return rc;
     if (opt) {
         if (opt->cls_stride < 0 || opt->cls_stride > ((int64_t)1 << 30)) return CLEARMOE_EINVAL;
         if (opt->b2 && misaligned(opt->b2)) return CLEARMOE_EINVAL;

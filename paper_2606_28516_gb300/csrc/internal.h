@@ -28,6 +28,7 @@ struct RouteArgs {
     // > 0: token t with t % cls_stride == 0 is a class token: it skips the router and forms group
     // E (idx = E), the dense path, whose slots follow every expert's: T - n_cls + t / cls_stride
     int64_t cls_stride;
+    int w_bf16;  // fp32 tokens (the MLP router's hidden layer) with bf16 W_g and b_g
 };
 // Class tokens of T: every cls_stride-th from token 0 (none when cls_stride is 0).
 __host__ __device__ inline int64_t n_class_tokens(int64_t T, int64_t cls_stride) {
@@ -71,6 +72,7 @@ struct SimtGemmArgs {
     int N;
     const float* bias;   // + bias[n]
     int gelu;            // GELU after bias
+    int relu;            // max(., 0) after bias
     const float* scale;  // * scale[n]
     float* C;
     int64_t ldc;
@@ -84,7 +86,7 @@ cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s);
 cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s);
 
 // ---- tcgen05 bf16 GEMMs ----
-enum TcEpi { TC_EPI_BIAS_GELU = 0, TC_EPI_SCALE = 1, TC_EPI_STORE = 2, TC_EPI_SCATTER = 3 };
+enum TcEpi { TC_EPI_BIAS_GELU = 0, TC_EPI_SCALE = 1, TC_EPI_STORE = 2, TC_EPI_SCATTER = 3, TC_EPI_BIAS_RELU = 4 };
 enum TcMode { TC_DENSE = 0, TC_GATHER = 1, TC_GROUPED = 2 };
 
 struct TcGemmArgs {
@@ -126,6 +128,8 @@ struct TcGemmArgs {
     int dense_last;
     // fused fc1: class tokens (t % rt_cls_stride == 0) go to slot M - n_cls + t / rt_cls_stride
     int64_t rt_cls_stride;
+    // C is fp32 (stored as computed, no rounding): the MLP router's hidden layer
+    int c_f32;
     // 2-SM kernel: A tiles loaded with the L2 evict-first policy (a stream read once), so that they
     // displace one another rather than lines the next reads are still to find in L2
     int a_evict_first;

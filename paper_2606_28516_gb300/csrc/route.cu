@@ -330,11 +330,18 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         }
     } else {
         float* Wf = reinterpret_cast<float*>(smem);
-        const float* W = static_cast<const float*>(a.Wg);
-        for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = W[i];
+        if (a.w_bf16) {  // bf16 router weights on fp32 tokens: widened exactly
+            const uint16_t* W = static_cast<const uint16_t*>(a.Wg);
+            for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = bf16_to_f32(W[i]);
+        } else {
+            const float* W = static_cast<const float*>(a.Wg);
+            for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = W[i];
+        }
         pdl_wait();
         __syncthreads();
-        const float* bgp = static_cast<const float*>(a.bg);
+        auto bias_of = [&](int e) -> float {
+            return a.w_bf16 ? bf16_to_f32(static_cast<const uint16_t*>(a.bg)[e]) : static_cast<const float*>(a.bg)[e];
+        };
         const float* X = static_cast<const float*>(a.x);
         for (int i = warp; i < nrows; i += NWARPS) {
             const float* xr = X + (row0 + i) * d;
@@ -355,7 +362,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                     float v = acc[e];
 #pragma unroll
                     for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-                    arg_better(bv, be, v + bgp[e], e);
+                    arg_better(bv, be, v + bias_of(e), e);
                 }
             }
             if (be > E - 1) be = 0;

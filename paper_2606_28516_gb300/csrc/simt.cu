@@ -105,6 +105,7 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
             float v = acc[i][j];
             if (a.bias) v += a.bias[n];
             if (a.gelu) v = gelu_erf(v);
+            if (a.relu) v = fmaxf(v, 0.f);
             if (a.scale) v *= a.scale[n];
             a.C[orow * a.ldc + n] = v;
         }

@@ -324,6 +324,18 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
                             f[j8 * 8 + 2 * h + 1] = g.y;
                         }
                     }
+                } else if (a.epi == TC_EPI_BIAS_RELU) {
+                    const uint4* bp = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.bias) + nb);
+#pragma unroll
+                    for (int j8 = 0; j8 < C::CW / 8; ++j8) {
+                        const uint4 b = __ldg(bp + j8);
+                        const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+                        for (int h = 0; h < 4; ++h) {
+                            f[j8 * 8 + 2 * h] = fmaxf(f[j8 * 8 + 2 * h] + bf16_lo(bw[h]), 0.f);
+                            f[j8 * 8 + 2 * h + 1] = fmaxf(f[j8 * 8 + 2 * h + 1] + bf16_hi(bw[h]), 0.f);
+                        }
+                    }
                 } else if (a.out_bias) {
                     const uint4* bp = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.out_bias) + nb);
 #pragma unroll
@@ -345,6 +357,15 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
                         f[4 * j4 + 2] *= s4.z;
                         f[4 * j4 + 3] *= s4.w;
                     }
+                }
+                if (a.c_f32) {  // fp32 output: each lane stores its row's values as computed
+                    if (orow >= 0) {
+                        float4* dstf = reinterpret_cast<float4*>(static_cast<float*>(a.C) + orow * a.ldc + nb);
+#pragma unroll
+                        for (int j4 = 0; j4 < C::CW / 4; ++j4)
+                            dstf[j4] = make_float4(f[4 * j4], f[4 * j4 + 1], f[4 * j4 + 2], f[4 * j4 + 3]);
+                    }
+                    continue;
                 }
                 uint4* dst = reinterpret_cast<uint4*>(wstg + lane * C::STG_ROW);
 #pragma unroll

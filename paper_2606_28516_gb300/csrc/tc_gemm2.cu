@@ -182,7 +182,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         mbar_fence_init();
     }
     // The bias or the column scale (weights, not produced by the previous kernel) as fp32, once per CTA.
-    if (MODE == TC_DENSE && a.epi == TC_EPI_BIAS_GELU && warp < NUM_EPI) {
+    if (MODE == TC_DENSE && (a.epi == TC_EPI_BIAS_GELU || a.epi == TC_EPI_BIAS_RELU) && warp < NUM_EPI) {
         const uint16_t* b = static_cast<const uint16_t*>(a.bias);
         for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = __uint_as_float((uint32_t)b[n] << 16);
     } else if (MODE == TC_DENSE && a.epi == TC_EPI_SCALE && warp < NUM_EPI) {
@@ -474,6 +474,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                         f[4 * j4 + 2] = g1.x;
                         f[4 * j4 + 3] = g1.y;
                     }
+                } else if (a.epi == TC_EPI_BIAS_RELU) {
+                    const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
+#pragma unroll
+                    for (int j4 = 0; j4 < CW / 4; ++j4) {
+                        const float4 b = bp[j4];
+                        f[4 * j4] = fmaxf(f[4 * j4] + b.x, 0.f);
+                        f[4 * j4 + 1] = fmaxf(f[4 * j4 + 1] + b.y, 0.f);
+                        f[4 * j4 + 2] = fmaxf(f[4 * j4 + 2] + b.z, 0.f);
+                        f[4 * j4 + 3] = fmaxf(f[4 * j4 + 3] + b.w, 0.f);
+                    }
                 } else if (a.out_bias) {
                     const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
 #pragma unroll
@@ -498,6 +508,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                         f[4 * j4 + 2] = p1.x;
                         f[4 * j4 + 3] = p1.y;
                     }
+                }
+                if (a.c_f32) {  // fp32 output: each lane stores its row's 32 values as computed
+                    if (orow >= 0) {
+                        float4* dstf = reinterpret_cast<float4*>(static_cast<float*>(a.C) + orow * a.ldc + nb);
+#pragma unroll
+                        for (int j4 = 0; j4 < CW / 4; ++j4)
+                            dstf[j4] = make_float4(f[4 * j4], f[4 * j4 + 1], f[4 * j4 + 2], f[4 * j4 + 3]);
+                    }
+                    continue;
                 }
 #pragma unroll
                 for (int s0 = 0; s0 < CW; s0 += SW) {
@@ -579,7 +598,8 @@ static cudaError_t launch2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
 
 cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     const int bn = tc2_pick_bn(a.mode, a.N);
-    const bool staged = a.epi == TC_EPI_BIAS_GELU || a.epi == TC_EPI_SCALE;  // fp32 vector in shared memory
+    const bool staged = a.epi == TC_EPI_BIAS_GELU || a.epi == TC_EPI_BIAS_RELU ||
+                        a.epi == TC_EPI_SCALE;  // fp32 vector in shared memory
     if (!bn || (staged && (a.mode != TC_DENSE || a.N > TC2_BIAS_CAP))) return cudaErrorInvalidValue;
     if (a.out_bias && (staged || a.N > TC2_BIAS_CAP)) return cudaErrorInvalidValue;
     return bn == 256 ? launch2<256>(a, num_sms, s) : launch2<128>(a, num_sms, s);
