@@ -161,6 +161,16 @@ def ffn_forward(x, W1, b1, U, S, Vh, residuals, Wg=None, bg=None, a=None,
     return experts_forward(z, shared_weight(U, S, Vh), residuals, a)
 
 
+def ffn_forward_scaled(x, W1, b1, U, S, Vh, R, s, Wg=None, bg=None, a=None,
+                       z_bf16: bool = False) -> np.ndarray:
+    """Eq. 2 with the residual structure of Algorithm 2, W_e^res = s_e (W2 - W_shared) = s_e R:
+    y_t = W_shared z_t + s_{a_t} R z_t (one residual matrix and a scalar per expert)."""
+    if a is None:
+        a = route(x, Wg, bg)["a"]
+    z = fc1_gelu(x, W1, b1, z_bf16)
+    return z @ shared_weight(U, S, Vh).T + f64(s)[np.asarray(a)][:, None] * (z @ f64(R).T)
+
+
 def fold_basis(U, S, Vh, residuals) -> np.ndarray:
     """W_e^comb = W_shared + W_e^res for every expert e: Eq. 2 regrouped, since both terms act
     on the same hidden state, y = W_shared z + W_a^res z = (W_shared + W_a^res) z."""

@@ -254,7 +254,7 @@ def make_layer(shape: LayerShape) -> dict:
     # fc2's bias (a pretrained ViT layer has one; Eq. 2 is printed without it), from its own stream
     b2 = to_dtype(WEIGHT_STD * np.random.default_rng(shape.seed + 2).standard_normal(shape.d), dt)
     return dict(
-        shape=shape, dtype=dt, x=x, W1=W1, b1=b1, W2=W2, b2=b2,
+        shape=shape, dtype=dt, x=x, W1=W1, b1=b1, W2=W2, b2=b2, R=to_dtype(conv["D"], dt),
         U=to_dtype(conv["U"], dt), S=conv["S"].astype(np.float32), Vh=to_dtype(conv["Vh"], dt),
         residuals=res, Wg=to_dtype(conv["Wg"], dt), bg=to_dtype(conv["bg"], dt),
         scales=conv["scales"], labels=labels, sigma_all=conv["sigma_all"],
@@ -333,11 +333,12 @@ def to_torch(layer: dict, device="cuda") -> dict:
 
     tdt = torch.bfloat16 if layer.get("dtype", "bf16") == "bf16" else torch.float32
     out = {}
-    for k in ("x", "W1", "b1", "W2", "b2", "U", "Vh", "residuals", "Wg", "bg", "W_in", "b_in", "W_out",
+    for k in ("x", "W1", "b1", "W2", "b2", "R", "U", "Vh", "residuals", "Wg", "bg", "W_in", "b_in", "W_out",
               "b_out"):
         if k in layer:
             out[k] = torch.from_numpy(np.ascontiguousarray(layer[k], dtype=np.float32)).to(
                 device=device, dtype=tdt).contiguous()
-    if "S" in layer:
-        out["S"] = torch.from_numpy(np.ascontiguousarray(layer["S"], dtype=np.float32)).to(device)
+    for k in ("S", "scales"):  # fp32 in every layer dtype
+        if k in layer:
+            out[k] = torch.from_numpy(np.ascontiguousarray(layer[k], dtype=np.float32)).to(device)
     return out

@@ -284,6 +284,26 @@ def test_mlp_router_generator_routes_like_linear():
     assert M["hidden"] == 32 and np.mean(a_lin == a_mlp) > 0.9
 
 
+# ------------------------------------------------------------------ scalar residuals (Algorithm 2)
+def check_scaled_brute(seed=15, T=21, d=12, H=48, E=3, r=5):
+    """W_e^res = s_e R: the one-matrix form against the brute force on the E scaled copies."""
+    rng = np.random.default_rng(seed)
+    L = rand_layer(rng, T, d, H, E, r)
+    R = rng.standard_normal((d, H)) / np.sqrt(H)
+    s = rng.uniform(0.3, 1.7, E)
+    res = [s[e] * R for e in range(E)]
+    a_b, y_b = B.layer(L["x"].tolist(), L["W1"].tolist(), L["b1"].tolist(), L["U"].tolist(),
+                       L["S"].tolist(), L["Vh"].tolist(), [m.tolist() for m in res],
+                       L["Wg"].tolist(), L["bg"].tolist())
+    y = O.ffn_forward_scaled(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], R, s, a=np.array(a_b))
+    return rel_err(y, np.array(y_b)) <= 1e-12
+
+
+def test_scaled_residual_form_brute_force():
+    assert check_scaled_brute()
+    assert check_scaled_brute(seed=16, T=8, E=1)
+
+
 # ------------------------------------------------------------------ brute force
 def check_brute(seed, T=23, d=16, H=64, E=4, r=16):
     rng = np.random.default_rng(seed)
@@ -414,6 +434,8 @@ MUTATIONS = {
         1 / O.f64(S)) @ O.f64(Vh)),
     "fold drops the shared term": ("fold_basis", lambda U, S, Vh, res: np.stack(
         [O.f64(R) for R in res])),
+    "scale on the shared term too": ("ffn_forward_scaled", lambda x, W1, b1, U, S, Vh, R, s, a=None, **k: (
+        O.f64(s)[np.asarray(a)][:, None] * (O.fc1_gelu(x, W1, b1) @ (O.shared_weight(U, S, Vh) + O.f64(R)).T))),
     "router hidden activation dropped": ("relu", lambda u: O.f64(u)),
     "router hidden bias dropped": ("mlp_hidden", lambda x, W_in, b_in, act: O.ROUTER_ACTS[act](
         O.f64(x) @ O.f64(W_in).T)),
@@ -435,7 +457,7 @@ def test_pins_catch_planted_mistakes(name, monkeypatch):
     checks = [check_gelu_table, check_worked_example, check_dense_reduction,
               check_d3_identity, check_scalar_residual, lambda: check_brute(0), check_fold_d3,
               check_folded_brute, check_cls_all_dense, check_cls_brute, check_cls_keeps_routed_rows,
-              check_mlp_identity, check_mlp_brute]
+              check_mlp_identity, check_mlp_brute, check_scaled_brute]
     results = []
     for c in checks:
         try:
