@@ -459,7 +459,7 @@ def main():
         v_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in vev)
         return {"value": world * s.T / (v_ms / 1e3), "unit": "tokens/s", "ms_per_step": v_ms, "note": note}
 
-    folded = materialized = class_tokens = mlp_router = None
+    folded = materialized = class_tokens = mlp_router = scaled = None
     if s.dtype == "bf16":
         W_comb = torch.empty_like(D["residuals"])
         cm.clearmoe_fold_basis(h, D["U"], D["S"], D["Vh"], D["residuals"], W_comb)
@@ -481,6 +481,10 @@ def main():
                                                D["residuals"], D["Wg"], D["bg"], out, b2=D["b2"], W2=D["W2"],
                                                cls_stride=197),
             "class token of each 197-token image on the dense path (W2), fc2 bias b2 added")
+        scaled = time_variant(
+            lambda: cm.clearmoe_ffn_forward_scaled(h, D["x"], D["W1"], D["b1"], D["U"], D["S"], D["Vh"], D["R"],
+                                                   D["scales"], D["Wg"], D["bg"], out),
+            "Algorithm 2's residuals as s_e R: one residual matrix, token order, no sort or scatter")
         M = synth.to_torch(synth.mlp_router(L, act="gelu") | {"dtype": s.dtype})
         mlp = cm.mlp_router(M["W_in"], M["b_in"], M["W_out"], M["b_out"], "gelu")
         mlp_router = time_variant(
@@ -625,6 +629,7 @@ def main():
         "materialized": materialized,
         "class_tokens": class_tokens,
         "mlp_router": mlp_router,
+        "scaled_residual": scaled,
         "wall_s_timed": wall,
     }
     if rank == 0:

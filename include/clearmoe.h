@@ -188,6 +188,21 @@ int clearmoe_ffn_forward_materialized(clearmoe_layer* layer, const void* x, int6
                                       const void* b1, const void* W_sh, const void* const* residual_e,
                                       const clearmoe_router* router, int32_t E, void* out, void* stream);
 
+/* The residual structure of Algorithm 2 exploited: its residual experts are scaled copies of one
+ * matrix, W_e^res = s_e R with R = W2 - W_shared, so y_t = W_shared z_t + s_{a_t} R z_t =
+ * s_{a_t} (U_r t'_t + R z_t) with t'_t = diag(S_r) Vh_r z_t / s_{a_t}. Routing (idx), fc1, the
+ * basis factor (column scale S_r and row scale 1 / s_a) and one GEMM with the K chain
+ * [z | t'] x [R | U_r] and row scale s_a, all in token order: no sort, no scatter, one residual
+ * matrix instead of E. Exact (up to rounding) only for residuals of that form; s_e [E] fp32
+ * device, every s_e finite and non-zero (Algorithm 2's are ratios of mean norms, positive), else
+ * the rows of that expert are not finite. R [d x H] row-major in the layer dtype. counts, offsets
+ * and perm are still produced (after the output) for clearmoe_get_routing. Errors as
+ * clearmoe_ffn_forward. */
+int clearmoe_ffn_forward_scaled(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                                const void* b1, const void* U_r, const float* S_r, const void* Vh_r,
+                                const void* R, const float* s_e, const clearmoe_router* router,
+                                int32_t E, int32_t r, void* out, void* stream);
+
 /* The dense FFN the layer was converted from, on the same device: out = W2 GELU(W1 x + b1)
  * (the comparison path; no bias on fc2, as in Eq. 2). 1 <= T <= max_tokens. */
 int clearmoe_dense_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,

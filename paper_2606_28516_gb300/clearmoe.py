@@ -65,6 +65,8 @@ _SIGS = {
     "clearmoe_materialize_basis": [_P, _P, _P, _P, _I32, _P, _P],
     "clearmoe_ffn_forward_materialized": [_P, _P, _I64, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
                                           ctypes.POINTER(clearmoe_router), _I32, _P, _P],
+    "clearmoe_ffn_forward_scaled": [_P, _P, _I64, _P, _P, _P, _P, _P, _P, _P,
+                                    ctypes.POINTER(clearmoe_router), _I32, _I32, _P, _P],
     "clearmoe_dense_ffn_forward": [_P, _P, _I64, _P, _P, _P, _P, _P],
     "clearmoe_dense_ffn_forward_ex": [_P, _P, _I64, _P, _P, _P, _P, _P, _P],
     "clearmoe_layer_norm": [_P, _P, _I64, _P, _P],
@@ -215,6 +217,15 @@ def clearmoe_ffn_forward_materialized(layer: int, x, W1, b1, W_sh, residual_e, W
     _check(lib().clearmoe_ffn_forward_materialized(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
                                                    _ptr(W_sh), res, ctypes.byref(r), E, _ptr(out),
                                                    _stream(stream)), "clearmoe_ffn_forward_materialized")
+
+
+def clearmoe_ffn_forward_scaled(layer: int, x, W1, b1, U_r, S_r, Vh_r, R, s_e, Wg, bg, out,
+                                stream=None) -> None:
+    r = _router(Wg, bg)
+    _check(lib().clearmoe_ffn_forward_scaled(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), _ptr(U_r),
+                                             _ptr(S_r), _ptr(Vh_r), _ptr(R), _ptr(s_e), ctypes.byref(r),
+                                             Wg.shape[0], S_r.shape[0], _ptr(out), _stream(stream)),
+           "clearmoe_ffn_forward_scaled")
 
 
 def clearmoe_dense_ffn_forward(layer: int, x, W1, b1, W2, out, stream=None) -> None:

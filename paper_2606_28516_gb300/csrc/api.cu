@@ -536,6 +536,148 @@ int clearmoe_ffn_forward_materialized(clearmoe_layer* L, const void* x, int64_t 
                     static_cast<cudaStream_t>(stream));
 }
 
+// Algorithm 2's residuals are scaled copies of one matrix, W_e^res = s_e R with R = W2 - W_shared,
+// so y = W_shared z + s_a R z = s_a (U_r t' + R z) with t' = diag(S_r) Vh_r z / s_a: every GEMM
+// runs in token order (no sort, no scatter) and the router's choice enters as a row scale only.
+int clearmoe_ffn_forward_scaled(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                                const void* U_r, const float* S_r, const void* Vh_r, const void* R,
+                                const float* s_e, const clearmoe_router* router, int32_t E, int32_t r, void* out,
+                                void* stream) {
+    int rc = check_common(L, x, T);
+    if (rc) return rc;
+    if ((rc = check_router(L, router, E))) return rc;
+    if (!W1 || !b1 || !U_r || !S_r || !Vh_r || !R || !s_e || !out) return CLEARMOE_EINVAL;
+    const int d = L->desc.d, H = L->desc.hidden;
+    if (r < 1 || r > L->desc.max_r || r > d || r > H) return CLEARMOE_EINVAL;
+    if (misaligned(W1) || misaligned(b1) || misaligned(U_r) || misaligned(S_r) || misaligned(Vh_r) ||
+        misaligned(R) || misaligned(out))
+        return CLEARMOE_EINVAL;
+    const bool bf16 = L->desc.dtype == CLEARMOE_BF16;
+    if (r % (bf16 ? 16 : 4)) return CLEARMOE_EUNSUPPORTED;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    mark(L, 0, s);
+    if ((rc = do_route(L, x, T, router, nullptr, E, 0, s))) return rc;  // idx, in token order
+    mark(L, 1, s);
+    if (!bf16) {
+        cm::SimtGemmArgs g;
+        std::memset(&g, 0, sizeof(g));
+        g.A0 = static_cast<const float*>(x);  // z = GELU(W1 x + b1), token order
+        g.lda0 = d;
+        g.K0 = d;
+        g.B0 = static_cast<const float*>(W1);
+        g.M = T;
+        g.N = H;
+        g.bias = static_cast<const float*>(b1);
+        g.gelu = 1;
+        g.C = static_cast<float*>(L->z);
+        g.ldc = H;
+        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        mark(L, 2, s);
+        std::memset(&g, 0, sizeof(g));  // t' = diag(S_r) Vh_r z / s_a
+        g.A0 = static_cast<const float*>(L->z);
+        g.lda0 = H;
+        g.K0 = H;
+        g.B0 = static_cast<const float*>(Vh_r);
+        g.M = T;
+        g.N = r;
+        g.scale = S_r;
+        g.row_group = L->idx;
+        g.group_scale = s_e;
+        g.scale_groups = E;
+        g.row_scale_inv = 1;
+        g.C = static_cast<float*>(L->t);
+        g.ldc = r;
+        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        mark(L, 3, s);
+        std::memset(&g, 0, sizeof(g));  // out = s_a (U_r t' + R z)
+        g.A0 = static_cast<const float*>(L->t);
+        g.lda0 = r;
+        g.K0 = r;
+        g.B0 = static_cast<const float*>(U_r);
+        g.A1 = static_cast<const float*>(L->z);
+        g.lda1 = H;
+        g.K1 = H;
+        g.B1[0] = static_cast<const float*>(R);
+        g.M = T;
+        g.N = d;
+        g.row_group = L->idx;
+        g.group_scale = s_e;
+        g.scale_groups = E;
+        g.C = static_cast<float*>(out);
+        g.ldc = d;
+        rc = cuda_fail(cm::launch_simt_gemm(g, s));
+    } else {
+        const int p1 = H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;
+        const int p2 = cm::tc2_pick_bn(cm::TC_DENSE, r), p3 = cm::tc2_pick_bn(cm::TC_GROUPED, d);
+        const int b1n = cm::tc_pick_bn(cm::TC_DENSE, H), b2n = cm::tc_pick_bn(cm::TC_DENSE, r);
+        const int b3n = cm::tc_pick_bn(cm::TC_GROUPED, d);
+        if ((!p1 && !b1n) || (!p2 && !b2n) || (!p3 && !b3n)) return CLEARMOE_EUNSUPPORTED;
+        cm::TcGemmArgs g;
+        std::memset(&g, 0, sizeof(g));
+        g.status = L->status;
+        g.wait_limit_ns = L->wait_limit_ns;
+        if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, p1 ? p1 / 2 : b1n))
+            return CLEARMOE_ECUDA;
+        g.mode = cm::TC_DENSE;
+        g.epi = cm::TC_EPI_BIAS_GELU;
+        g.M = T;
+        g.N = H;
+        g.K0 = d;
+        g.bias = b1;
+        g.C = L->z;
+        g.ldc = H;
+        if ((rc = cuda_fail(p1 ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s))))
+            return rc;
+        mark(L, 2, s);
+        cm::TcGemmArgs g2;
+        std::memset(&g2, 0, sizeof(g2));
+        g2.status = L->status;
+        g2.wait_limit_ns = L->wait_limit_ns;
+        if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, Vh_r, r, H, p2 ? p2 / 2 : b2n))
+            return CLEARMOE_ECUDA;
+        g2.mode = cm::TC_DENSE;
+        g2.epi = cm::TC_EPI_SCALE;
+        g2.M = T;
+        g2.N = r;
+        g2.K0 = H;
+        g2.scale = S_r;
+        g2.row_group = L->idx;
+        g2.group_scale = s_e;
+        g2.scale_groups = E;
+        g2.row_scale_inv = 1;
+        g2.C = L->t;
+        g2.ldc = r;
+        g2.a_evict_first = 1;
+        if ((rc = cuda_fail(p2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s))))
+            return rc;
+        mark(L, 3, s);
+        cm::TcGemmArgs g3;
+        std::memset(&g3, 0, sizeof(g3));
+        g3.status = L->status;
+        g3.wait_limit_ns = L->wait_limit_ns;
+        const int box3 = p3 ? p3 / 2 : b3n;
+        if (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, box3) ||
+            encode_tmap_bf16(&g3.tmA1, L->z, T, H, 128) || encode_tmap_bf16(&g3.tmB1[0], R, d, H, box3))
+            return CLEARMOE_ECUDA;
+        g3.mode = cm::TC_GROUPED;  // one group over all tokens (no offsets): [z | t'] x [R | U_r]
+        g3.epi = cm::TC_EPI_STORE;
+        g3.M = T;
+        g3.N = d;
+        g3.K0 = r;
+        g3.K1 = H;
+        g3.E = 1;
+        g3.row_group = L->idx;
+        g3.group_scale = s_e;
+        g3.scale_groups = E;
+        g3.C = out;
+        g3.ldc = d;
+        rc = cuda_fail(p3 ? cm::launch_tc_gemm2(g3, L->num_sms, s) : cm::launch_tc_gemm(g3, L->num_sms, s));
+    }
+    mark(L, 4, s);
+    if (rc) return rc;
+    return do_finalize(L, s);  // counts, offsets, perm for clearmoe_get_routing (off the path)
+}
+
 int clearmoe_materialize_basis(clearmoe_layer* L, const void* U_r, const float* S_r, const void* Vh_r, int32_t r,
                                void* W_sh, void* stream) {
     if (!L || !U_r || !S_r || !Vh_r || !W_sh) return CLEARMOE_EINVAL;

@@ -80,6 +80,11 @@ struct SimtGemmArgs {
     const int32_t* offsets;  // grouped: expert boundaries [E + 1] (nullable = not grouped)
     int E;
     int dense_last;          // grouped: the last group (the dense path) has no first K segment
+    // row scale: C[m, :] *= group_scale[row_group[m]] (1 / that with row_scale_inv), m < M
+    const int32_t* row_group;
+    const float* group_scale;
+    int scale_groups;
+    int row_scale_inv;
 };
 cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s);
 
@@ -130,10 +135,31 @@ struct TcGemmArgs {
     int64_t rt_cls_stride;
     // C is fp32 (stored as computed, no rounding): the MLP router's hidden layer
     int c_f32;
+    // row scale applied last: output row m (before any scatter) times group_scale[row_group[m]]
+    // (its reciprocal with row_scale_inv); a group index outside [0, scale_groups) scales by 1.
+    // Grouped mode with offsets == nullptr is a single group [0, M).
+    const int32_t* row_group;
+    const float* group_scale;
+    int scale_groups;
+    int row_scale_inv;
     // 2-SM kernel: A tiles loaded with the L2 evict-first policy (a stream read once), so that they
     // displace one another rather than lines the next reads are still to find in L2
     int a_evict_first;
 };
+// Boundary e of a grouped GEMM's groups: offsets[e], or the single group [0, M) without offsets.
+__host__ __device__ inline int64_t tc_group_off(const TcGemmArgs& a, int e) {
+    return a.offsets ? (int64_t)a.offsets[e] : (e == 0 ? 0 : a.M);
+}
+#ifdef __CUDACC__
+// The row scale of output row m (1 without group_scale or for an out-of-range group index).
+__device__ __forceinline__ float tc_row_scale(const TcGemmArgs& a, int64_t m) {
+    if (!a.group_scale) return 1.f;
+    const int g = a.row_group[m];
+    if ((unsigned)g >= (unsigned)a.scale_groups) return 1.f;
+    const float s = a.group_scale[g];
+    return a.row_scale_inv ? 1.f / s : s;
+}
+#endif
 int tc_pick_bn(int mode, int N);
 // 2-SM (cta_group::2) variant for the dense and grouped modes: 256 x BN tiles per CTA pair, BN =
 // tc2_pick_bn(mode, N) (256 or 128; 0 = shape not supported; each CTA's B box is BN / 2 rows).

@@ -342,32 +342,45 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         auto bias_of = [&](int e) -> float {
             return a.w_bf16 ? bf16_to_f32(static_cast<const uint16_t*>(a.bg)[e]) : static_cast<const float*>(a.bg)[e];
         };
+        // one row per lane: each lane streams its row in 16-float chunks (float4 loads; the L1
+        // merges the 32 rows' sectors) against W_g broadcast from shared memory, fp32 FMA in k
+        // order, so a warp routes 32 rows with no cross-lane reduction (d % 4 == 0)
         const float* X = static_cast<const float*>(a.x);
-        for (int i = warp; i < nrows; i += NWARPS) {
-            const float* xr = X + (row0 + i) * d;
+        for (int b0 = warp * 32; b0 < nrows; b0 += NWARPS * 32) {
+            const int i = b0 + lane;
+            const bool valid = i < nrows;
+            const float4* xr = reinterpret_cast<const float4*>(X + (row0 + (valid ? i : 0)) * d);
             float acc[CM_MAX_E];
 #pragma unroll
             for (int e = 0; e < CM_MAX_E; ++e) acc[e] = 0.f;
-            for (int k = lane; k < d; k += 32) {
-                const float xv = xr[k];
+            for (int k4 = 0; k4 < d / 4; k4 += 4) {
+                float4 xv[4];
 #pragma unroll
-                for (int e = 0; e < CM_MAX_E; ++e)
-                    if (e < E) acc[e] = fmaf(xv, Wf[e * d + k], acc[e]);
+                for (int j = 0; j < 4; ++j) xv[j] = (k4 + j < d / 4) ? xr[k4 + j] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    if (k4 + j < d / 4) {
+#pragma unroll
+                        for (int e = 0; e < CM_MAX_E; ++e) {
+                            if (e < E) {
+                                const float4 w = reinterpret_cast<const float4*>(Wf + (size_t)e * d)[k4 + j];
+                                acc[e] = fmaf(xv[j].x, w.x, acc[e]);
+                                acc[e] = fmaf(xv[j].y, w.y, acc[e]);
+                                acc[e] = fmaf(xv[j].z, w.z, acc[e]);
+                                acc[e] = fmaf(xv[j].w, w.w, acc[e]);
+                            }
+                        }
+                    }
+                }
             }
             float bv = -INFINITY;
             int be = 0x7fffffff;
 #pragma unroll
-            for (int e = 0; e < CM_MAX_E; ++e) {
-                if (e < E) {
-                    float v = acc[e];
-#pragma unroll
-                    for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-                    arg_better(bv, be, v + bias_of(e), e);
-                }
-            }
-            if (be > E - 1) be = 0;
+            for (int e = 0; e < CM_MAX_E; ++e)
+                if (e < E) arg_better(bv, be, acc[e] + bias_of(e), e);
+            if (be > E - 1) be = 0;  // only reachable with non-finite logits
             if (a.cls_stride > 0 && (row0 + i) % a.cls_stride == 0) be = E;  // a class token
-            if (lane == 0) record(i, be, 0);
+            if (valid) record(i, be, 0);
         }
     }
     __syncthreads();

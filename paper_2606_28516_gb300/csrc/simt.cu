@@ -107,6 +107,10 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
             if (a.gelu) v = gelu_erf(v);
             if (a.relu) v = fmaxf(v, 0.f);
             if (a.scale) v *= a.scale[n];
+            if (a.group_scale) {
+                const int g = a.row_group[m];
+                if ((unsigned)g < (unsigned)a.scale_groups) v = a.row_scale_inv ? v / a.group_scale[g] : v * a.group_scale[g];
+            }
             a.C[orow * a.ldc + n] = v;
         }
     }

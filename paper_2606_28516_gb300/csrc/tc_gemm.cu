@@ -66,7 +66,7 @@ __device__ __forceinline__ TileInfo decode_tile(const TcGemmArgs& a, int tile, i
     if (a.mode == TC_GROUPED) {
         int e = 0;
         while (e + 1 < a.E && s_prefix[e + 1] <= mt) ++e;
-        const int64_t lo = a.offsets[e], hi = a.offsets[e + 1];
+        const int64_t lo = tc_group_off(a, e), hi = tc_group_off(a, e + 1);
         t.m0 = lo + (int64_t)(mt - s_prefix[e]) * TC_BM;
         t.rows = (int)min((int64_t)TC_BM, hi - t.m0);
         t.e = e;
@@ -130,7 +130,7 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
             int acc = 0;
             for (int e = 0; e < a.E; ++e) {
                 s_prefix[e] = acc;
-                acc += (a.offsets[e + 1] - a.offsets[e] + TC_BM - 1) / TC_BM;
+                acc += (int)((tc_group_off(a, e + 1) - tc_group_off(a, e) + TC_BM - 1) / TC_BM);
             }
             s_prefix[a.E] = acc;
         }
@@ -294,6 +294,7 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
             const int r = q * 32 + lane;
             int64_t orow = -1;
             if (r < t.rows) orow = (a.epi == TC_EPI_SCATTER) ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
+            const float rsc = (a.group_scale && r < t.rows) ? tc_row_scale(a, t.m0 + r) : 1.f;
             if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;
             for (int c = c_lo; c < c_lo + C::HALF; c += C::CW) {
                 uint32_t v[32];
@@ -357,6 +358,10 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
                         f[4 * j4 + 2] *= s4.z;
                         f[4 * j4 + 3] *= s4.w;
                     }
+                }
+                if (a.group_scale) {
+#pragma unroll
+                    for (int j = 0; j < C::CW; ++j) f[j] *= rsc;
                 }
                 if (a.c_f32) {  // fp32 output: each lane stores its row's values as computed
                     if (orow >= 0) {

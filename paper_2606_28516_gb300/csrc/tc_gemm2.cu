@@ -119,8 +119,8 @@ __device__ __forceinline__ PairTile decode_pair(const TcGemmArgs& a, int unit, i
     if (a.mode == TC_GROUPED) {
         int e = 0;
         while (e + 1 < a.E && s_prefix[e + 1] <= mp) ++e;
-        t.m0 = (int64_t)a.offsets[e] + (int64_t)(mp - s_prefix[e]) * 2 * BM;
-        t.hi = a.offsets[e + 1];
+        t.m0 = tc_group_off(a, e) + (int64_t)(mp - s_prefix[e]) * 2 * BM;
+        t.hi = tc_group_off(a, e + 1);
         t.e = e;
     } else {
         t.m0 = (int64_t)mp * 2 * BM;
@@ -280,7 +280,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
             int acc = 0;
             for (int e = 0; e < a.E; ++e) {
                 s_prefix[e] = acc;
-                acc += (a.offsets[e + 1] - a.offsets[e] + 2 * BM - 1) / (2 * BM);
+                acc += (int)((tc_group_off(a, e + 1) - tc_group_off(a, e) + 2 * BM - 1) / (2 * BM));
             }
             s_prefix[a.E] = acc;
         }
@@ -442,6 +442,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                     if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
                 }
             }
+            const float rsc = (a.group_scale && mrow < t.hi) ? tc_row_scale(a, mrow) : 1.f;
             // this lane stores rows p * RPP + lane / LPR of the warp's 32 (p < LPR), 16-byte chunk
             // lane % LPR: their destinations, once per tile
             uint16_t* dst_row[LPR];
@@ -507,6 +508,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                         f[4 * j4 + 1] = p0.y;
                         f[4 * j4 + 2] = p1.x;
                         f[4 * j4 + 3] = p1.y;
+                    }
+                }
+                if (a.group_scale) {
+#pragma unroll
+                    for (int j2 = 0; j2 < CW / 2; ++j2) {
+                        const float2 p2 = __fmul2_rn(make_float2(f[2 * j2], f[2 * j2 + 1]), make_float2(rsc, rsc));
+                        f[2 * j2] = p2.x;
+                        f[2 * j2 + 1] = p2.y;
                     }
                 }
                 if (a.c_f32) {  // fp32 output: each lane stores its row's 32 values as computed
