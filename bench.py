@@ -352,6 +352,8 @@ def main():
     ap.add_argument("--workload", default="deit_base_bf16", choices=sorted(workloads()))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--no-variants", action="store_true",
+                    help="skip the variant timings (folded, materialised, class tokens, MLP router, one residual)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
@@ -460,7 +462,7 @@ def main():
         return {"value": world * s.T / (v_ms / 1e3), "unit": "tokens/s", "ms_per_step": v_ms, "note": note}
 
     folded = materialized = class_tokens = mlp_router = scaled = None
-    if s.dtype == "bf16":
+    if s.dtype == "bf16" and not args.no_variants:
         W_comb = torch.empty_like(D["residuals"])
         cm.clearmoe_fold_basis(h, D["U"], D["S"], D["Vh"], D["residuals"], W_comb)
         folded = time_variant(
