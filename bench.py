@@ -51,6 +51,35 @@ TRAFFIC = {
 }
 
 
+def init_replicas(backend="nccl"):
+    """One process per GPU (torchrun's RANK / WORLD_SIZE / LOCAL_RANK): (world, rank, local, dist),
+    dist None for a single process. Each rank runs an independent replica on its own token shard;
+    the only collectives are the barriers and the max of the rank times."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group(backend)
+    return world, rank, local, dist
+
+
+def max_over_ranks(x: float, dist, device="cuda") -> float:
+    """The largest of the ranks' values (a time: the job is as slow as its slowest rank)."""
+    if not dist:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: int, world: int, steps: int, ms: float) -> float:
+    """Units per second over all ranks (weak scaling: every rank processes units_per_rank per step)."""
+    return world * units_per_rank * steps / (ms / 1e3)
+
+
 def workloads():
     import synth
     return {"deit_base_bf16": synth.DEIT_BASE_BF16, "deit_small_bf16": synth.DEIT_SMALL_BF16,
@@ -219,14 +248,8 @@ def run_stack(args):
     from paper_2606_28516_gb300 import clearmoe as cm
     from oracle import clearmoe as O
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local, dist = init_replicas("nccl")
     torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
     if rank == 0:
         __graft_entry__.build()
     if dist:
@@ -279,17 +302,13 @@ def run_stack(args):
             ev[k][1].record()
         torch.cuda.synchronize()
         assert cm.clearmoe_layer_status(h) == 0
-        ms = float(sum(e[0].elapsed_time(e[1]) for e in ev))
-        if dist:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
+        ms = max_over_ranks(float(sum(e[0].elapsed_time(e[1]) for e in ev)), dist)
         return ms / K
 
     K = max(1, min(args.steps, 50))
     with ClockSampler(local) as clk:
         ms = timed(K)
-    value = world * T / (ms / 1e3)
+    value = whole_job_rate(T, world, 1, ms)
     # folded variant of the same stack (each converted sublayer's basis folded once)
     for G in layers:
         if G["moe"]:
@@ -309,7 +328,7 @@ def run_stack(args):
         outh.copy_(stack_pass(xd), non_blocking=True)
     e1.record()
     torch.cuda.synchronize()
-    e2e_value = world * T * Ke / (e0.elapsed_time(e1) / 1e3)
+    e2e_value = whole_job_rate(T, world, Ke, max_over_ranks(e0.elapsed_time(e1), dist))
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n = 2048
@@ -335,7 +354,7 @@ def run_stack(args):
         "gpu_launches": 6 * 4 + 6 * 2 + 12,
         "cpu_baseline": cpu,
         "clocks": clk.summary(),
-        "folded": {"value": world * T / (ms_f / 1e3), "unit": "tokens/s", "ms_per_step": ms_f},
+        "folded": {"value": whole_job_rate(T, world, 1, ms_f), "unit": "tokens/s", "ms_per_step": ms_f},
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -368,14 +387,8 @@ def main():
     import __graft_entry__
     from paper_2606_28516_gb300 import clearmoe as cm
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local, dist = init_replicas("nccl")
     torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
     if rank == 0:
         __graft_entry__.build()
     if dist:
@@ -439,11 +452,8 @@ def main():
     assert cm.clearmoe_layer_status(h) == 0
     stage_ms = {st: [sev[k][i].elapsed_time(sev[k][i + 1]) for k in range(Ks)]
                 for i, st in enumerate(STAGES)}
-    if dist:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    value = world * s.T * K / (total_ms / 1e3)
+    total_ms = max_over_ranks(total_ms, dist)
+    value = whole_job_rate(s.T, world, K, total_ms)
 
     # Variants of the same layer, same timing rules (events around each forward only, L2 flushed
     # before each). Reported beside the headline, not as it.
@@ -458,8 +468,9 @@ def main():
                 vev[k - args.warmup][1].record(stream)
         torch.cuda.synchronize()
         assert cm.clearmoe_layer_status(h) == 0
-        v_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in vev)
-        return {"value": world * s.T / (v_ms / 1e3), "unit": "tokens/s", "ms_per_step": v_ms, "note": note}
+        v_ms = max_over_ranks(statistics.mean(e[0].elapsed_time(e[1]) for e in vev), dist)
+        return {"value": whole_job_rate(s.T, world, 1, v_ms), "unit": "tokens/s", "ms_per_step": v_ms,
+                "note": note}
 
     folded = materialized = class_tokens = mlp_router = scaled = None
     if s.dtype == "bf16" and not args.no_variants:
@@ -506,7 +517,7 @@ def main():
             dev[k - args.warmup][1].record(stream)
     torch.cuda.synchronize()
     dense_ms = [e[0].elapsed_time(e[1]) for e in dev]
-    dense_value = s.T / (statistics.mean(dense_ms) / 1e3)
+    dense_value = whole_job_rate(s.T, world, 1, max_over_ranks(statistics.mean(dense_ms), dist))
 
     # End to end through the C ABI with host buffers: every step copies its tokens from pinned
     # host memory and its output back. Steps are pipelined over three streams (copy-in of step
@@ -556,11 +567,8 @@ def main():
     e2e_ms = e2e_t0.elapsed_time(e2e_t1)
     if not torch.equal(out_host[(Ke - 1) & 1].cuda(), o_dev[(Ke - 1) & 1]):
         raise RuntimeError("end-to-end output copy mismatch")
-    if dist:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e_value = world * s.T * Ke / (e2e_ms / 1e3)
+    e2e_ms = max_over_ranks(e2e_ms, dist)
+    e2e_value = whole_job_rate(s.T, world, Ke, e2e_ms)
     assert cm.clearmoe_layer_status(h) == 0
     cm.clearmoe_layer_destroy(h)
 
