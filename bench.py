@@ -83,7 +83,8 @@ def whole_job_rate(units_per_rank: int, world: int, steps: int, ms: float) -> fl
 def workloads():
     import synth
     return {"deit_base_bf16": synth.DEIT_BASE_BF16, "deit_small_bf16": synth.DEIT_SMALL_BF16,
-            "deit_tiny_fp32": synth.DEIT_TINY_FP32, "vit_base_stack12": synth.VIT_BASE_STACK12}
+            "deit_tiny_fp32": synth.DEIT_TINY_FP32, "vit_base_stack12": synth.VIT_BASE_STACK12,
+            "deit_small_zipf_sweep": None}
 
 
 def peaks():
@@ -207,6 +208,9 @@ def run_reference(args):
     if rank != 0:
         return
     shape = workloads()[args.workload]
+    if not isinstance(shape, synth.LayerShape):  # the sweep and the stack: one of their layers
+        shape = (synth.deit_small_zipf(4, 64) if args.workload == "deit_small_zipf_sweep"
+                 else synth.DEIT_BASE_BF16.with_(T=synth.VIT_BASE_STACK12.T))
     L = synth.make_layer(shape)
     # per-step sample sized so that warmup + steps take about a minute of CPU time in total
     probe, _, _ = oracle_rate(L, budget_s=2.0, chunk=256, max_tokens=512)
@@ -234,6 +238,79 @@ def run_reference(args):
         "gpu_launches": 0,
     }
     print(json.dumps(line), flush=True)
+
+
+def run_sweep(args):
+    """The expert-count x rank sweep on the DeiT-S shape with Zipf(1.2) cluster sizes (E in
+    {2, 3, 4, 6, 8} x r in {16, 32, 64, 128, 256}, T = 12,608, bf16): tokens/s of the whole layer at
+    each point, timed like the headline (L2 flushed before each forward: the 9.7 MB of tokens fit
+    in L2), beside the same-shape dense FFN. value = the median over the 25 points."""
+    import torch
+
+    import synth
+    import __graft_entry__
+    from paper_2606_28516_gb300 import clearmoe as cm
+
+    world, rank, local, dist = init_replicas("nccl")
+    torch.cuda.set_device(local)
+    if rank == 0:
+        __graft_entry__.build()
+    if dist:
+        dist.barrier()
+    cm.lib()
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.int32, device="cuda")
+    K = max(1, min(args.steps, 100))
+
+    def time_fn(fn):
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
+        for k in range(args.warmup + K):
+            flush.zero_()
+            if k >= args.warmup:
+                ev[k - args.warmup][0].record()
+            fn()
+            if k >= args.warmup:
+                ev[k - args.warmup][1].record()
+        torch.cuda.synchronize()
+        return max_over_ranks(statistics.mean(e[0].elapsed_time(e[1]) for e in ev), dist)
+
+    points, dense = [], None
+    with ClockSampler(local) as clk:
+        for E in synth.ZIPF_E:
+            for r in synth.ZIPF_R:
+                shape = synth.deit_small_zipf(E, r, seed=rank).with_(n_cal=8000)
+                L = synth.make_layer(shape)
+                D = synth.to_torch(L)
+                h = cm.clearmoe_layer_create(shape.T, shape.d, shape.H, E, r, cm.BF16)
+                out = torch.empty(shape.T, shape.d, device="cuda", dtype=torch.bfloat16)
+                ms = time_fn(lambda: cm.clearmoe_ffn_forward(h, D["x"], D["W1"], D["b1"], D["U"], D["S"], D["Vh"],
+                                                             D["residuals"], D["Wg"], D["bg"], out))
+                if dense is None:
+                    dms = time_fn(lambda: cm.clearmoe_dense_ffn_forward(h, D["x"], D["W1"], D["b1"], D["W2"], out))
+                    dense = {"value": whole_job_rate(shape.T, world, 1, dms), "unit": "tokens/s", "ms_per_step": dms}
+                assert cm.clearmoe_layer_status(h) == 0
+                counts = torch.empty(E, dtype=torch.int32, device="cuda")
+                cm.clearmoe_get_routing(h, counts=counts)
+                c = counts.cpu().tolist()
+                points.append({"E": E, "r": r, "tokens_s": whole_job_rate(shape.T, world, 1, ms), "ms": ms,
+                               "largest_expert_share": max(c) / shape.T})
+                cm.clearmoe_layer_destroy(h)
+                del D, L
+    value = statistics.median(p["tokens_s"] for p in points)
+    if rank == 0:
+        print(json.dumps({
+            "metric": "CLEAR-MoE FFN tokens/sec/layer over the E x r sweep (DeiT-S shape, Zipf cluster sizes)",
+            "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K, "warmup": args.warmup,
+            "ms_per_step": statistics.median(p["ms"] for p in points), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "deit_small_zipf_sweep", "T": 12608, "d": 384, "H": 1536,
+                       "E": list(synth.ZIPF_E), "r": list(synth.ZIPF_R), "sizes": "zipf(1.2)",
+                       "n_cal": 8000, "value": "median over the 25 points", "l2": "flushed between steps",
+                       "parallelism": f"replicas{world}"},
+            "points": points, "dense_ffn": dense, "clocks": clk.summary(),
+            "gpu_launches": 4 * K * len(points),
+        }), flush=True)
+    if dist:
+        dist.destroy_process_group()
 
 
 def run_stack(args):
@@ -379,6 +456,8 @@ def main():
         return run_reference(args)
     if args.workload == "vit_base_stack12":
         return run_stack(args)
+    if args.workload == "deit_small_zipf_sweep":
+        return run_sweep(args)
 
     import numpy as np
     import torch
