@@ -162,7 +162,7 @@ __device__ __forceinline__ float tc_row_scale(const TcGemmArgs& a, int64_t m) {
 #endif
 int tc_pick_bn(int mode, int N);
 // 2-SM (cta_group::2) variant for the dense and grouped modes: 256 x BN tiles per CTA pair, BN =
-// tc2_pick_bn(mode, N) (256 or 128; 0 = shape not supported; each CTA's B box is BN / 2 rows).
+// tc2_pick_bn(mode, N) (256, 192 or 128; 0 = shape not supported; each CTA's B box is BN / 2 rows).
 // Its bias + GELU and column-scale epilogues stage the vector in shared memory (N <= TC2_BIAS_CAP).
 constexpr int TC2_BIAS_CAP = 4096;
 constexpr int TC2_TAB_CAP = 2432;  // routing prefix table entries (ranges x experts)

@@ -20,7 +20,7 @@
 #include "internal.h"
 
 namespace cm {
-// Tile configuration by pair-tile width BN (256 or 128 columns).
+// Tile configuration by pair-tile width BN (256, 192 or 128 columns).
 template <int BN_>
 struct T2 {
     static constexpr int BM = 128;                        // rows per CTA; the pair covers 256
@@ -28,9 +28,9 @@ struct T2 {
     static constexpr int BH = BN / 2;                     // B rows per CTA
     static constexpr int BK = 64;
     static constexpr int A_BYTES = BM * BK * 2;           // 16 KB
-    static constexpr int B_BYTES = BH * BK * 2;           // 16 KB (BN 256) / 8 KB (BN 128)
+    static constexpr int B_BYTES = BH * BK * 2;           // 16 KB (BN 256), 12 KB (192), 8 KB (128)
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES = BN == 256 ? 6 : 8;      // 192 KB of operands either way
+    static constexpr int STAGES = 192 * 1024 / STAGE_BYTES;  // at most 192 KB of operands: 6 / 6 / 8
     static constexpr int NUM_EPI = 8;                     // two per TMEM lane quarter
     static constexpr int WARP_MMA = NUM_EPI, WARP_TMA = NUM_EPI + 1;
     static constexpr int THREADS = 32 * (WARP_TMA + 1);
@@ -46,7 +46,7 @@ struct T2 {
     static constexpr int NBARS = 2 * STAGES + 5;
     static constexpr int SMEM =
         1024 + STAGES * STAGE_BYTES + STG_BYTES + BIAS_CAP * 4 + (TAB_CAP + CM_MAX_E) * 4 + NBARS * 8 + 128;
-    static constexpr int TMEM_COLS = 2 * BN;              // two accumulators
+    static constexpr int TMEM_COLS = 2 * BN <= 256 ? 256 : 512;  // two accumulators (a power of 2)
 };
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -570,6 +570,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
 int tc2_pick_bn(int mode, int N) {
     if (mode != TC_DENSE && mode != TC_GROUPED) return 0;
     if (N % 256 == 0) return 256;
+    if (N % 192 == 0) return 192;  // e.g. d = 384: two 192-wide tiles instead of three 128-wide ones
     if (N % 128 == 0) return 128;
     return 0;
 }
@@ -611,7 +612,9 @@ cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
                         a.epi == TC_EPI_SCALE;  // fp32 vector in shared memory
     if (!bn || (staged && (a.mode != TC_DENSE || a.N > TC2_BIAS_CAP))) return cudaErrorInvalidValue;
     if (a.out_bias && (staged || a.N > TC2_BIAS_CAP)) return cudaErrorInvalidValue;
-    return bn == 256 ? launch2<256>(a, num_sms, s) : launch2<128>(a, num_sms, s);
+    if (bn == 256) return launch2<256>(a, num_sms, s);
+    if (bn == 192) return launch2<192>(a, num_sms, s);
+    return launch2<128>(a, num_sms, s);
 }
 
 }  // namespace cm
