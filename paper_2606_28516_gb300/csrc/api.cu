@@ -399,6 +399,9 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         } else {
             g.rows = L->inv;
         }
+        // x and W1 are ready before the routing (which releases fc1 only after its own wait): the
+        // operand loads and MMAs start at once; the epilogue waits for the routing's results
+        g.pdl_wait_role = 1;
         rc = cuda_fail(cm::launch_tc_gemm2(g, L->num_sms, s));
     } else {
         if (encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
@@ -428,6 +431,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         g2.C = L->t;
         g2.ldc = r;
         g2.a_evict_first = 1;  // z is streamed once here; its rows still in L2 from fc1 stay there
+        g2.pdl_trigger_late = 1;  // the grouped GEMM may start once fc1 has completed
         rc = cuda_fail(p2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
         if (rc) return rc;
     }
@@ -452,6 +456,9 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         g3.dense_last = 1;
     }
     g3.out_bias = b2;
+    // after the 2-SM basis kernel (which releases it only once fc1 has completed) the grouped GEMM
+    // starts its z segments at once and waits for the basis only before its first t segment
+    if (factored && cm::tc2_pick_bn(cm::TC_DENSE, r)) g3.pdl_wait_role = 2;
     g3.mode = cm::TC_GROUPED;
     g3.epi = cm::TC_EPI_SCATTER;
     g3.M = T;

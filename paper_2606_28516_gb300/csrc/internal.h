@@ -142,6 +142,14 @@ struct TcGemmArgs {
     const float* group_scale;
     int scale_groups;
     int row_scale_inv;
+    // 2-SM kernel, launch overlap with the previous kernel (programmatic dependent launch):
+    // pdl_wait_role 0: every thread waits for it after the setup; 1: only the epilogue warps wait
+    // (their routing table and slots are its results; the operand loads and MMAs start at once);
+    // 2: only the producer waits, before its first load of the K0 (t) segment (the z segment and the
+    // epilogue need nothing from it). pdl_trigger_late: release the next kernel only after the wait,
+    // so that it starts once this kernel's own predecessors have completed.
+    int pdl_wait_role;
+    int pdl_trigger_late;
     // 2-SM kernel: A tiles loaded with the L2 evict-first policy (a stream read once), so that they
     // displace one another rather than lines the next reads are still to find in L2
     int a_evict_first;

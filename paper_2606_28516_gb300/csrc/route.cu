@@ -123,7 +123,6 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
     __shared__ int s_wc[RT_MAX_WARPS][CM_MAX_E];
     __shared__ int s_abort;
 
-    pdl_launch_dependents();  // the kernel that follows may set itself up meanwhile
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int E = a.E, d = a.d;
     const int64_t row0 = (int64_t)blockIdx.x * chunk;
@@ -176,6 +175,9 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
             for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(smem) + e * WRB, Wb + (size_t)e * d * 2, d * 2, wbar);
         }
         pdl_wait();  // from here on the previous kernel's results (x) are read and outputs written
+        // the next kernel may start now (its CTAs set up, and may read x, while this one streams):
+        // released only after the wait, so every kernel before this one has completed by then
+        pdl_launch_dependents();
         if (warp == NCONS_MAX) {
             if (producer) {
                 const unsigned char* xb = static_cast<const unsigned char*>(a.x) + row0 * d * 2;
@@ -338,6 +340,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
             for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = W[i];
         }
         pdl_wait();
+        pdl_launch_dependents();
         __syncthreads();
         auto bias_of = [&](int e) -> float {
             return a.w_bf16 ? bf16_to_f32(static_cast<const uint16_t*>(a.bg)[e]) : static_cast<const float*>(a.bg)[e];

@@ -151,7 +151,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* s_prefix = reinterpret_cast<int*>(tmem_slot + 4);  // [CM_MAX_E + 1]
 
-    pdl_launch_dependents();
+    if (!a.pdl_trigger_late) pdl_launch_dependents();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = cluster_rank();
     const bool leader = rank == 0;
@@ -203,8 +203,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
     __syncthreads();
     cluster_sync();  // barriers initialised and TMEM bases written in both CTAs
     tc_fence_after();
-    // everything above overlaps the predecessor kernel; from here on its results are read
-    pdl_wait();
+    // everything above overlaps the predecessor kernel; from here on its results are read (by
+    // every thread, or by the roles that read them: see pdl_wait_role)
+    if (a.pdl_wait_role == 0 || (a.pdl_wait_role == 1 && warp < NUM_EPI)) pdl_wait();
+    if (a.pdl_trigger_late) pdl_launch_dependents();
     if (MODE == TC_DENSE && a.rt_info && warp < NUM_EPI) {
         // Routing prefix table, by the epilogue warps while the producer and MMA warps start:
         // thread c holds routing range c's counts; per expert, an exclusive scan over ranges (warp
@@ -306,6 +308,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         if (lane == 0) {
             const uint32_t full_leader0 = map_to_rank(full_bar(0), 0);
             const uint64_t pol_a = l2_policy_evict_first();
+            bool waited = a.pdl_wait_role != 2;  // role 2: wait before the first t-segment load
             int stage = 0;
             uint32_t ph = 0;
             bool ok = true;
@@ -335,6 +338,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                         mB = &a.tmB1[t.e];
                         kk = kb * BK;
                     } else {  // t x U_r
+                        if (!waited) {
+                            pdl_wait();
+                            waited = true;
+                        }
                         mA = &a.tmA0;
                         mB = &a.tmB0;
                         kk = (kb - nk1) * BK;
