@@ -125,8 +125,10 @@ def test_class_tokens_ragged(workload, T):
     assert out_error(out, y, "bf16") <= tol("bf16")
 
 
-@pytest.mark.parametrize("shape", [synth.DEIT_TINY_FP32, synth.DEIT_SMALL_BF16])
+@pytest.mark.parametrize("shape", [synth.DEIT_TINY_FP32, synth.DEIT_SMALL_BF16, synth.DEIT_BASE_BF16])
 def test_every_token_a_class_token_is_the_dense_ffn(workload, shape):
+    """No routed rows: no basis launch, so the grouped GEMM follows fc1 directly (DeiT-B: after the
+    2-SM basis it would start early; here it must wait for fc1)."""
     L = workload(shape)
     T = min(shape.T, 2000)
     out, gr = _forward(L, 1, T=T)
@@ -138,9 +140,10 @@ def test_every_token_a_class_token_is_the_dense_ffn(workload, shape):
 
 
 def test_one_sm_kernels_and_slot_kernel():
-    """d = 64, H = 192: fc1 gathers rows by perm (slot kernel, no fused epilogue), the basis and
-    grouped GEMMs run on the 1-SM kernel, whose last group skips the t segment."""
-    shape = synth.LayerShape("small_1sm_bf16", 1500, 64, 192, 3, 16, "bf16", n_cal=2000)
+    """d = 64, H = 320 (no 2-SM tile width divides it): fc1 gathers rows by perm (slot kernel, no
+    fused epilogue), the basis and grouped GEMMs run on the 1-SM kernel, whose last group skips the
+    t segment."""
+    shape = synth.LayerShape("small_1sm_bf16", 1500, 64, 320, 3, 16, "bf16", n_cal=2000)
     L = synth.make_layer(shape)
     out, gr = _forward(L, 50)
     _check_routing(gr, L, 50, shape.T)
