@@ -131,6 +131,8 @@ cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
 // variance of the centred values); x = (y - mean) / sqrt(var + 1e-6).
 template <bool BF16>
 __global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x, int64_t T, int d) {
+    pdl_wait();  // y is the previous kernel's output
+    pdl_launch_dependents();  // the next sublayer's first kernel may set itself up meanwhile
     const int lane = threadIdx.x & 31;
     const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
     if (row >= T) return;
@@ -201,12 +203,17 @@ __global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x,
 }
 
 cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s) {
-    const unsigned blocks = (unsigned)((T + 7) / 8);
-    if (dtype == CLEARMOE_BF16)
-        layer_norm_kernel<true><<<blocks, 256, 0, s>>>(y, x, T, d);
-    else
-        layer_norm_kernel<false><<<blocks, 256, 0, s>>>(y, x, T, d);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((T + 7) / 8));
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (dtype == CLEARMOE_BF16) return cudaLaunchKernelEx(&cfg, layer_norm_kernel<true>, y, x, T, d);
+    return cudaLaunchKernelEx(&cfg, layer_norm_kernel<false>, y, x, T, d);
 }
 
 }  // namespace cm
