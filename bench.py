@@ -44,10 +44,10 @@ KERNEL_OF_STAGE = {"route": "cm::route_kernel<1, 1>",
 # capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel sources
 # it was taken on; a different hash means the kernels changed and the figure is void.
 TRAFFIC = {
-    "route": {"bytes": 78.402048e6, "src": "f7c2fdba999c1fd9"},
-    "fc1_gelu": {"bytes": 338.240768e6, "src": "f7c2fdba999c1fd9"},
-    "basis": {"bytes": 315.837696e6, "src": "f7c2fdba999c1fd9"},
-    "grouped": {"bytes": 426.781696e6, "src": "f7c2fdba999c1fd9"},
+    "route": {"bytes": 78.551296e6, "src": "67c2c10bb509ef2c"},
+    "fc1_gelu": {"bytes": 338.262016e6, "src": "67c2c10bb509ef2c"},
+    "basis": {"bytes": 315.866368e6, "src": "67c2c10bb509ef2c"},
+    "grouped": {"bytes": 430.195200e6, "src": "67c2c10bb509ef2c"},
 }
 
 
