@@ -13,11 +13,15 @@
 
 namespace cm {
 
-constexpr int SG_M = 64, SG_N = 64, SG_K = 16;
+constexpr int SG_K = 64;  // K per shared-memory step (each thread keeps one k column of it)
 
+// TM x TM output tiles (64, or 32 when 64-wide tiles would leave most SMs idle), 256 threads, each
+// thread an (TM / 16) x (TM / 16) block of outputs.
+template <int TM>
 __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, const int n_tiles_n) {
-    __shared__ float As[SG_K][SG_M + 4];
-    __shared__ float Bs[SG_K][SG_N + 4];
+    constexpr int SG_M = TM, SG_N = TM, R = TM / 16, LD = TM * SG_K / 256;
+    __shared__ float As[SG_K][SG_M + 1];  // +1: the per-step stores (one k per thread) hit distinct banks
+    __shared__ float Bs[SG_K][SG_N + 1];
     const int tid = threadIdx.x;
     const int nt = blockIdx.x % n_tiles_n;
     const int mt = blockIdx.x / n_tiles_n;
@@ -46,12 +50,16 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
     const int n0 = nt * SG_N;
     const float* B1 = a.B1[a.offsets ? e : 0];
     const int tx = tid & 15, ty = tid >> 4;
-    float acc[4][4];
+    float acc[R][R];
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < R; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+        for (int j = 0; j < R; ++j) acc[i][j] = 0.f;
 
+    // Thread tid loads column kk = tid % SG_K of rows tid / SG_K + (256 / SG_K) i (i < LD) of both
+    // operand tiles; the next step's values are loaded into registers while this step computes.
+    const int kk = tid % SG_K, r0 = tid / SG_K;
+    constexpr int RS = 256 / SG_K;
     for (int seg = 0; seg < 2; ++seg) {
         const float* A = seg == 0 ? a.A0 : a.A1;
         const float* B = seg == 0 ? a.B0 : B1;
@@ -59,48 +67,59 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
         const int64_t lda = seg == 0 ? a.lda0 : a.lda1;
         if (A == nullptr || K == 0) continue;
         if (seg == 0 && a.offsets && a.dense_last && e == a.E - 1) continue;  // the dense path: z x W2 alone
+        int arow[LD];  // this thread's A rows (gathered for fc1), -1 outside the tile
+#pragma unroll
+        for (int i = 0; i < LD; ++i) {
+            const int64_t m = m_lo + r0 + RS * i;
+            arow[i] = -1;
+            if (m < m_hi) {
+                const int64_t ar = (seg == 0 && a.a_rows) ? (int64_t)a.a_rows[m] : m;
+                if ((uint64_t)ar < (uint64_t)a.M) arow[i] = (int)ar;  // M < 2^31
+            }
+        }
+        float ra[LD], rb[LD];
+        auto gload = [&](int k0) {
+            const int k = k0 + kk;
+#pragma unroll
+            for (int i = 0; i < LD; ++i) {
+                const int n = n0 + r0 + RS * i;
+                ra[i] = (arow[i] >= 0 && k < K) ? A[(int64_t)arow[i] * lda + k] : 0.f;
+                rb[i] = (n < a.N && k < K) ? B[(int64_t)n * K + k] : 0.f;
+            }
+        };
+        gload(0);
         for (int k0 = 0; k0 < K; k0 += SG_K) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int idx = tid + i * 256;
-                const int r = idx >> 4, kk = idx & 15;
-                const int64_t m = m_lo + r;
-                float v = 0.f;
-                if (m < m_hi && k0 + kk < K) {
-                    const int64_t ar = (seg == 0 && a.a_rows) ? (int64_t)a.a_rows[m] : m;
-                    if ((uint64_t)ar < (uint64_t)a.M) v = A[ar * lda + k0 + kk];
-                }
-                As[kk][r] = v;
-                const int n = n0 + r;
-                float w = 0.f;
-                if (n < a.N && k0 + kk < K) w = B[(int64_t)n * K + k0 + kk];
-                Bs[kk][r] = w;
+            for (int i = 0; i < LD; ++i) {
+                As[kk][r0 + RS * i] = ra[i];
+                Bs[kk][r0 + RS * i] = rb[i];
             }
             __syncthreads();
+            if (k0 + SG_K < K) gload(k0 + SG_K);
+#pragma unroll 8
+            for (int k = 0; k < SG_K; ++k) {
+                float av[R], bv[R];
 #pragma unroll
-            for (int kk = 0; kk < SG_K; ++kk) {
-                float av[4], bv[4];
+                for (int i = 0; i < R; ++i) av[i] = As[k][ty * R + i];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) av[i] = As[kk][ty * 4 + i];
+                for (int j = 0; j < R; ++j) bv[j] = Bs[k][tx * R + j];
 #pragma unroll
-                for (int j = 0; j < 4; ++j) bv[j] = Bs[kk][tx * 4 + j];
+                for (int i = 0; i < R; ++i)
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+                    for (int j = 0; j < R; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
             }
             __syncthreads();
         }
     }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int64_t m = m_lo + ty * 4 + i;
+    for (int i = 0; i < R; ++i) {
+        const int64_t m = m_lo + ty * R + i;
         if (m >= m_hi) continue;
         const int64_t orow = a.c_rows ? (int64_t)a.c_rows[m] : m;
         if ((uint64_t)orow >= (uint64_t)a.M) continue;  // only a launch that gave up leaves such rows
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int n = n0 + tx * 4 + j;
+        for (int j = 0; j < R; ++j) {
+            const int n = n0 + tx * R + j;
             if (n >= a.N) continue;
             float v = acc[i][j];
             if (a.bias) v += a.bias[n];
@@ -116,13 +135,29 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
     }
 }
 
-cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
-    const int n_tiles_n = (a.N + SG_N - 1) / SG_N;
-    int64_t m_tiles = (a.M + SG_M - 1) / SG_M;
+template <int TM>
+static int64_t simt_blocks(const SimtGemmArgs& a, int* n_tiles_n) {
+    *n_tiles_n = (a.N + TM - 1) / TM;
+    int64_t m_tiles = (a.M + TM - 1) / TM;
     if (a.offsets) m_tiles += a.E;  // each expert adds at most one ragged tile
-    const int64_t blocks = m_tiles * n_tiles_n;
-    if (blocks <= 0) return cudaSuccess;
-    simt_gemm_kernel<<<(unsigned)blocks, 256, 0, s>>>(a, n_tiles_n);
+    return m_tiles * *n_tiles_n;
+}
+
+cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
+    static int num_sms = 0;
+    if (!num_sms) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            num_sms = 1;
+    }
+    int n64 = 0, n32 = 0;
+    const int64_t b64 = simt_blocks<64>(a, &n64), b32 = simt_blocks<32>(a, &n32);
+    if (b64 <= 0) return cudaSuccess;
+    if (b64 < 2 * (int64_t)num_sms)  // too few 64-wide tiles to fill the GPU: 32-wide ones
+        simt_gemm_kernel<32><<<(unsigned)b32, 256, 0, s>>>(a, n32);
+    else
+        simt_gemm_kernel<64><<<(unsigned)b64, 256, 0, s>>>(a, n64);
     return cudaGetLastError();
 }
 
