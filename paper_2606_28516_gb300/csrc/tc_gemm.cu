@@ -19,6 +19,8 @@
 // expert offsets and chains two K segments into one accumulator: [t | z] x [U_r | W_e^res].
 // Every wait is bounded; on time-out the CTA records CLEARMOE_ETIMEOUT, drains its in-flight
 // copies and MMAs, frees TMEM and returns.
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -465,7 +467,43 @@ typedef CUresult (*PFN_encodeTiled_t)(CUtensorMap*, CUtensorMapDataType, cuuint3
                                       const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                       CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
+// Encoded maps are cached by (base, rows, cols, box rows), which determine them entirely: a forward
+// encodes up to ~20 maps, and the driver call costs microseconds each on the host.
+namespace {
+struct TmapEntry {
+    const void* base;
+    int64_t rows, cols;
+    int box_rows;
+    bool valid;
+    CUtensorMap map;
+};
+constexpr int TMAP_CACHE = 64;
+TmapEntry g_tmaps[TMAP_CACHE];
+int g_tmap_next = 0;
+std::mutex g_tmap_mu;
+}  // namespace
+
+static int encode_tmap_bf16_uncached(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows);
+
 int encode_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
+    std::lock_guard<std::mutex> lock(g_tmap_mu);
+    for (int i = 0; i < TMAP_CACHE; ++i) {
+        const TmapEntry& c = g_tmaps[i];
+        if (c.valid && c.base == base && c.rows == rows && c.cols == cols && c.box_rows == box_rows) {
+            *map = c.map;
+            return 0;
+        }
+    }
+    const int rc = encode_tmap_bf16_uncached(map, base, rows, cols, box_rows);
+    if (rc == 0) {
+        TmapEntry& c = g_tmaps[g_tmap_next];
+        c = TmapEntry{base, rows, cols, box_rows, true, *map};
+        g_tmap_next = (g_tmap_next + 1) % TMAP_CACHE;
+    }
+    return rc;
+}
+
+static int encode_tmap_bf16_uncached(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
     static PFN_encodeTiled_t fn = nullptr;
     if (!fn) {
         void* p = nullptr;
