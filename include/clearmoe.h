@@ -172,6 +172,14 @@ int clearmoe_ffn_forward_folded(clearmoe_layer* layer, const void* x, int64_t T,
                                 const void* b1, const void* const* W_comb,
                                 const clearmoe_router* router, int32_t E, void* out, void* stream);
 
+/* clearmoe_ffn_forward_folded with the deployment options of clearmoe_ffn_forward_ex (fc2 bias,
+ * class tokens on the dense path W2, the MLP router); opt may be NULL. Same errors as
+ * clearmoe_ffn_forward_ex. */
+int clearmoe_ffn_forward_folded_ex(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                                   const void* b1, const void* const* W_comb,
+                                   const clearmoe_router* router, int32_t E,
+                                   const clearmoe_ffn_options* opt, void* out, void* stream);
+
 /* The paper's own form of the shared basis (Phase 3 text: W_shared materialised before
  * inference): W_sh = U_r diag(S_r) Vh_r as one [d x H] row-major matrix in the layer dtype, formed
  * in fp32 (products in fp32, summed over k ascending) and rounded once. W_sh is a caller-owned
@@ -187,6 +195,13 @@ int clearmoe_materialize_basis(clearmoe_layer* layer, const void* U_r, const flo
 int clearmoe_ffn_forward_materialized(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
                                       const void* b1, const void* W_sh, const void* const* residual_e,
                                       const clearmoe_router* router, int32_t E, void* out, void* stream);
+
+/* clearmoe_ffn_forward_materialized with the deployment options of clearmoe_ffn_forward_ex; opt
+ * may be NULL. Same errors as clearmoe_ffn_forward_ex. */
+int clearmoe_ffn_forward_materialized_ex(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                                         const void* b1, const void* W_sh, const void* const* residual_e,
+                                         const clearmoe_router* router, int32_t E,
+                                         const clearmoe_ffn_options* opt, void* out, void* stream);
 
 /* The residual structure of Algorithm 2 exploited: its residual experts are scaled copies of one
  * matrix, W_e^res = s_e R with R = W2 - W_shared, so y_t = W_shared z_t + s_{a_t} R z_t =

@@ -63,6 +63,12 @@ _SIGS = {
                                 ctypes.POINTER(clearmoe_router), _I32, _I32,
                                 ctypes.POINTER(clearmoe_ffn_options), _P, _P],
     "clearmoe_materialize_basis": [_P, _P, _P, _P, _I32, _P, _P],
+    "clearmoe_ffn_forward_folded_ex": [_P, _P, _I64, _P, _P, ctypes.POINTER(ctypes.c_void_p),
+                                       ctypes.POINTER(clearmoe_router), _I32,
+                                       ctypes.POINTER(clearmoe_ffn_options), _P, _P],
+    "clearmoe_ffn_forward_materialized_ex": [_P, _P, _I64, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
+                                             ctypes.POINTER(clearmoe_router), _I32,
+                                             ctypes.POINTER(clearmoe_ffn_options), _P, _P],
     "clearmoe_ffn_forward_materialized": [_P, _P, _I64, _P, _P, _P, ctypes.POINTER(ctypes.c_void_p),
                                           ctypes.POINTER(clearmoe_router), _I32, _P, _P],
     "clearmoe_ffn_forward_scaled": [_P, _P, _I64, _P, _P, _P, _P, _P, _P, _P,
@@ -226,6 +232,37 @@ def clearmoe_ffn_forward_scaled(layer: int, x, W1, b1, U_r, S_r, Vh_r, R, s_e, W
                                              _ptr(S_r), _ptr(Vh_r), _ptr(R), _ptr(s_e), ctypes.byref(r),
                                              Wg.shape[0], S_r.shape[0], _ptr(out), _stream(stream)),
            "clearmoe_ffn_forward_scaled")
+
+
+def _options(b2, W2, cls_stride, mlp):
+    return clearmoe_ffn_options(_ptr(b2), int(cls_stride), _ptr(W2),
+                                ctypes.pointer(mlp) if mlp is not None else None)
+
+
+def clearmoe_ffn_forward_folded_ex(layer: int, x, W1, b1, W_comb, Wg, bg, out, b2=None, W2=None,
+                                   cls_stride: int = 0, mlp: clearmoe_mlp_router | None = None,
+                                   E: int | None = None, stream=None) -> None:
+    E = Wg.shape[0] if E is None else E
+    comb = (ctypes.c_void_p * E)(*[_ptr(W_comb[e]) for e in range(E)])
+    r = _router(Wg, bg) if Wg is not None else None
+    opt = _options(b2, W2, cls_stride, mlp)
+    _check(lib().clearmoe_ffn_forward_folded_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), comb,
+                                                ctypes.byref(r) if r else None, E, ctypes.byref(opt),
+                                                _ptr(out), _stream(stream)), "clearmoe_ffn_forward_folded_ex")
+
+
+def clearmoe_ffn_forward_materialized_ex(layer: int, x, W1, b1, W_sh, residual_e, Wg, bg, out, b2=None,
+                                         W2=None, cls_stride: int = 0,
+                                         mlp: clearmoe_mlp_router | None = None, E: int | None = None,
+                                         stream=None) -> None:
+    E = Wg.shape[0] if E is None else E
+    res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
+    r = _router(Wg, bg) if Wg is not None else None
+    opt = _options(b2, W2, cls_stride, mlp)
+    _check(lib().clearmoe_ffn_forward_materialized_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
+                                                      _ptr(W_sh), res, ctypes.byref(r) if r else None, E,
+                                                      ctypes.byref(opt), _ptr(out), _stream(stream)),
+           "clearmoe_ffn_forward_materialized_ex")
 
 
 def clearmoe_dense_ffn_forward(layer: int, x, W1, b1, W2, out, stream=None) -> None:

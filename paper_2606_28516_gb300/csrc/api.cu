@@ -112,6 +112,24 @@ int check_mlp(const clearmoe_layer* L, const clearmoe_mlp_router* m, int E) {
     return CLEARMOE_OK;
 }
 
+int check_router(const clearmoe_layer* L, const clearmoe_router* router, int E);
+
+// The router (linear, or the MLP router of the options) and the deployment options of a forward.
+int check_router_and_options(const clearmoe_layer* L, const clearmoe_router* router, const clearmoe_ffn_options* opt,
+                             int E) {
+    const int rc = (opt && opt->mlp_router) ? check_mlp(L, opt->mlp_router, E) : check_router(L, router, E);
+    if (rc) return rc;
+    if (opt) {
+        if (opt->cls_stride < 0 || opt->cls_stride > ((int64_t)1 << 30)) return CLEARMOE_EINVAL;
+        if (opt->b2 && misaligned(opt->b2)) return CLEARMOE_EINVAL;
+        if (opt->cls_stride > 0) {
+            if (!opt->W2 || misaligned(opt->W2)) return CLEARMOE_EINVAL;
+            if (E + 1 > CM_MAX_E) return CLEARMOE_EUNSUPPORTED;  // the dense path takes a group
+        }
+    }
+    return CLEARMOE_OK;
+}
+
 int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router,
              const clearmoe_mlp_router* mlp, int E, int64_t cls_stride, cudaStream_t s) {
     // the MLP router: its hidden layer first, then the routing kernel on it (fp32 tokens)
@@ -488,19 +506,7 @@ int clearmoe_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, const v
                             void* out, void* stream) {
     int rc = check_common(L, x, T);
     if (rc) return rc;
-    if (opt && opt->mlp_router)
-        rc = check_mlp(L, opt->mlp_router, E);
-    else
-        rc = check_router(L, router, E);
-    if (rc) return rc;
-    if (opt) {
-        if (opt->cls_stride < 0 || opt->cls_stride > ((int64_t)1 << 30)) return CLEARMOE_EINVAL;
-        if (opt->b2 && misaligned(opt->b2)) return CLEARMOE_EINVAL;
-        if (opt->cls_stride > 0) {
-            if (!opt->W2 || misaligned(opt->W2)) return CLEARMOE_EINVAL;
-            if (E + 1 > CM_MAX_E) return CLEARMOE_EUNSUPPORTED;  // the dense path takes a group
-        }
-    }
+    if ((rc = check_router_and_options(L, router, opt, E))) return rc;
     if (!W1 || !b1 || !U_r || !S_r || !Vh_r || !residual_e || !out) return CLEARMOE_EINVAL;
     const int d = L->desc.d, H = L->desc.hidden;
     if (r < 1 || r > L->desc.max_r || r > d || r > H) return CLEARMOE_EINVAL;
@@ -519,28 +525,41 @@ int clearmoe_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, const v
 int clearmoe_ffn_forward_folded(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
                                 const void* const* W_comb, const clearmoe_router* router, int32_t E, void* out,
                                 void* stream) {
+    return clearmoe_ffn_forward_folded_ex(L, x, T, W1, b1, W_comb, router, E, nullptr, out, stream);
+}
+
+int clearmoe_ffn_forward_folded_ex(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                                   const void* const* W_comb, const clearmoe_router* router, int32_t E,
+                                   const clearmoe_ffn_options* opt, void* out, void* stream) {
     int rc = check_common(L, x, T);
     if (rc) return rc;
-    if ((rc = check_router(L, router, E))) return rc;
+    if ((rc = check_router_and_options(L, router, opt, E))) return rc;
     if (!W1 || !b1 || !W_comb || !out) return CLEARMOE_EINVAL;
     for (int e = 0; e < E; ++e)
         if (!W_comb[e] || misaligned(W_comb[e])) return CLEARMOE_EINVAL;
     if (misaligned(W1) || misaligned(b1) || misaligned(out)) return CLEARMOE_EINVAL;
-    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, nullptr, W_comb, router, E, 0, nullptr, out,
+    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, nullptr, W_comb, router, E, 0, opt, out,
                     static_cast<cudaStream_t>(stream));
 }
 
 int clearmoe_ffn_forward_materialized(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
                                       const void* W_sh, const void* const* residual_e, const clearmoe_router* router,
                                       int32_t E, void* out, void* stream) {
+    return clearmoe_ffn_forward_materialized_ex(L, x, T, W1, b1, W_sh, residual_e, router, E, nullptr, out, stream);
+}
+
+int clearmoe_ffn_forward_materialized_ex(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
+                                         const void* b1, const void* W_sh, const void* const* residual_e,
+                                         const clearmoe_router* router, int32_t E, const clearmoe_ffn_options* opt,
+                                         void* out, void* stream) {
     int rc = check_common(L, x, T);
     if (rc) return rc;
-    if ((rc = check_router(L, router, E))) return rc;
+    if ((rc = check_router_and_options(L, router, opt, E))) return rc;
     if (!W1 || !b1 || !W_sh || !residual_e || !out) return CLEARMOE_EINVAL;
     for (int e = 0; e < E; ++e)
         if (!residual_e[e] || misaligned(residual_e[e])) return CLEARMOE_EINVAL;
     if (misaligned(W1) || misaligned(b1) || misaligned(W_sh) || misaligned(out)) return CLEARMOE_EINVAL;
-    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, W_sh, residual_e, router, E, 0, nullptr, out,
+    return ffn_impl(L, x, T, W1, b1, nullptr, nullptr, nullptr, W_sh, residual_e, router, E, 0, opt, out,
                     static_cast<cudaStream_t>(stream));
 }
 

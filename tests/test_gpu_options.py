@@ -190,3 +190,35 @@ def test_option_errors_enqueue_nothing(workload):
             cm.clearmoe_ffn_forward_ex(h.h, x, D["W1"], D["b1"], D["U"], D["S"], D["Vh"], res, Wg, bg,
                                        out, W2=D["W2"], cls_stride=CLS)
         assert ei.value.code == cm.EUNSUPPORTED
+
+
+@pytest.mark.parametrize("shape", [synth.DEIT_SMALL_BF16, synth.DEIT_BASE_BF16])
+@pytest.mark.parametrize("form", ["folded", "materialized"])
+def test_options_on_folded_and_materialized_forms(workload, shape, form):
+    """Class tokens and b2 with the basis folded into the experts or materialised, against Eq. 2
+    (the oracle's exact W_shared) with the same options: the whole layer at DeiT-S, sampled rows
+    plus every class row at DeiT-B."""
+    L = workload(shape)
+    s = L["shape"]
+    D = synth.to_torch(L)
+    with handle_for(L) as h:
+        out = torch.full_like(D["x"], float("nan"))
+        kw = dict(b2=D["b2"], W2=D["W2"], cls_stride=CLS)
+        if form == "folded":
+            W = torch.empty_like(D["residuals"])
+            cm.clearmoe_fold_basis(h.h, D["U"], D["S"], D["Vh"], D["residuals"], W)
+            cm.clearmoe_ffn_forward_folded_ex(h.h, D["x"], D["W1"], D["b1"], W, D["Wg"], D["bg"], out, **kw)
+        else:
+            W = torch.empty(s.d, s.H, device="cuda", dtype=D["x"].dtype)
+            cm.clearmoe_materialize_basis(h.h, D["U"], D["S"], D["Vh"], W)
+            cm.clearmoe_ffn_forward_materialized_ex(h.h, D["x"], D["W1"], D["b1"], W, D["residuals"], D["Wg"],
+                                                    D["bg"], out, **kw)
+        gr = get_routing(h, s.T, s.E + 1)
+        assert cm.clearmoe_layer_status(h.h) == 0
+    _check_routing(gr, L, CLS, s.T)
+    rows = np.arange(s.T) if s.T <= 20000 else np.unique(
+        np.concatenate([sample_rows(gr, s.T), np.arange(0, s.T, CLS)]))
+    y = _oracle(L, rows, gr["a"], CLS)
+    got = out if len(rows) == s.T else out[torch.from_numpy(rows).cuda()]
+    err = out_error(got, y, "bf16")
+    assert err <= tol("bf16"), f"{form} {s.name}: {err:.3e}"
