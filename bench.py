@@ -41,13 +41,13 @@ KERNEL_OF_STAGE = {"route": "cm::route_kernel<1, 1>",
                    "basis": "cm::tc_gemm2_kernel<128, 0> (2-SM dense, column scale)",
                    "grouped": "cm::tc_gemm2_kernel<256, 2> (2-SM grouped, rows stored at perm[slot])"}
 # DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from the committed ncu
-# capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel sources
-# it was taken on; a different hash means the kernels changed and the figure is void.
+# capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel's sources
+# it was taken on (source_hash); a different hash means the kernel changed and the figure is void.
 TRAFFIC = {
-    "route": {"bytes": 78.551296e6, "src": "67c2c10bb509ef2c"},
-    "fc1_gelu": {"bytes": 338.262016e6, "src": "67c2c10bb509ef2c"},
-    "basis": {"bytes": 315.866368e6, "src": "67c2c10bb509ef2c"},
-    "grouped": {"bytes": 430.195200e6, "src": "67c2c10bb509ef2c"},
+    "route": {"bytes": 78.551296e6, "src": "0ec5201dfa545d93"},
+    "fc1_gelu": {"bytes": 338.262016e6, "src": "762f4db4a3774b3f"},
+    "basis": {"bytes": 315.866368e6, "src": "762f4db4a3774b3f"},
+    "grouped": {"bytes": 430.195200e6, "src": "762f4db4a3774b3f"},
 }
 
 
@@ -116,10 +116,18 @@ def layer_roofline_s(s, pk):
     return max(flops / (pk["bf16_tflops_sustained"] * 1e12), bytes_ / (pk["hbm_gbs"] * 1e9))
 
 
-def source_hash():
+KERNEL_SOURCES = {"route": ("route.cu", "common.cuh", "internal.h"),
+                  "fc1_gelu": ("tc_gemm2.cu", "common.cuh", "internal.h"),
+                  "basis": ("tc_gemm2.cu", "common.cuh", "internal.h"),
+                  "grouped": ("tc_gemm2.cu", "common.cuh", "internal.h")}
+
+
+def source_hash(stage):
+    """Hash of the sources the stage's kernel is compiled from: a capture's traffic figure holds
+    only while they are unchanged."""
     h = hashlib.sha256()
-    for f in sorted((ROOT / "paper_2606_28516_gb300" / "csrc").glob("*")):
-        h.update(f.read_bytes())
+    for f in KERNEL_SOURCES[stage]:
+        h.update((ROOT / "paper_2606_28516_gb300" / "csrc" / f).read_bytes())
     return h.hexdigest()[:16]
 
 
@@ -665,7 +673,7 @@ def main():
                 "unit": "TFLOP/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     tr = TRAFFIC.get(dom)
-    roof["traffic"] = tr["bytes"] if tr and tr["src"] == source_hash() else None
+    roof["traffic"] = tr["bytes"] if tr and tr["src"] == source_hash(dom) else None
     roof["kernel"] = KERNEL_OF_STAGE[dom]
     roof["peak_source"] = f"{pk_src} ({'sustained bf16' if roof['bound'] == 'tensor' else 'HBM copy'})"
 
@@ -682,7 +690,7 @@ def main():
 
     for st in STAGES:  # per-kernel DRAM traffic where the committed capture still applies
         t = TRAFFIC.get(st)
-        per_stage[st]["traffic"] = t["bytes"] if t and t["src"] == source_hash() else None
+        per_stage[st]["traffic"] = t["bytes"] if t and t["src"] == source_hash(st) else None
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
