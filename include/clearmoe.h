@@ -19,8 +19,10 @@
  *     return; they never synchronise, except clearmoe_layer_status and clearmoe_layer_destroy.
  *   - One handle may be used by one stream at a time: its workspace holds the hidden states and
  *     routing of the last forward.
- *   - Arguments are validated on the host first; on any error nothing is enqueued and the
- *     outputs are untouched. Return values are clearmoe_status codes.
+ *   - Arguments are validated on the host first; on a validation error (EINVAL, EUNSUPPORTED)
+ *     nothing is enqueued and the outputs are untouched. CLEARMOE_ECUDA can also come from a
+ *     launch after earlier kernels of the same call were enqueued; the outputs are then
+ *     undefined. Return values are clearmoe_status codes.
  *   - Device-side waits are bounded. A wait that runs out writes CLEARMOE_ETIMEOUT into the
  *     handle's device status word (read by clearmoe_layer_status); the outputs of that call are
  *     then undefined, and the handle stays usable.
@@ -50,8 +52,9 @@ typedef enum { CLEARMOE_F32 = 0, CLEARMOE_BF16 = 1 } clearmoe_dtype;
  *   CLEARMOE_BF16: bf16 storage, fp32 accumulation on the tcgen05 tensor cores; z, the shared-
  *                  basis coefficients t = diag(S_r) Vh_r z and out are stored in bf16.
  *   CLEARMOE_F32:  fp32 storage and fp32 FMA on the CUDA cores (exact-fp32 path).
- * Tiling limits (else CLEARMOE_EUNSUPPORTED): bf16 needs d % 64 == 0, hidden % 64 == 0 and
- * r % 16 == 0 per call; fp32 needs d % 4 == 0 and hidden % 4 == 0. max_E <= 16, max_r <= 256. */
+ * Tiling limits (else CLEARMOE_EUNSUPPORTED): bf16 needs d % 64 == 0, d <= 1024, hidden % 64 == 0
+ * and r % 16 == 0 per call; fp32 needs d % 4 == 0, d <= 512, hidden % 4 == 0 and r % 4 == 0.
+ * max_E <= 16, max_r <= 256, max_tokens <= 2^30. */
 typedef struct {
     int64_t max_tokens;
     int32_t d;
