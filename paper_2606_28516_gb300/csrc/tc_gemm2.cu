@@ -421,7 +421,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         const int q = warp & 3;  // a warp reads the TMEM lanes of its index mod 4
         const int c_lo = (warp >> 2) * WCOLS;
         unsigned char* wstg = stg + warp * 32 * STG_ROW;
-        constexpr int LPR = SW / 8, RPP = 32 / LPR;
+        // Staging by half warps: the 16 rows of lanes 16 h .. 16 h + 15 as 64-byte rows (a 32-column
+        // chunk), 16-byte piece j of row r at piece j ^ ((r >> 1) & 3) (conflict-free for the
+        // row-wise writes and the 4-lanes-per-row reads); each store instruction then writes
+        // 8 rows x 64 contiguous bytes.
+        static_assert(CW == 32 && 16 * 64 == 32 * STG_ROW, "a half warp's 64-byte rows fill the warp's staging");
         const uint32_t tempty_leader0 = map_to_rank(tempty_bar(0), 0);
         int acc = 0;
         uint32_t aph = 0;
@@ -450,13 +454,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                 }
             }
             const float rsc = (a.group_scale && mrow < t.hi) ? tc_row_scale(a, mrow) : 1.f;
-            // this lane stores rows p * RPP + lane / LPR of the warp's 32 (p < LPR), 16-byte chunk
-            // lane % LPR: their destinations, once per tile
-            uint16_t* dst_row[LPR];
+            // this lane stores warp rows 16 h + 8 p + lane / 4 (h, p < 2), 16-byte piece lane % 4 of
+            // each 32-column chunk: their destinations, once per tile
+            uint16_t* dst_row[4];
 #pragma unroll
-            for (int p = 0; p < LPR; ++p) {
-                const int64_t o = __shfl_sync(0xffffffffu, orow, p * RPP + lane / LPR);
-                dst_row[p] = o >= 0 ? static_cast<uint16_t*>(a.C) + o * a.ldc + t.n0 + (lane % LPR) * 8 : nullptr;
+            for (int hp = 0; hp < 4; ++hp) {
+                const int64_t o = __shfl_sync(0xffffffffu, orow, 8 * hp + lane / 4);
+                dst_row[hp] = o >= 0 ? static_cast<uint16_t*>(a.C) + o * a.ldc + t.n0 + (lane % 4) * 8 : nullptr;
             }
             for (int c = c_lo; c < c_lo + WCOLS; c += CW) {
                 uint32_t v[CW];
@@ -535,22 +539,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                     continue;
                 }
 #pragma unroll
-                for (int s0 = 0; s0 < CW; s0 += SW) {
-                    unsigned char* dst = wstg + lane * STG_ROW;
+                for (int h = 0; h < 2; ++h) {
+                    if ((lane >> 4) == h) {
+                        const int rw = lane & 15;
+                        unsigned char* dst = wstg + rw * 64;
 #pragma unroll
-                    for (int j8 = 0; j8 < SW / 8; ++j8) {
-                        const float* g = f + s0 + 8 * j8;
-                        *reinterpret_cast<uint4*>(dst + ((j8 ^ ((lane >> 2) & 1)) << 4)) =
-                            make_uint4(pack_bf16(g[0], g[1]), pack_bf16(g[2], g[3]), pack_bf16(g[4], g[5]),
-                                       pack_bf16(g[6], g[7]));
+                        for (int j8 = 0; j8 < 4; ++j8) {
+                            const float* g = f + 8 * j8;
+                            *reinterpret_cast<uint4*>(dst + ((j8 ^ ((rw >> 1) & 3)) << 4)) =
+                                make_uint4(pack_bf16(g[0], g[1]), pack_bf16(g[2], g[3]), pack_bf16(g[4], g[5]),
+                                           pack_bf16(g[6], g[7]));
+                        }
                     }
                     __syncwarp();
 #pragma unroll
-                    for (int p = 0; p < LPR; ++p) {
-                        const int rr = p * RPP + lane / LPR;
-                        const int ch = (lane % LPR) ^ ((rr >> 2) & 1);
-                        const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * STG_ROW + ch * 16);
-                        if (dst_row[p]) *reinterpret_cast<uint4*>(dst_row[p] + (c + s0)) = val;
+                    for (int p = 0; p < 2; ++p) {
+                        const int rr = 8 * p + lane / 4;  // row of the half
+                        const int ch = (lane % 4) ^ ((rr >> 1) & 3);
+                        const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * 64 + ch * 16);
+                        if (dst_row[2 * h + p]) *reinterpret_cast<uint4*>(dst_row[2 * h + p] + c) = val;
                     }
                     __syncwarp();
                 }
