@@ -220,9 +220,9 @@ def run_reference(args):
         shape = (synth.deit_small_zipf(4, 64) if args.workload == "deit_small_zipf_sweep"
                  else synth.DEIT_BASE_BF16.with_(T=synth.VIT_BASE_STACK12.T))
     L = synth.make_layer(shape)
-    # per-step sample sized so that warmup + steps take about a minute of CPU time in total
-    probe, _, _ = oracle_rate(L, budget_s=2.0, chunk=256, max_tokens=512)
-    per_step = max(16, min(4096, int(probe * 60.0 / max(1, args.steps + args.warmup))))
+    # per-step sample sized so that warmup + steps take about --ref-budget-s of CPU time in total
+    probe, _, _ = oracle_rate(L, budget_s=min(2.0, args.ref_budget_s / 4), chunk=256, max_tokens=512)
+    per_step = max(16, min(4096, int(probe * args.ref_budget_s / max(1, args.steps + args.warmup))))
     for _ in range(args.warmup):
         oracle_rate(L, budget_s=1e9, chunk=per_step, max_tokens=per_step, warm=False)
     t0 = time.perf_counter()
@@ -456,6 +456,8 @@ def main():
     ap.add_argument("--workload", default="deit_base_bf16", choices=sorted(workloads()))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--ref-budget-s", type=float, default=60.0,
+                    help="--impl reference: CPU seconds the oracle's warm-up and timed steps take in total")
     ap.add_argument("--no-variants", action="store_true",
                     help="skip the variant timings (folded, materialised, class tokens, MLP router, one residual)")
     args = ap.parse_args()
