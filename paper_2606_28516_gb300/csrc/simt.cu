@@ -7,7 +7,8 @@
 // with an optional row gather of A0 (fc1 on tokens in expert order), an optional second K
 // segment with a per-expert B (the grouped residual GEMM, Algorithm 3 step 5; with dense_last the
 // last group is the class tokens' dense path, second segment only), an epilogue of
-// bias, GELU and per-column scale, and an optional row scatter of C (the unshuffle, step 6).
+// bias, GELU or ReLU, per-column scale and per-row scale, and an optional row scatter of C (the
+// unshuffle, step 6).
 #include "common.cuh"
 #include "internal.h"
 
