@@ -35,6 +35,9 @@ sys.path.insert(0, str(ROOT))
 METRIC = ("CLEAR-MoE FFN tokens/sec/layer (1×GB300) + % HBM peak (dispatch), "
           "% tensor peak (GEMMs)")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# the GB300's nominal figures (HBM3e ~7.9 TB/s; dense bf16 2.25 PFLOP/s), reported beside the
+# measured peaks for context
+NOMINAL_PEAKS = {"hbm_gbs": 7900.0, "bf16_tflops": 2250.0}
 STAGES = ("route", "fc1_gelu", "basis", "grouped")
 KERNEL_OF_STAGE = {"route": "cm::route_kernel<1, 1>",
                    "fc1_gelu": "cm::tc_gemm2_kernel<256, 0> (2-SM dense, rows stored at their routing slots)",
@@ -684,11 +687,13 @@ def main():
         d_s = avg[st] / 1e3
         if "bytes" in work[st]:
             g = work[st]["bytes"] / d_s / 1e9
-            per_stage[st] = {"us": avg[st] * 1e3, "GB_s": g, "hbm_frac": g / pk["hbm_gbs"]}
+            per_stage[st] = {"us": avg[st] * 1e3, "GB_s": g, "hbm_frac": g / pk["hbm_gbs"],
+                             "hbm_frac_nominal": g / NOMINAL_PEAKS["hbm_gbs"]}
         else:
             tf = work[st]["flops"] / d_s / 1e12
             per_stage[st] = {"us": avg[st] * 1e3, "TFLOP_s": tf,
-                             "tensor_frac": tf / pk["bf16_tflops_sustained"]}
+                             "tensor_frac": tf / pk["bf16_tflops_sustained"],
+                             "tensor_frac_nominal": tf / NOMINAL_PEAKS["bf16_tflops"]}
 
     for st in STAGES:  # per-kernel DRAM traffic where the committed capture still applies
         t = TRAFFIC.get(st)
@@ -722,6 +727,9 @@ def main():
         "stage_timing": f"separate pass of {Ks} steps with an event between consecutive kernels "
                         "(which also cancels their programmatic launch overlap)",
         "layer_roofline_frac": layer_roofline_s(s, pk) / (mean_step / 1e3),
+        "layer_roofline_frac_nominal": layer_roofline_s(
+            s, {"bf16_tflops_sustained": NOMINAL_PEAKS["bf16_tflops"], "hbm_gbs": NOMINAL_PEAKS["hbm_gbs"]})
+        / (mean_step / 1e3),
         "dense_ffn": {"value": dense_value, "unit": "tokens/s",
                       "ms_per_step": statistics.mean(dense_ms)},
         "folded": folded,
