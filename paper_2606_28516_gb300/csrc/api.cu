@@ -474,10 +474,11 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         g3.dense_last = 1;
     }
     g3.out_bias = b2;
-    // right after the 2-SM basis kernel (which releases it only once fc1 has completed) the grouped
-    // GEMM starts its z segments at once and waits for the basis only before its first t segment;
-    // with no routed rows no basis kernel runs, and fc1 (which releases early) precedes it
-    if (factored && cm::tc2_pick_bn(cm::TC_DENSE, r) && T - n_cls > 0) g3.pdl_wait_role = 2;
+    // right after the basis kernel (which releases it only once fc1 has completed) the grouped GEMM
+    // starts its z segments at once, on the SMs the basis leaves idle, and waits for the basis only
+    // before its first t segment; with no routed rows no basis kernel runs, and fc1 (which releases
+    // early) precedes it
+    if (factored && T - n_cls > 0) g3.pdl_wait_role = 2;
     g3.mode = cm::TC_GROUPED;
     g3.epi = cm::TC_EPI_SCATTER;
     g3.M = T;

@@ -83,7 +83,7 @@ __device__ __forceinline__ TileInfo decode_tile(const TcGemmArgs& a, int tile, i
 template <int BN, int MODE>
 __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THREADS_TMA, 1)
     tc_gemm_kernel(const __grid_constant__ TcGemmArgs a) {
-    pdl_launch_dependents();
+    if (!a.pdl_trigger_late) pdl_launch_dependents();
     using C = TcCfg<BN>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
@@ -127,6 +127,7 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
     tc_fence_after();
     // everything above overlaps the predecessor kernel; from here on its results are read
     pdl_wait();
+    if (a.pdl_trigger_late) pdl_launch_dependents();
     if (MODE == TC_GROUPED) {
         if (threadIdx.x == 0) {
             int acc = 0;
