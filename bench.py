@@ -361,9 +361,23 @@ def run_stack(args):
     buf = [torch.empty_like(x0) for _ in range(2)]
     y = torch.empty_like(x0)
 
-    def stack_pass(x_in, folded=False):
+    def stack_pass(x_in, folded=False, ln_fold=False):
+        """ln_fold: each LayerNorm folded into the next sublayer's router and fc1 (that sublayer is
+        given y itself); the last one still runs, so that both forms return LN(y_11)."""
         x = x_in
         for l, G in enumerate(layers):
+            if ln_fold:
+                ln, yl = l > 0, buf[l & 1]
+                if G["moe"] and folded:
+                    cm.clearmoe_ffn_forward_folded_ex(h, x, G["W1"], G["b1"], G["W_comb"], G["Wg"], G["bg"], yl,
+                                                      input_layernorm=ln)
+                elif G["moe"]:
+                    cm.clearmoe_ffn_forward_ex(h, x, G["W1"], G["b1"], G["U"], G["S"], G["Vh"], G["residuals"],
+                                               G["Wg"], G["bg"], yl, input_layernorm=ln)
+                else:
+                    cm.clearmoe_dense_ffn_forward_opt(h, x, G["W1"], G["b1"], G["W2"], yl, input_layernorm=ln)
+                x = yl
+                continue
             if G["moe"] and folded:
                 cm.clearmoe_ffn_forward_folded(h, x, G["W1"], G["b1"], G["W_comb"], G["Wg"], G["bg"], y)
             elif G["moe"]:
@@ -373,11 +387,14 @@ def run_stack(args):
                 cm.clearmoe_dense_ffn_forward(h, x, G["W1"], G["b1"], G["W2"], y)
             x = buf[l & 1]
             cm.clearmoe_layer_norm(h, y, x)
+        if ln_fold:
+            cm.clearmoe_layer_norm(h, x, y)
+            x = y
         return x
 
-    def timed(K, folded=False):
+    def timed(K, folded=False, ln_fold=False):
         for _ in range(args.warmup):
-            stack_pass(x0, folded)
+            stack_pass(x0, folded, ln_fold)
         torch.cuda.synchronize()
         assert cm.clearmoe_layer_status(h) == 0
         ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
@@ -386,7 +403,7 @@ def run_stack(args):
         torch.cuda.synchronize()
         for k in range(K):
             ev[k][0].record()
-            stack_pass(x0, folded)
+            stack_pass(x0, folded, ln_fold)
             ev[k][1].record()
         torch.cuda.synchronize()
         assert cm.clearmoe_layer_status(h) == 0
@@ -403,6 +420,8 @@ def run_stack(args):
             G["W_comb"] = torch.empty_like(G["residuals"])
             cm.clearmoe_fold_basis(h, G["U"], G["S"], G["Vh"], G["residuals"], G["W_comb"])
     ms_f = timed(K, folded=True)
+    ms_ln = timed(K, ln_fold=True)
+    ms_fln = timed(K, folded=True, ln_fold=True)
     # end to end: the tokens copied in from pinned host memory, the last output copied back
     xh = x0.cpu().pin_memory()
     outh = torch.empty(x0.shape, dtype=x0.dtype).pin_memory()
@@ -443,6 +462,10 @@ def run_stack(args):
         "cpu_baseline": cpu,
         "clocks": clk.summary(),
         "folded": {"value": whole_job_rate(T, world, 1, ms_f), "unit": "tokens/s", "ms_per_step": ms_f},
+        # the LayerNorm between sublayers folded into the next one's router and fc1 (never written)
+        "layernorm_folded": {"value": whole_job_rate(T, world, 1, ms_ln), "unit": "tokens/s", "ms_per_step": ms_ln},
+        "folded_and_layernorm_folded": {"value": whole_job_rate(T, world, 1, ms_fln), "unit": "tokens/s",
+                                        "ms_per_step": ms_fln},
     }
     if rank == 0:
         print(json.dumps(line), flush=True)

@@ -140,12 +140,20 @@ int clearmoe_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const 
  *              idx = E, counts[E] = n_cls = ceil(T / cls_stride), slots [T - n_cls, T) in token
  *              order. Requires W2 and E + 1 <= 16 (EUNSUPPORTED otherwise). 0: every token routed.
  *  W2          the layer's dense fc2 [d x H] row-major (device), read for class tokens only.
- *  mlp_router  the MLP router in place of the linear one (see clearmoe_mlp_router). */
+ *  mlp_router  the MLP router in place of the linear one (see clearmoe_mlp_router).
+ *  input_layernorm  non-zero: x is the un-normalised residual stream y of a ViT block, and the
+ *              sublayer's input is its per-token LayerNorm without affine, LN(y) = (y - mean) /
+ *              sqrt(biased variance + 1e-6), as clearmoe_layer_norm computes it (a pretrained
+ *              block's LN affine folds into W1, b1 and the router offline). LN(y) is never
+ *              written: one launch forms (mean, rstd) per token and the row sums c = W 1 of W1 and
+ *              of the router's first matrix (W_g, or the MLP router's W_in), and the router and fc1
+ *              use W LN(y) = rstd (W y - mean c) on their fp32 accumulators. 0: x is the input. */
 typedef struct {
     const void* b2;
     int64_t cls_stride;
     const void* W2;
     const clearmoe_mlp_router* mlp_router; /* non-NULL: routes with it (router may then be NULL) */
+    int32_t input_layernorm;
 } clearmoe_ffn_options;
 
 /* clearmoe_ffn_forward with deployment options (opt may be NULL: then identical to it). With
@@ -231,6 +239,13 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, 
 int clearmoe_dense_ffn_forward_ex(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
                                   const void* b1, const void* W2, const void* b2, void* out,
                                   void* stream);
+
+/* The dense FFN with the options of clearmoe_ffn_forward_ex that apply to it: b2 (as
+ * clearmoe_dense_ffn_forward_ex) and input_layernorm (x is y; LN(y) folded into fc1 as there).
+ * opt may be NULL. EINVAL for cls_stride != 0 or a non-NULL mlp_router; opt->W2 is not read. */
+int clearmoe_dense_ffn_forward_opt(clearmoe_layer* layer, const void* x, int64_t T, const void* W1,
+                                   const void* b1, const void* W2, const clearmoe_ffn_options* opt,
+                                   void* out, void* stream);
 
 /* Per-token LayerNorm without affine between stacked sublayers: x_out = (y - mean(y)) /
  * sqrt(var(y) + 1e-6), biased variance, fp32 statistics; y and x_out [T x d] in the layer's

@@ -39,7 +39,7 @@ class clearmoe_mlp_router(ctypes.Structure):
 
 class clearmoe_ffn_options(ctypes.Structure):
     _fields_ = [("b2", ctypes.c_void_p), ("cls_stride", ctypes.c_int64), ("W2", ctypes.c_void_p),
-                ("mlp_router", ctypes.POINTER(clearmoe_mlp_router))]
+                ("mlp_router", ctypes.POINTER(clearmoe_mlp_router)), ("input_layernorm", ctypes.c_int32)]
 
 
 ACT_RELU, ACT_GELU = 0, 1
@@ -75,6 +75,7 @@ _SIGS = {
                                     ctypes.POINTER(clearmoe_router), _I32, _I32, _P, _P],
     "clearmoe_dense_ffn_forward": [_P, _P, _I64, _P, _P, _P, _P, _P],
     "clearmoe_dense_ffn_forward_ex": [_P, _P, _I64, _P, _P, _P, _P, _P, _P],
+    "clearmoe_dense_ffn_forward_opt": [_P, _P, _I64, _P, _P, _P, ctypes.POINTER(clearmoe_ffn_options), _P, _P],
     "clearmoe_layer_norm": [_P, _P, _I64, _P, _P],
     "clearmoe_get_routing": [_P, _P, _P, _P, _P, _P],
     "clearmoe_layer_status": [_P],
@@ -178,14 +179,14 @@ def clearmoe_ffn_forward(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, 
 
 def clearmoe_ffn_forward_ex(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, bg, out,
                             b2=None, W2=None, cls_stride: int = 0, mlp: clearmoe_mlp_router | None = None,
-                            E: int | None = None, stream=None) -> None:
+                            E: int | None = None, input_layernorm: bool = False, stream=None) -> None:
     """clearmoe_ffn_forward with fc2's bias b2, class tokens (every cls_stride-th token from token 0)
-    on the dense path W2, and the MLP router `mlp` (then Wg, bg may be None and E is given)."""
+    on the dense path W2, the MLP router `mlp` (then Wg, bg may be None and E is given), and
+    input_layernorm (x is the un-normalised stream y; the layer's input is LN(y))."""
     E = Wg.shape[0] if E is None else E
     res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
     r = _router(Wg, bg) if Wg is not None else None
-    opt = clearmoe_ffn_options(_ptr(b2), int(cls_stride), _ptr(W2),
-                               ctypes.pointer(mlp) if mlp is not None else None)
+    opt = _options(b2, W2, cls_stride, mlp, input_layernorm)
     _check(lib().clearmoe_ffn_forward_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), _ptr(U_r),
                                          _ptr(S_r), _ptr(Vh_r), res, ctypes.byref(r) if r else None, E,
                                          S_r.shape[0], ctypes.byref(opt), _ptr(out),
@@ -234,18 +235,18 @@ def clearmoe_ffn_forward_scaled(layer: int, x, W1, b1, U_r, S_r, Vh_r, R, s_e, W
            "clearmoe_ffn_forward_scaled")
 
 
-def _options(b2, W2, cls_stride, mlp):
+def _options(b2, W2, cls_stride, mlp, input_layernorm=False):
     return clearmoe_ffn_options(_ptr(b2), int(cls_stride), _ptr(W2),
-                                ctypes.pointer(mlp) if mlp is not None else None)
+                                ctypes.pointer(mlp) if mlp is not None else None, int(bool(input_layernorm)))
 
 
 def clearmoe_ffn_forward_folded_ex(layer: int, x, W1, b1, W_comb, Wg, bg, out, b2=None, W2=None,
                                    cls_stride: int = 0, mlp: clearmoe_mlp_router | None = None,
-                                   E: int | None = None, stream=None) -> None:
+                                   E: int | None = None, input_layernorm: bool = False, stream=None) -> None:
     E = Wg.shape[0] if E is None else E
     comb = (ctypes.c_void_p * E)(*[_ptr(W_comb[e]) for e in range(E)])
     r = _router(Wg, bg) if Wg is not None else None
-    opt = _options(b2, W2, cls_stride, mlp)
+    opt = _options(b2, W2, cls_stride, mlp, input_layernorm)
     _check(lib().clearmoe_ffn_forward_folded_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), comb,
                                                 ctypes.byref(r) if r else None, E, ctypes.byref(opt),
                                                 _ptr(out), _stream(stream)), "clearmoe_ffn_forward_folded_ex")
@@ -254,11 +255,11 @@ def clearmoe_ffn_forward_folded_ex(layer: int, x, W1, b1, W_comb, Wg, bg, out, b
 def clearmoe_ffn_forward_materialized_ex(layer: int, x, W1, b1, W_sh, residual_e, Wg, bg, out, b2=None,
                                          W2=None, cls_stride: int = 0,
                                          mlp: clearmoe_mlp_router | None = None, E: int | None = None,
-                                         stream=None) -> None:
+                                         input_layernorm: bool = False, stream=None) -> None:
     E = Wg.shape[0] if E is None else E
     res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
     r = _router(Wg, bg) if Wg is not None else None
-    opt = _options(b2, W2, cls_stride, mlp)
+    opt = _options(b2, W2, cls_stride, mlp, input_layernorm)
     _check(lib().clearmoe_ffn_forward_materialized_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
                                                       _ptr(W_sh), res, ctypes.byref(r) if r else None, E,
                                                       ctypes.byref(opt), _ptr(out), _stream(stream)),
@@ -275,6 +276,15 @@ def clearmoe_dense_ffn_forward_ex(layer: int, x, W1, b1, W2, b2, out, stream=Non
     _check(lib().clearmoe_dense_ffn_forward_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
                                                _ptr(W2), _ptr(b2), _ptr(out), _stream(stream)),
            "clearmoe_dense_ffn_forward_ex")
+
+
+def clearmoe_dense_ffn_forward_opt(layer: int, x, W1, b1, W2, out, b2=None, input_layernorm: bool = False,
+                                   stream=None) -> None:
+    """The dense FFN with fc2's bias b2 and input_layernorm (x is y; the input is LN(y))."""
+    opt = _options(b2, None, 0, None, input_layernorm)
+    _check(lib().clearmoe_dense_ffn_forward_opt(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), _ptr(W2),
+                                                ctypes.byref(opt), _ptr(out), _stream(stream)),
+           "clearmoe_dense_ffn_forward_opt")
 
 
 def clearmoe_layer_norm(layer: int, y, x_out, stream=None) -> None:

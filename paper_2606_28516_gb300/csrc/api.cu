@@ -23,6 +23,8 @@ struct clearmoe_layer {
     int32_t* cta_counts;  // [route_max_ctas x CM_MAX_E] the routing kernel's per-range histograms
     int32_t* tinfo;       // [max_tokens] per token: expert | rank within its routing range << 8
     int32_t* status;
+    float2* ln_stats;  // [max_tokens]  (mean, rstd) per token when the input LayerNorm is folded
+    float* ln_sums;    // [2 hidden + CM_MAX_E]  row sums of W1, then of the router's first matrix
     int64_t wait_limit_ns;
     int32_t phantom;  // fault injection: > 0 makes the routing withhold one stage copy
     cm::RouteArgs rt;  // the last routing launch (its consumers reuse the shape)
@@ -47,7 +49,8 @@ int cuda_fail(cudaError_t e) {
 }
 
 void free_ws(clearmoe_layer* L) {
-    void* ptrs[] = {L->z, L->t, L->idx, L->perm, L->inv, L->counts, L->offsets, L->cta_counts, L->tinfo, L->status};
+    void* ptrs[] = {L->z,     L->t,          L->idx,   L->perm,   L->inv,     L->counts,
+                    L->offsets, L->cta_counts, L->tinfo, L->status, L->ln_stats, L->ln_sums};
     for (void* p : ptrs)
         if (p) cudaFree(p);
 }
@@ -62,8 +65,11 @@ int check_common(const clearmoe_layer* L, const void* x, int64_t T) {
 // The MLP router's hidden layer h = act(W_in x + b_in) [T x hidden], fp32, into the hidden-state
 // workspace (free until fc1 runs): the tensor-core GEMM with an fp32-store epilogue, or the fp32
 // SIMT GEMM on the fp32 layer.
-int mlp_hidden(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_mlp_router* m, cudaStream_t s) {
+// ln: x is the un-normalised stream; its LayerNorm is folded in (stats and W_in's row sums from ln_prep)
+int mlp_hidden(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_mlp_router* m, bool ln, cudaStream_t s) {
     const int d = L->desc.d, nh = m->hidden;
+    const float2* lns = ln ? L->ln_stats : nullptr;
+    const float* lnc = ln ? L->ln_sums + L->desc.hidden : nullptr;
     if (L->desc.dtype == CLEARMOE_F32) {
         cm::SimtGemmArgs g;
         std::memset(&g, 0, sizeof(g));
@@ -78,6 +84,8 @@ int mlp_hidden(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_mlp_r
         g.relu = m->act == CLEARMOE_ACT_RELU;
         g.C = static_cast<float*>(L->z);
         g.ldc = nh;
+        g.ln_stats = lns;
+        g.ln_colsum = lnc;
         return cuda_fail(cm::launch_simt_gemm(g, s));
     }
     cm::TcGemmArgs g;
@@ -98,6 +106,8 @@ int mlp_hidden(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_mlp_r
     g.C = L->z;
     g.ldc = nh;
     g.c_f32 = 1;
+    g.ln_stats = lns;
+    g.ln_colsum = lnc;
     return cuda_fail(p ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s));
 }
 
@@ -130,8 +140,22 @@ int check_router_and_options(const clearmoe_layer* L, const clearmoe_router* rou
     return CLEARMOE_OK;
 }
 
+// The LayerNorm of x folded into its consumers (input_layernorm): (mean, rstd) of every token row,
+// the row sums of W1 and those of the router's matrix applied to x (W_g, or the MLP router's W_in),
+// in one launch ahead of the routing.
+int ln_prep(clearmoe_layer* L, const void* y, int64_t T, const void* W1, const void* Wr, int rows_r, cudaStream_t s) {
+    cm::LnSums w = {};
+    w.W[0] = W1;
+    w.c[0] = L->ln_sums;
+    w.rows[0] = W1 ? L->desc.hidden : 0;
+    w.W[1] = Wr;
+    w.c[1] = L->ln_sums + L->desc.hidden;
+    w.rows[1] = Wr ? rows_r : 0;
+    return cuda_fail(cm::launch_ln_prep(y, L->ln_stats, T, L->desc.d, w, L->desc.dtype, s));
+}
+
 int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router,
-             const clearmoe_mlp_router* mlp, int E, int64_t cls_stride, cudaStream_t s) {
+             const clearmoe_mlp_router* mlp, int E, int64_t cls_stride, cudaStream_t s, bool ln = false) {
     // the MLP router: its hidden layer first, then the routing kernel on it (fp32 tokens)
     const int rd = mlp ? mlp->hidden : L->desc.d;
     const int rdtype = mlp ? CLEARMOE_F32 : L->desc.dtype;
@@ -140,7 +164,7 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
     if (g) return g == -2 ? CLEARMOE_EUNSUPPORTED : CLEARMOE_ECUDA;
     if (grid > cm::route_max_ctas(L->num_sms, rdtype, rd, E)) return CLEARMOE_EUNSUPPORTED;
     if (mlp) {
-        const int rc = mlp_hidden(L, x, T, mlp, s);
+        const int rc = mlp_hidden(L, x, T, mlp, ln, s);
         if (rc) return rc;
     }
     cm::RouteArgs& a = L->rt;
@@ -164,6 +188,10 @@ int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router*
     a.wait_limit_ns = L->wait_limit_ns;
     a.status = L->status;
     a.cls_stride = cls_stride;
+    if (ln && !mlp) {  // the MLP router folds it into its hidden layer instead
+        a.ln_stats = L->ln_stats;
+        a.ln_wsum = L->ln_sums + L->desc.hidden;
+    }
     L->rt_grid = grid;
     L->rt_chunk = chunk;
     const int rc = cuda_fail(cm::launch_route(a, grid, chunk, s));
@@ -245,7 +273,9 @@ int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out)
               cudaMalloc((void**)&L->offsets, (CM_MAX_E + 1) * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->cta_counts, ncta * CM_MAX_E * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->tinfo, T * 4) == cudaSuccess &&
-              cudaMalloc((void**)&L->status, 4) == cudaSuccess;
+              cudaMalloc((void**)&L->status, 4) == cudaSuccess &&
+              cudaMalloc((void**)&L->ln_stats, T * sizeof(float2)) == cudaSuccess &&
+              cudaMalloc((void**)&L->ln_sums, (2 * (size_t)D.hidden + CM_MAX_E) * 4) == cudaSuccess;
     if (ok) {
         // index workspaces start at zero (valid rows), so no launch ever reads garbage indices
         ok = cudaMemset(L->status, 0, 4) == cudaSuccess && cudaMemset(L->perm, 0, T * 4) == cudaSuccess &&
@@ -307,9 +337,12 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     const int64_t n_cls = cm::n_class_tokens(T, cls_stride);
     const int G = E + (cls_stride > 0 ? 1 : 0);  // groups of the grouped GEMM
     const void* b2 = opt ? opt->b2 : nullptr;
+    const clearmoe_mlp_router* mlp = opt ? opt->mlp_router : nullptr;
+    const bool ln = opt && opt->input_layernorm;  // x is y: LN(y) folded into the router and fc1
     int rc;
     mark(L, 0, s);
-    if ((rc = do_route(L, x, T, router, opt ? opt->mlp_router : nullptr, E, cls_stride, s))) return rc;
+    if (ln && (rc = ln_prep(L, x, T, W1, mlp ? mlp->W_in : router->W, mlp ? mlp->hidden : E, s))) return rc;
+    if ((rc = do_route(L, x, T, router, mlp, E, cls_stride, s, ln))) return rc;
     // bf16 with the 2-SM fc1: the fc1 epilogue assigns the slots itself (no finalize launch)
     const int p1 = bf16 && H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;
     const bool fused = p1 && L->rt_grid <= 256 && L->rt_grid * E <= cm::TC2_TAB_CAP;
@@ -331,6 +364,10 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         g.gelu = 1;
         g.C = static_cast<float*>(L->z);
         g.ldc = H;
+        if (ln) {
+            g.ln_stats = L->ln_stats;
+            g.ln_colsum = L->ln_sums;
+        }
         if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
         mark(L, 2, s);
         if (factored) {  // t = diag(S_r) Vh_r z
@@ -400,6 +437,10 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     g.bias = b1;
     g.C = L->z;
     g.ldc = H;
+    if (ln) {
+        g.ln_stats = L->ln_stats;
+        g.ln_colsum = L->ln_sums;
+    }
     if (p1) {
         if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, p1 / 2))
             return CLEARMOE_ECUDA;
@@ -752,16 +793,18 @@ int clearmoe_dense_ffn_forward(clearmoe_layer* L, const void* x, int64_t T, cons
     return clearmoe_dense_ffn_forward_ex(L, x, T, W1, b1, W2, nullptr, out, stream);
 }
 
-int clearmoe_dense_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
-                                  const void* W2, const void* b2, void* out, void* stream) {
+static int dense_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1, const void* W2,
+                      const void* b2, bool ln, void* out, cudaStream_t s) {
     int rc = check_common(L, x, T);
     if (rc) return rc;
     if (!W1 || !b1 || !W2 || !out) return CLEARMOE_EINVAL;
     if (misaligned(W1) || misaligned(b1) || misaligned(W2) || misaligned(out) || misaligned(b2))
         return CLEARMOE_EINVAL;
     const int d = L->desc.d, H = L->desc.hidden;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
     mark(L, 0, s);
+    if (ln && (rc = ln_prep(L, x, T, W1, nullptr, 0, s))) return rc;  // x is y: LN(y) folded into fc1
+    const float2* lns = ln ? L->ln_stats : nullptr;
+    const float* lnc = ln ? L->ln_sums : nullptr;
     if (L->desc.dtype == CLEARMOE_F32) {
         cm::SimtGemmArgs g;
         std::memset(&g, 0, sizeof(g));
@@ -775,6 +818,8 @@ int clearmoe_dense_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, c
         g.gelu = 1;
         g.C = static_cast<float*>(L->z);
         g.ldc = H;
+        g.ln_stats = lns;
+        g.ln_colsum = lnc;
         if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
         mark(L, 1, s);
         std::memset(&g, 0, sizeof(g));
@@ -809,6 +854,8 @@ int clearmoe_dense_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, c
     g.bias = b1;
     g.C = L->z;
     g.ldc = H;
+    g.ln_stats = lns;
+    g.ln_colsum = lnc;
     if ((rc = cuda_fail(pair1 ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s))))
         return rc;
     mark(L, 1, s);
@@ -829,6 +876,18 @@ int clearmoe_dense_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, c
     rc = cuda_fail(pair2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
     mark(L, 2, s);
     return rc;
+}
+
+int clearmoe_dense_ffn_forward_ex(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                                  const void* W2, const void* b2, void* out, void* stream) {
+    return dense_impl(L, x, T, W1, b1, W2, b2, false, out, static_cast<cudaStream_t>(stream));
+}
+
+int clearmoe_dense_ffn_forward_opt(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                                   const void* W2, const clearmoe_ffn_options* opt, void* out, void* stream) {
+    if (opt && (opt->cls_stride != 0 || opt->mlp_router)) return CLEARMOE_EINVAL;
+    return dense_impl(L, x, T, W1, b1, W2, opt ? opt->b2 : nullptr, opt && opt->input_layernorm, out,
+                      static_cast<cudaStream_t>(stream));
 }
 
 int clearmoe_layer_norm(clearmoe_layer* L, const void* y, int64_t T, void* x_out, void* stream) {

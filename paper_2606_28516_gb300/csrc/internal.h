@@ -29,6 +29,10 @@ struct RouteArgs {
     // E (idx = E), the dense path, whose slots follow every expert's: T - n_cls + t / cls_stride
     int64_t cls_stride;
     int w_bf16;  // fp32 tokens (the MLP router's hidden layer) with bf16 W_g and b_g
+    // x is the un-normalised stream y (nullable = x is the router's input as is): logits
+    // rstd_t (W_g y_t - mean_t g) + b_g with (mean_t, rstd_t) = ln_stats[t], g_e = ln_wsum[e] = sum_k W_g[e, k]
+    const float2* ln_stats;
+    const float* ln_wsum;
 };
 // Class tokens of T: every cls_stride-th from token 0 (none when cls_stride is 0).
 __host__ __device__ inline int64_t n_class_tokens(int64_t T, int64_t cls_stride) {
@@ -85,10 +89,23 @@ struct SimtGemmArgs {
     const float* group_scale;
     int scale_groups;
     int row_scale_inv;
+    // the LayerNorm folded into A0 (A0 = un-normalised rows y): acc <- rstd (acc - mean c_n) before
+    // the bias, with (mean, rstd) = ln_stats[A0's row] and c_n = ln_colsum[n] = sum_k B0[n, k]
+    const float2* ln_stats;
+    const float* ln_colsum;
 };
 cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s);
 
 cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s);
+// Row sums of up to two weight matrices of d columns (layer dtype): c[m][n] = sum_k W[m][n, k], fp32.
+struct LnSums {
+    const void* W[2];
+    float* c[2];
+    int64_t rows[2];
+};
+// The LayerNorm folded into its consumers, one launch: stats[t] = (mean, 1 / sqrt(var + 1e-6)) of
+// every row of y [T x d], and the row sums w of the weights that multiply the normalised rows.
+cudaError_t launch_ln_prep(const void* y, float2* stats, int64_t T, int d, const LnSums& w, int dtype, cudaStream_t s);
 
 // ---- tcgen05 bf16 GEMMs ----
 enum TcEpi { TC_EPI_BIAS_GELU = 0, TC_EPI_SCALE = 1, TC_EPI_STORE = 2, TC_EPI_SCATTER = 3, TC_EPI_BIAS_RELU = 4 };
@@ -153,6 +170,11 @@ struct TcGemmArgs {
     // 2-SM kernel: A tiles loaded with the L2 evict-first policy (a stream read once), so that they
     // displace one another rather than lines the next reads are still to find in L2
     int a_evict_first;
+    // The LayerNorm folded into A (A = un-normalised rows y; single-segment modes): the accumulator
+    // becomes rstd (acc - mean c_n) before the epilogue, with (mean, rstd) = ln_stats[A's row] (the
+    // gathered row in TC_GATHER) and c_n = ln_colsum[n] = sum_k B[n, k]; nullable
+    const float2* ln_stats;
+    const float* ln_colsum;
 };
 // Boundary e of a grouped GEMM's groups: offsets[e], or the single group [0, M) without offsets.
 __host__ __device__ inline int64_t tc_group_off(const TcGemmArgs& a, int e) {

@@ -273,6 +273,12 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                     for (int i = 0; i < 4; ++i)
                         acc[nt][i] = (part[nt][0][i] + part[nt][1][i]) + (part[nt][2][i] + part[nt][3][i]);
                 // D fragment: acc[nt][0..1] = row g, experts nt*8 + 2*tig + {0,1}; [2..3] = row g+8
+                float2 lnA = make_float2(0.f, 1.f), lnB = make_float2(0.f, 1.f);  // (mean, rstd)
+                if (a.ln_stats) {
+                    const int64_t tA = row0 + (int64_t)k * RT_STAGE_ROWS + g;
+                    if (vA) lnA = a.ln_stats[tA];
+                    if (vB) lnB = a.ln_stats[tA + 8];
+                }
                 float bA = -INFINITY, bB = -INFINITY;
                 int eA = 0x7fffffff, eB = 0x7fffffff;
 #pragma unroll
@@ -283,8 +289,14 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                         if (nt < NT && e < E) {
                             const uint16_t bb = bgp[e];
                             const float bias = __uint_as_float((uint32_t)bb << 16);
-                            arg_better(bA, eA, acc[nt][j] + bias, e);
-                            arg_better(bB, eB, acc[nt][2 + j] + bias, e);
+                            float lA = acc[nt][j], lB = acc[nt][2 + j];
+                            if (a.ln_stats) {  // W_g LN(y) = rstd (W_g y - mean g)
+                                const float ge = a.ln_wsum[e];
+                                lA = lnA.y * fmaf(-lnA.x, ge, lA);
+                                lB = lnB.y * fmaf(-lnB.x, ge, lB);
+                            }
+                            arg_better(bA, eA, lA + bias, e);
+                            arg_better(bB, eB, lB + bias, e);
                         }
                     }
                 }
@@ -375,6 +387,12 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                         }
                     }
                 }
+            }
+            if (a.ln_stats) {  // W_g LN(y) = rstd (W_g y - mean g)
+                const float2 st = valid ? a.ln_stats[row0 + i] : make_float2(0.f, 1.f);
+#pragma unroll
+                for (int e = 0; e < CM_MAX_E; ++e)
+                    if (e < E) acc[e] = st.y * fmaf(-st.x, a.ln_wsum[e], acc[e]);
             }
             float bv = -INFINITY;
             int be = 0x7fffffff;

@@ -8,7 +8,8 @@
 // segment with a per-expert B (the grouped residual GEMM, Algorithm 3 step 5; with dense_last the
 // last group is the class tokens' dense path, second segment only), an epilogue of
 // bias, GELU or ReLU, per-column scale and per-row scale, and an optional row scatter of C (the
-// unshuffle, step 6).
+// unshuffle, step 6). With the LayerNorm folded into A0 (rows of the un-normalised stream y) the
+// epilogue first forms rstd (acc - mean c_n), c_n = sum_k B0[n, k], since W LN(y) = rstd (W y - mean W 1).
 #include "common.cuh"
 #include "internal.h"
 
@@ -118,11 +119,17 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
         if (m >= m_hi) continue;
         const int64_t orow = a.c_rows ? (int64_t)a.c_rows[m] : m;
         if ((uint64_t)orow >= (uint64_t)a.M) continue;  // only a launch that gave up leaves such rows
+        float2 ln = make_float2(0.f, 1.f);  // the LayerNorm folded into A0: (mean, rstd) of its row
+        if (a.ln_stats) {
+            const int64_t ar = a.a_rows ? (int64_t)a.a_rows[m] : m;
+            if ((uint64_t)ar < (uint64_t)a.M) ln = a.ln_stats[ar];
+        }
 #pragma unroll
         for (int j = 0; j < R; ++j) {
             const int n = n0 + tx * R + j;
             if (n >= a.N) continue;
             float v = acc[i][j];
+            if (a.ln_stats) v = ln.y * fmaf(-ln.x, a.ln_colsum[n], v);  // W LN(y) = rstd (W y - mean c)
             if (a.bias) v += a.bias[n];
             if (a.gelu) v = gelu_erf(v);
             if (a.relu) v = fmaxf(v, 0.f);
@@ -165,13 +172,27 @@ cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
 // ------------------------------------------------------------------ LayerNorm (no affine)
 // One warp per token row; fp32 statistics in two passes over registers (mean, then the biased
 // variance of the centred values); x = (y - mean) / sqrt(var + 1e-6).
-template <bool BF16>
-__global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x, int64_t T, int d) {
-    pdl_wait();  // y is the previous kernel's output
+// STATS (the LayerNorm folded into its consumers): warp rows [0, T) write (mean, 1 / sqrt(var +
+// 1e-6)) of row `row` of y to x as float2; the warp rows after them sum the rows of the weight
+// matrices in w (c[n] = sum_k W[n, k], d columns each), in the same chunk order and warp tree.
+template <bool BF16, bool STATS>
+__global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x, int64_t T, int d, const LnSums w) {
+    pdl_wait();  // y is the previous kernel's output; the sums' buffers may still be read by it
     pdl_launch_dependents();  // the next sublayer's first kernel may set itself up meanwhile
     const int lane = threadIdx.x & 31;
-    const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
-    if (row >= T) return;
+    int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+    const void* src = y;
+    float* csum = nullptr;  // a weight row: its sum goes to csum[row]
+    if (row >= T) {
+        if constexpr (!STATS) return;
+        int64_t wr = row - T;
+        int m = 0;
+        while (m < 2 && wr >= w.rows[m]) wr -= w.rows[m++];
+        if (m == 2) return;
+        src = w.W[m];
+        csum = w.c[m];
+        row = wr;
+    }
     constexpr int VEC = BF16 ? 8 : 4;  // elements per 16-byte chunk
     constexpr int MAXC = 4;            // chunks per lane: d <= 32 * MAXC * VEC
     float v[MAXC][VEC];
@@ -182,7 +203,7 @@ __global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x,
         const int ch = lane + 32 * c;
         if (ch < nch) {
             const uint4 u = reinterpret_cast<const uint4*>(
-                static_cast<const unsigned char*>(y) + (row * d + (int64_t)ch * VEC) * (BF16 ? 2 : 4))[0];
+                static_cast<const unsigned char*>(src) + (row * d + (int64_t)ch * VEC) * (BF16 ? 2 : 4))[0];
             if constexpr (BF16) {
                 const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
@@ -202,6 +223,10 @@ __global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x,
     }
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    if (STATS && csum) {
+        if (lane == 0) csum[row] = sum;
+        return;
+    }
     const float mean = sum / (float)d;
     float sq = 0.f;
 #pragma unroll
@@ -217,6 +242,10 @@ __global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x,
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
     const float inv = 1.0f / sqrtf(sq / (float)d + 1e-6f);
+    if constexpr (STATS) {
+        if (lane == 0) static_cast<float2*>(x)[row] = make_float2(mean, inv);
+        return;
+    }
 #pragma unroll
     for (int c = 0; c < MAXC; ++c) {
         const int ch = lane + 32 * c;
@@ -238,18 +267,33 @@ __global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x,
     }
 }
 
-cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)((T + 7) / 8));
+static void pdl_config(cudaLaunchConfig_t& cfg, cudaLaunchAttribute* attr, unsigned grid, cudaStream_t s) {
+    cfg = {};
+    cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(256);
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (dtype == CLEARMOE_BF16) return cudaLaunchKernelEx(&cfg, layer_norm_kernel<true>, y, x, T, d);
-    return cudaLaunchKernelEx(&cfg, layer_norm_kernel<false>, y, x, T, d);
+}
+
+cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s) {
+    cudaLaunchConfig_t cfg;
+    cudaLaunchAttribute attr[1];
+    pdl_config(cfg, attr, (unsigned)((T + 7) / 8), s);
+    const LnSums none = {};
+    if (dtype == CLEARMOE_BF16) return cudaLaunchKernelEx(&cfg, layer_norm_kernel<true, false>, y, x, T, d, none);
+    return cudaLaunchKernelEx(&cfg, layer_norm_kernel<false, false>, y, x, T, d, none);
+}
+
+cudaError_t launch_ln_prep(const void* y, float2* stats, int64_t T, int d, const LnSums& w, int dtype, cudaStream_t s) {
+    cudaLaunchConfig_t cfg;
+    cudaLaunchAttribute attr[1];
+    pdl_config(cfg, attr, (unsigned)((T + w.rows[0] + w.rows[1] + 7) / 8), s);
+    void* out = stats;
+    if (dtype == CLEARMOE_BF16) return cudaLaunchKernelEx(&cfg, layer_norm_kernel<true, true>, y, out, T, d, w);
+    return cudaLaunchKernelEx(&cfg, layer_norm_kernel<false, true>, y, out, T, d, w);
 }
 
 }  // namespace cm

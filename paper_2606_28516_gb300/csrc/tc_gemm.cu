@@ -299,6 +299,12 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
             if (r < t.rows) orow = (a.epi == TC_EPI_SCATTER) ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
             const float rsc = (a.group_scale && r < t.rows) ? tc_row_scale(a, t.m0 + r) : 1.f;
             if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;
+            // the LayerNorm folded into A: (mean, rstd) of the token whose row this lane holds
+            float2 ln = make_float2(0.f, 1.f);
+            if (a.ln_stats && r < t.rows) {
+                const int64_t tok = a.mode == TC_GATHER ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
+                if ((uint64_t)tok < (uint64_t)a.M) ln = a.ln_stats[tok];
+            }
             for (int c = c_lo; c < c_lo + C::HALF; c += C::CW) {
                 uint32_t v[32];
                 const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
@@ -313,6 +319,10 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
 #pragma unroll
                 for (int j = 0; j < C::CW; ++j) f[j] = __uint_as_float(v[j]);
                 const int nb = t.n0 + c;
+                if (a.ln_stats) {  // W LN(y) = rstd (W y - mean c), c_n = sum_k W[n, k]
+#pragma unroll
+                    for (int j = 0; j < C::CW; ++j) f[j] = ln.y * fmaf(-ln.x, __ldg(a.ln_colsum + nb + j), f[j]);
+                }
                 if (a.epi == TC_EPI_BIAS_GELU) {
                     const uint4* bp = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.bias) + nb);
 #pragma unroll

@@ -454,6 +454,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                 }
             }
             const float rsc = (a.group_scale && mrow < t.hi) ? tc_row_scale(a, mrow) : 1.f;
+            // the LayerNorm folded into A: (mean, rstd) of this lane's row
+            const float2 ln = (a.ln_stats && mrow < t.hi) ? a.ln_stats[mrow] : make_float2(0.f, 1.f);
             // this lane stores warp rows 16 h + 8 p + lane / 4 (h, p < 2), 16-byte piece lane % 4 of
             // each 32-column chunk: their destinations, once per tile
             uint16_t* dst_row[4];
@@ -472,6 +474,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
 #pragma unroll
                 for (int j = 0; j < CW; ++j) f[j] = __uint_as_float(v[j]);
                 const int nb = t.n0 + c;
+                if (a.ln_stats) {  // W LN(y) = rstd (W y - mean c), c_n = sum_k W[n, k]
+                    const float4* cp = reinterpret_cast<const float4*>(a.ln_colsum + nb);  // same for all lanes
+#pragma unroll
+                    for (int j4 = 0; j4 < CW / 4; ++j4) {
+                        const float4 c4 = __ldg(cp + j4);
+                        f[4 * j4] = ln.y * fmaf(-ln.x, c4.x, f[4 * j4]);
+                        f[4 * j4 + 1] = ln.y * fmaf(-ln.x, c4.y, f[4 * j4 + 1]);
+                        f[4 * j4 + 2] = ln.y * fmaf(-ln.x, c4.z, f[4 * j4 + 2]);
+                        f[4 * j4 + 3] = ln.y * fmaf(-ln.x, c4.w, f[4 * j4 + 3]);
+                    }
+                }
                 if (a.epi == TC_EPI_BIAS_GELU) {
                     const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
 #pragma unroll

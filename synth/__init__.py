@@ -134,6 +134,17 @@ def layer_norm(x: np.ndarray) -> np.ndarray:
     return (x - mu) / np.sqrt(var + LN_EPS)
 
 
+def residual_stream(x: np.ndarray, dtype: str, seed: int = 7, scale=(0.5, 4.0), shift: float = 1.0):
+    """An un-normalised stream y whose per-token LayerNorm is x again (x's rows have mean 0 and
+    variance 1; up to the eps and the rounding of y): y_t = s_t x_t + m_t with s_t ~ U(scale) and
+    m_t ~ N(0, shift^2) drawn per token, rounded to the layer dtype."""
+    rng = np.random.default_rng(seed)
+    T = x.shape[0]
+    s = rng.uniform(scale[0], scale[1], size=(T, 1))
+    m = shift * rng.standard_normal((T, 1))
+    return to_dtype(np.asarray(x, np.float64) * s + m, dtype)
+
+
 def mixture_tokens(rng: np.random.Generator, centroids: np.ndarray, sizes: np.ndarray,
                    sigma: float):
     labels = rng.permutation(np.repeat(np.arange(len(sizes)), sizes))

@@ -3,7 +3,8 @@ CLEAR-MoE with E = 8, r = 128, even sublayers dense, x_{l+1} = LN(y_l), bf16), t
 
 Every sublayer is checked against the oracle on the GPU's own input to that sublayer, so errors do
 not compound across layers: routing on all tokens (bit-exact outside near ties), the sublayer's
-output on sampled rows (plus the whole smallest expert), and the LayerNorm on sampled rows."""
+output on sampled rows (plus the whole smallest expert), and the LayerNorm on sampled rows; then
+the same with the LayerNorm folded into each next sublayer (input_layernorm)."""
 import numpy as np
 import pytest
 import torch
@@ -81,5 +82,57 @@ def test_vit_base_stack12(workload):
                     f"first: got {ln_got[i, j]!r} want {ln_want[i, j]!r}; row mean {yr.mean():.6g} "
                     f"std {yr.std():.6g} max|y| {np.abs(yr).max():.6g}")
             x = x_next
+    finally:
+        cm.clearmoe_layer_destroy(h)
+
+
+def test_vit_base_stack12_layernorm_folded(workload):
+    """The same stack with the LayerNorm between sublayers folded into the next sublayer's router
+    and fc1 (input_layernorm): sublayer l > 0 is given y_{l-1} itself, and is checked against the
+    oracle on LN(y_{l-1}) formed in float64 from the GPU's y_{l-1}."""
+    import __graft_entry__
+    __graft_entry__.build()
+    S = workload(synth.VIT_BASE_STACK12)
+    sh = S["shape"]
+    T = S["T"]
+    h = cm.clearmoe_layer_create(T, sh.d, sh.H, sh.E, sh.r, cm.BF16)
+    try:
+        x = _dev(S["x"])
+        rng = np.random.default_rng(2)
+        for l, L in enumerate(S["layers"]):
+            W1, b1 = _dev(L["W1"]), _dev(L["b1"])
+            y = torch.empty(T, sh.d, device="cuda", dtype=torch.bfloat16)
+            ln = l > 0
+            if L["moe"]:
+                U, Vh, res = _dev(L["U"]), _dev(L["Vh"]), _dev(L["residuals"])
+                Wg, bg = _dev(L["Wg"]), _dev(L["bg"])
+                Sr = torch.from_numpy(L["S"].astype(np.float32)).cuda()
+                cm.clearmoe_ffn_forward_ex(h, x, W1, b1, U, Sr, Vh, res, Wg, bg, y, input_layernorm=ln)
+                idx = torch.empty(T, dtype=torch.int32, device="cuda")
+                perm = torch.empty_like(idx)
+                counts = torch.empty(sh.E, dtype=torch.int32, device="cuda")
+                offsets = torch.empty(sh.E + 1, dtype=torch.int32, device="cuda")
+                cm.clearmoe_get_routing(h, idx, counts, offsets, perm)
+            else:
+                cm.clearmoe_dense_ffn_forward_opt(h, x, W1, b1, _dev(L["W2"]), y, input_layernorm=ln)
+            torch.cuda.synchronize()
+            assert cm.clearmoe_layer_status(h) == 0
+            x_in = x.float().cpu().numpy()
+            if ln:
+                x_in = O.layer_norm(x_in)
+            if L["moe"]:
+                gr = dict(a=idx.cpu().numpy().astype(np.int64), counts=counts.cpu().numpy().astype(np.int64),
+                          offsets=offsets.cpu().numpy().astype(np.int64),
+                          perm=perm.cpu().numpy().astype(np.int64))
+                check_routing(gr, x_in, L["Wg"], L["bg"])
+                rows = sample_rows(gr, T, n=1024, seed=l)
+                want = O.ffn_forward(x_in[rows], L["W1"], L["b1"], L["U"], L["S"], L["Vh"],
+                                     L["residuals"], a=gr["a"][rows], z_bf16=True)
+            else:
+                rows = np.sort(rng.choice(T, 1024, replace=False))
+                want = O.dense_ffn(x_in[rows], L["W1"], L["b1"], L["W2"], z_bf16=True)
+            err = out_error(y[torch.from_numpy(rows).cuda()], want, "bf16")
+            assert err <= tol("bf16"), f"sublayer {l}: output error {err:.3e}"
+            x = y  # the next sublayer normalises it itself
     finally:
         cm.clearmoe_layer_destroy(h)

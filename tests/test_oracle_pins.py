@@ -465,3 +465,15 @@ def test_pins_catch_planted_mistakes(name, monkeypatch):
         except Exception:
             results.append(False)
     assert not all(results), f"no pin caught the planted mistake: {name}"
+
+
+def test_layernorm_fold_identity():
+    """The fold the router and fc1 use for input_layernorm: W LN(y) = rstd (W y - mean W 1), with
+    (mean, rstd) the per-row statistics of the oracle's LayerNorm (eps included)."""
+    rng = np.random.default_rng(5)
+    y = rng.uniform(0.5, 4.0, (64, 1)) * rng.standard_normal((64, 96)) + rng.standard_normal((64, 1))
+    W = rng.standard_normal((40, 96))
+    mu = y.astype(np.float64).mean(axis=1, keepdims=True)
+    rstd = 1.0 / np.sqrt(((y - mu) ** 2).mean(axis=1, keepdims=True) + O.LN_EPS)
+    fold = rstd * (y.astype(np.float64) @ W.T - mu * W.sum(axis=1)[None, :])
+    assert np.allclose(O.layer_norm(y) @ W.T, fold, rtol=1e-12, atol=1e-10)

@@ -84,3 +84,13 @@ def test_layer_shapes_and_dtype(workload):
     Lb = synth.make_layer(synth.DEIT_SMALL_BF16.with_(T=256, n_cal=1024))
     for k in ("x", "W1", "b1", "U", "Vh", "residuals", "Wg", "bg"):
         assert np.array_equal(synth.round_bf16(Lb[k]), Lb[k]), k
+
+
+@pytest.mark.parametrize("dtype,bound", [("f32", 1e-5), ("bf16", 2e-2)])
+def test_residual_stream_normalises_back(dtype, bound):
+    """y_t = s_t x_t + m_t per token: its LayerNorm is x again, up to the eps and y's rounding."""
+    x = synth.layer_norm(np.random.default_rng(4).standard_normal((128, 192)))
+    y = synth.residual_stream(x, dtype)
+    assert y.dtype == np.float32 and np.array_equal(y, synth.to_dtype(y, dtype))
+    assert np.abs(synth.layer_norm(y) - x).max() < bound
+    assert np.abs(y.mean(axis=1)).max() > 0.5  # the rows are shifted and scaled
