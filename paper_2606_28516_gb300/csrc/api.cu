@@ -25,6 +25,8 @@ struct clearmoe_layer {
     int32_t* status;
     float2* ln_stats;  // [max_tokens]  (mean, rstd) per token when the input LayerNorm is folded
     float* ln_sums;    // [2 hidden + CM_MAX_E]  row sums of W1, then of the router's first matrix
+    uint16_t* ln_aug_x;  // bf16 layers: [max_tokens x LN_AUG_K]  fc1's augmentation block, token side
+    uint16_t* ln_aug_w;  // bf16 layers: [hidden x LN_AUG_K]      and W1's side
     int64_t wait_limit_ns;
     int32_t phantom;  // fault injection: > 0 makes the routing withhold one stage copy
     cm::RouteArgs rt;  // the last routing launch (its consumers reuse the shape)
@@ -50,7 +52,8 @@ int cuda_fail(cudaError_t e) {
 
 void free_ws(clearmoe_layer* L) {
     void* ptrs[] = {L->z,     L->t,          L->idx,   L->perm,   L->inv,     L->counts,
-                    L->offsets, L->cta_counts, L->tinfo, L->status, L->ln_stats, L->ln_sums};
+                    L->offsets, L->cta_counts, L->tinfo, L->status, L->ln_stats, L->ln_sums,
+                    L->ln_aug_x, L->ln_aug_w};
     for (void* p : ptrs)
         if (p) cudaFree(p);
 }
@@ -142,7 +145,8 @@ int check_router_and_options(const clearmoe_layer* L, const clearmoe_router* rou
 
 // The LayerNorm of x folded into its consumers (input_layernorm): (mean, rstd) of every token row,
 // the row sums of W1 and those of the router's matrix applied to x (W_g, or the MLP router's W_in),
-// in one launch ahead of the routing.
+// and in bf16 layers the augmentation block that carries -mean W1 1 into fc1's MMAs, in one launch
+// ahead of the routing.
 int ln_prep(clearmoe_layer* L, const void* y, int64_t T, const void* W1, const void* Wr, int rows_r, cudaStream_t s) {
     cm::LnSums w = {};
     w.W[0] = W1;
@@ -151,7 +155,21 @@ int ln_prep(clearmoe_layer* L, const void* y, int64_t T, const void* W1, const v
     w.W[1] = Wr;
     w.c[1] = L->ln_sums + L->desc.hidden;
     w.rows[1] = Wr ? rows_r : 0;
+    w.aug_tok = L->ln_aug_x;  // null in fp32 layers
+    w.aug_w0 = W1 ? L->ln_aug_w : nullptr;
     return cuda_fail(cm::launch_ln_prep(y, L->ln_stats, T, L->desc.d, w, L->desc.dtype, s));
+}
+
+// A 2-SM fc1 (or the dense FFN's) with the LayerNorm folded: the mean term enters as one more K
+// block (LnSums' augmentation rows), and the epilogue scales by rstd inside its bias add.
+int ln_fc1_aug(clearmoe_layer* L, cm::TcGemmArgs& g, int64_t T, int b_box) {
+    g.ln_stats = L->ln_stats;
+    g.ln_colsum = nullptr;
+    g.ln_aug = 1;
+    if (encode_tmap_bf16(&g.tmA1, L->ln_aug_x, T, cm::LN_AUG_K, 128) ||
+        encode_tmap_bf16(&g.tmB1[0], L->ln_aug_w, L->desc.hidden, cm::LN_AUG_K, b_box))
+        return CLEARMOE_ECUDA;
+    return CLEARMOE_OK;
 }
 
 int do_route(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_router* router,
@@ -275,7 +293,10 @@ int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out)
               cudaMalloc((void**)&L->tinfo, T * 4) == cudaSuccess &&
               cudaMalloc((void**)&L->status, 4) == cudaSuccess &&
               cudaMalloc((void**)&L->ln_stats, T * sizeof(float2)) == cudaSuccess &&
-              cudaMalloc((void**)&L->ln_sums, (2 * (size_t)D.hidden + CM_MAX_E) * 4) == cudaSuccess;
+              cudaMalloc((void**)&L->ln_sums, (2 * (size_t)D.hidden + CM_MAX_E) * 4) == cudaSuccess &&
+              (D.dtype != CLEARMOE_BF16 ||
+               (cudaMalloc((void**)&L->ln_aug_x, T * cm::LN_AUG_K * 2) == cudaSuccess &&
+                cudaMalloc((void**)&L->ln_aug_w, (size_t)D.hidden * cm::LN_AUG_K * 2) == cudaSuccess));
     if (ok) {
         // index workspaces start at zero (valid rows), so no launch ever reads garbage indices
         ok = cudaMemset(L->status, 0, 4) == cudaSuccess && cudaMemset(L->perm, 0, T * 4) == cudaSuccess &&
@@ -444,6 +465,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     if (p1) {
         if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, p1 / 2))
             return CLEARMOE_ECUDA;
+        if (ln && (rc = ln_fc1_aug(L, g, T, p1 / 2))) return rc;
         g.mode = cm::TC_DENSE;
         if (fused) {  // slots from the routing's per-range counts and ranks; writes perm, counts, offsets
             g.rt_info = L->tinfo;
@@ -855,7 +877,8 @@ static int dense_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W
     g.C = L->z;
     g.ldc = H;
     g.ln_stats = lns;
-    g.ln_colsum = lnc;
+    g.ln_colsum = lnc;  // the 1-SM kernel: the column sums in the epilogue
+    if (ln && pair1 && (rc = ln_fc1_aug(L, g, T, pair1 / 2))) return rc;  // 2-SM: the augmentation block
     if ((rc = cuda_fail(pair1 ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s))))
         return rc;
     mark(L, 1, s);

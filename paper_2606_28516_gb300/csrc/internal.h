@@ -98,10 +98,18 @@ cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s);
 
 cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s);
 // Row sums of up to two weight matrices of d columns (layer dtype): c[m][n] = sum_k W[m][n, k], fp32.
+// aug_tok / aug_w0 (nullable, bf16, LN_AUG_K columns per row): the augmentation K block of a GEMM
+// whose A rows are the un-normalised tokens and whose B rows are W[0]'s. With mean = h + m + l and
+// c = h' + m' + l' split into bf16 parts (each the rounded remainder of the previous), a token row
+// holds (-h, -h, -h, -m, -m, -m, -l, -l, -l, 0, ...) and a weight row (h', m', l', h', m', l', h', m',
+// l', 0, ...), so that their 9 exact products sum to -mean c in the tensor cores' fp32 accumulator.
+constexpr int LN_AUG_K = 64;
 struct LnSums {
     const void* W[2];
     float* c[2];
     int64_t rows[2];
+    uint16_t* aug_tok;
+    uint16_t* aug_w0;
 };
 // The LayerNorm folded into its consumers, one launch: stats[t] = (mean, 1 / sqrt(var + 1e-6)) of
 // every row of y [T x d], and the row sums w of the weights that multiply the normalised rows.
@@ -175,6 +183,11 @@ struct TcGemmArgs {
     // gathered row in TC_GATHER) and c_n = ln_colsum[n] = sum_k B[n, k]; nullable
     const float2* ln_stats;
     const float* ln_colsum;
+    // TC_DENSE: one more K block after K0, A from tmA1 and B from tmB1[0] (the LayerNorm
+    // augmentation blocks of LnSums, 16 useful columns), which adds -mean c to the accumulator;
+    // with ln_stats set and ln_colsum null the epilogue then only scales by rstd, inside the bias
+    // add (BIAS_GELU / BIAS_RELU)
+    int ln_aug;
 };
 // Boundary e of a grouped GEMM's groups: offsets[e], or the single group [0, M) without offsets.
 __host__ __device__ inline int64_t tc_group_off(const TcGemmArgs& a, int e) {

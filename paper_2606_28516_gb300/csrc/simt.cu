@@ -170,6 +170,28 @@ cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
 }
 
 // ------------------------------------------------------------------ LayerNorm (no affine)
+// v = h + m + l with h, m, l bf16: each the nearest bf16 of what the previous parts leave over (the
+// remainders are exact in fp32), so that the three carry v's 24 significant bits.
+__device__ __forceinline__ void split3_bf16(float v, uint16_t* p) {
+    p[0] = f32_to_bf16(v);
+    const float r1 = v - bf16_to_f32(p[0]);
+    p[1] = f32_to_bf16(r1);
+    p[2] = f32_to_bf16(r1 - bf16_to_f32(p[1]));
+}
+// Lane j < LN_AUG_K / 8 of a warp writes columns 8 j .. 8 j + 7 of an augmentation row: v0..v8 in
+// columns 0..8, zeros after them.
+__device__ __forceinline__ void store_aug_row(uint16_t* row, int lane, uint16_t v0, uint16_t v1, uint16_t v2,
+                                              uint16_t v3, uint16_t v4, uint16_t v5, uint16_t v6, uint16_t v7,
+                                              uint16_t v8) {
+    uint4 u = make_uint4(0, 0, 0, 0);
+    if (lane == 0)
+        u = make_uint4((uint32_t)v0 | ((uint32_t)v1 << 16), (uint32_t)v2 | ((uint32_t)v3 << 16),
+                       (uint32_t)v4 | ((uint32_t)v5 << 16), (uint32_t)v6 | ((uint32_t)v7 << 16));
+    else if (lane == 1)
+        u.x = v8;
+    reinterpret_cast<uint4*>(row)[lane] = u;
+}
+
 // One warp per token row; fp32 statistics in two passes over registers (mean, then the biased
 // variance of the centred values); x = (y - mean) / sqrt(var + 1e-6).
 // STATS (the LayerNorm folded into its consumers): warp rows [0, T) write (mean, 1 / sqrt(var +
@@ -225,6 +247,11 @@ __global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x,
     for (int off = 16; off >= 1; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
     if (STATS && csum) {
         if (lane == 0) csum[row] = sum;
+        if (csum == w.c[0] && w.aug_w0 && lane < LN_AUG_K / 8) {  // W[0]'s augmentation row
+            uint16_t p[3];
+            split3_bf16(sum, p);
+            store_aug_row(w.aug_w0 + row * LN_AUG_K, lane, p[0], p[1], p[2], p[0], p[1], p[2], p[0], p[1], p[2]);
+        }
         return;
     }
     const float mean = sum / (float)d;
@@ -244,6 +271,11 @@ __global__ void __launch_bounds__(256) layer_norm_kernel(const void* y, void* x,
     const float inv = 1.0f / sqrtf(sq / (float)d + 1e-6f);
     if constexpr (STATS) {
         if (lane == 0) static_cast<float2*>(x)[row] = make_float2(mean, inv);
+        if (w.aug_tok && lane < LN_AUG_K / 8) {  // the token's augmentation row: -mean in 3 parts
+            uint16_t p[3];
+            split3_bf16(-mean, p);
+            store_aug_row(w.aug_tok + row * LN_AUG_K, lane, p[0], p[0], p[0], p[1], p[1], p[1], p[2], p[2], p[2]);
+        }
         return;
     }
 #pragma unroll

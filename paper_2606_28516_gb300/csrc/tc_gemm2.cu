@@ -10,7 +10,8 @@
 // Hand-offs: both CTAs' TMA loads complete on the even CTA's full barrier (the odd CTA's loads
 // name it through the cluster); the even CTA's MMA commits arrive on both CTAs' empty / tfull
 // barriers (multicast); the epilogue warps of both CTAs arrive on the even CTA's tempty barrier.
-// Modes: dense (one K segment, epilogue bias+GELU / plain store) and grouped (the residual
+// Modes: dense (one K segment, epilogue bias+GELU / plain store; with a LayerNorm folded into A, one
+// more K block of 16 useful columns carries -mean W 1 and the bias add scales by rstd) and grouped (the residual
 // experts: tile pairs never straddle an expert, K chain [z | t] x [W_e | U_r]; with dense_last
 // the last group is the class tokens' dense path, K chain z x W2 alone). Store epilogues may add
 // an output bias (fc2's b2). With a.rows set,
@@ -165,7 +166,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
 
     const int n_tiles = a.N / BN;
     const int nk0 = (a.K0 + BK - 1) / BK;
-    const int nk1 = MODE == TC_GROUPED ? (a.K1 + BK - 1) / BK : 0;
+    // grouped: the z x W_e^res segment; dense: the LayerNorm augmentation block, if any
+    const int nk1 = MODE == TC_GROUPED ? (a.K1 + BK - 1) / BK : (a.ln_aug ? 1 : 0);
     const int nkb = nk0 + nk1;
 
     if (threadIdx.x == 0) {
@@ -329,10 +331,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                     const CUtensorMap* mA;
                     const CUtensorMap* mB;
                     int kk;
-                    if (MODE != TC_GROUPED) {
-                        mA = &a.tmA0;
-                        mB = &a.tmB0;
-                        kk = kb * BK;
+                    if (MODE != TC_GROUPED) {  // x x W, then the augmentation block
+                        mA = kb < nk0 ? &a.tmA0 : &a.tmA1;
+                        mB = kb < nk0 ? &a.tmB0 : &a.tmB1[0];
+                        kk = kb < nk0 ? kb * BK : 0;
                     } else if (kb < nk1) {  // z x W_e^res
                         mA = &a.tmA1;
                         mB = &a.tmB1[t.e];
@@ -386,8 +388,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                     const uint64_t da = dA0 + (uint64_t)((stage * STAGE_BYTES) >> 4);
                     const uint64_t db = da + (uint64_t)(A_BYTES >> 4);
                     int krem;
-                    if (MODE != TC_GROUPED)
-                        krem = a.K0 - kb * BK;
+                    if (MODE != TC_GROUPED)  // the augmentation block's products sit in its first 16 columns
+                        krem = kb < nk0 ? a.K0 - kb * BK : 16;
                     else
                         krem = kb < nk1 ? a.K1 - kb * BK : a.K0 - (kb - nk1) * BK;
                     if (krem >= BK) {
@@ -434,6 +436,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
             const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
             // the token's routing word, loaded before the accumulator wait so that the wait hides it
             const uint32_t rtw = (MODE == TC_DENSE && a.rt_info && mrow < t.hi) ? (uint32_t)a.rt_info[mrow] : 0u;
+            // the LayerNorm folded into A: (mean, rstd) of this lane's row, loaded early for the same reason
+            const float2 ln = (a.ln_stats && mrow < t.hi) ? a.ln_stats[mrow] : make_float2(0.f, 1.f);
             if (!mbar_wait(tfull_bar(acc), aph, abort_flag, a.status, lim)) break;
             tc_fence_after();
             int64_t orow = -1;
@@ -454,8 +458,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                 }
             }
             const float rsc = (a.group_scale && mrow < t.hi) ? tc_row_scale(a, mrow) : 1.f;
-            // the LayerNorm folded into A: (mean, rstd) of this lane's row
-            const float2 ln = (a.ln_stats && mrow < t.hi) ? a.ln_stats[mrow] : make_float2(0.f, 1.f);
+            // with the mean term in the accumulator (augmentation block) the bias add also scales by
+            // rstd: fma(acc, 1, b) = acc + b exactly, so without the LayerNorm nothing changes
+            const float lns = (a.ln_stats && !a.ln_colsum) ? ln.y : 1.f;
+            const float2 lns2 = make_float2(lns, lns);
             // this lane stores warp rows 16 h + 8 p + lane / 4 (h, p < 2), 16-byte piece lane % 4 of
             // each 32-column chunk: their destinations, once per tile
             uint16_t* dst_row[4];
@@ -474,7 +480,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
 #pragma unroll
                 for (int j = 0; j < CW; ++j) f[j] = __uint_as_float(v[j]);
                 const int nb = t.n0 + c;
-                if (a.ln_stats) {  // W LN(y) = rstd (W y - mean c), c_n = sum_k W[n, k]
+                if (a.ln_stats && a.ln_colsum) {  // W LN(y) = rstd (W y - mean c), c_n = sum_k W[n, k]
                     const float4* cp = reinterpret_cast<const float4*>(a.ln_colsum + nb);  // same for all lanes
 #pragma unroll
                     for (int j4 = 0; j4 < CW / 4; ++j4) {
@@ -491,9 +497,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                     for (int j4 = 0; j4 < CW / 4; ++j4) {
                         const float4 b = bp[j4];
                         const float2 g0 = gelu_pair_as(
-                            __fadd2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), make_float2(b.x, b.y)));
+                            __ffma2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), lns2, make_float2(b.x, b.y)));
                         const float2 g1 = gelu_pair_as(
-                            __fadd2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), make_float2(b.z, b.w)));
+                            __ffma2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), lns2, make_float2(b.z, b.w)));
                         f[4 * j4] = g0.x;
                         f[4 * j4 + 1] = g0.y;
                         f[4 * j4 + 2] = g1.x;
@@ -504,10 +510,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
 #pragma unroll
                     for (int j4 = 0; j4 < CW / 4; ++j4) {
                         const float4 b = bp[j4];
-                        f[4 * j4] = fmaxf(f[4 * j4] + b.x, 0.f);
-                        f[4 * j4 + 1] = fmaxf(f[4 * j4 + 1] + b.y, 0.f);
-                        f[4 * j4 + 2] = fmaxf(f[4 * j4 + 2] + b.z, 0.f);
-                        f[4 * j4 + 3] = fmaxf(f[4 * j4 + 3] + b.w, 0.f);
+                        f[4 * j4] = fmaxf(fmaf(f[4 * j4], lns, b.x), 0.f);
+                        f[4 * j4 + 1] = fmaxf(fmaf(f[4 * j4 + 1], lns, b.y), 0.f);
+                        f[4 * j4 + 2] = fmaxf(fmaf(f[4 * j4 + 2], lns, b.z), 0.f);
+                        f[4 * j4 + 3] = fmaxf(fmaf(f[4 * j4 + 3], lns, b.w), 0.f);
                     }
                 } else if (a.out_bias) {
                     const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
@@ -639,6 +645,11 @@ cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
                         a.epi == TC_EPI_SCALE;  // fp32 vector in shared memory
     if (!bn || (staged && (a.mode != TC_DENSE || a.N > TC2_BIAS_CAP))) return cudaErrorInvalidValue;
     if (a.out_bias && (staged || a.N > TC2_BIAS_CAP)) return cudaErrorInvalidValue;
+    // the LayerNorm fold: the augmentation block only ahead of a bias epilogue, and with the
+    // statistics but no column sums only together with it
+    const bool bias_epi = a.epi == TC_EPI_BIAS_GELU || a.epi == TC_EPI_BIAS_RELU;
+    if (a.ln_aug && (a.mode != TC_DENSE || !bias_epi || !a.ln_stats || a.ln_colsum)) return cudaErrorInvalidValue;
+    if (a.ln_stats && !a.ln_colsum && !a.ln_aug) return cudaErrorInvalidValue;
     if (bn == 256) return launch2<256>(a, num_sms, s);
     if (bn == 192) return launch2<192>(a, num_sms, s);
     return launch2<128>(a, num_sms, s);

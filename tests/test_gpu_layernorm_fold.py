@@ -91,7 +91,7 @@ def test_mlp_router(workload, shape, act):
     L = workload(shape)
     M = synth.mlp_router(L, act=act)
     D, Ln = _streams(L)
-    Dm = synth.to_torch(M)
+    Dm = synth.to_torch(dict(M, dtype=L["dtype"]))  # the weights in the layer dtype
     T = min(shape.T, 12608)
     with handle_for(L) as h:
         out = _nan_out(T, shape.d, D["x"])
@@ -168,7 +168,7 @@ def test_dense_rejects_router_options(workload):
     shape = synth.DEIT_SMALL_BF16
     L = workload(shape)
     D = synth.to_torch(L)
-    M = synth.to_torch(synth.mlp_router(L))
+    M = synth.to_torch(dict(synth.mlp_router(L), dtype=L["dtype"]))
     x = D["x"][:256]
     out = torch.zeros(256, shape.d, device="cuda", dtype=x.dtype)
     lib = cm.lib()
