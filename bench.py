@@ -587,7 +587,7 @@ def main():
         return {"value": whole_job_rate(s.T, world, 1, v_ms), "unit": "tokens/s", "ms_per_step": v_ms,
                 "note": note}
 
-    folded = materialized = class_tokens = mlp_router = scaled = None
+    folded = materialized = class_tokens = mlp_router = scaled = layernorm = None
     if s.dtype == "bf16" and not args.no_variants:
         W_comb = torch.empty_like(D["residuals"])
         cm.clearmoe_fold_basis(h, D["U"], D["S"], D["Vh"], D["residuals"], W_comb)
@@ -619,6 +619,27 @@ def main():
             lambda: cm.clearmoe_ffn_forward_ex(h, D["x"], D["W1"], D["b1"], D["U"], D["S"], D["Vh"],
                                                D["residuals"], None, None, out, mlp=mlp, E=s.E),
             f"MLP router d -> {s.d // 6} -> E (GELU) in place of the linear router")
+        # The sublayer's input as the LayerNorm of an un-normalised stream y: the LayerNorm kernel
+        # then the forward, against the forward with the LayerNorm folded in (input_layernorm).
+        try:
+            y_in = synth.to_torch({"x": synth.residual_stream(L["x"], s.dtype), "dtype": s.dtype})["x"]
+            x_ln = torch.empty_like(y_in)
+            layernorm = {
+                "layernorm_then_forward": time_variant(
+                    lambda: (cm.clearmoe_layer_norm(h, y_in, x_ln),
+                             cm.clearmoe_ffn_forward(h, x_ln, D["W1"], D["b1"], D["U"], D["S"], D["Vh"],
+                                                     D["residuals"], D["Wg"], D["bg"], out)),
+                    "clearmoe_layer_norm(y) into a T x d buffer, then the forward on it"),
+                "layernorm_folded": time_variant(
+                    lambda: cm.clearmoe_ffn_forward_ex(h, y_in, D["W1"], D["b1"], D["U"], D["S"], D["Vh"],
+                                                       D["residuals"], D["Wg"], D["bg"], out,
+                                                       input_layernorm=True),
+                    "input_layernorm: per-token statistics and fc1's augmentation block in one launch; "
+                    "the router and fc1 read y itself"),
+            }
+            del y_in, x_ln
+        except (cm.ClearMoEError, RuntimeError, TypeError, NameError, KeyError) as exc:
+            layernorm = {"error": f"{type(exc).__name__}: {exc}"}
 
     # same-GPU dense FFN, same timing rules (events around each forward only)
     dout = torch.empty_like(out)
@@ -760,6 +781,7 @@ def main():
         "class_tokens": class_tokens,
         "mlp_router": mlp_router,
         "scaled_residual": scaled,
+        "input_layernorm": layernorm,
         "wall_s_timed": wall,
     }
     if rank == 0:
