@@ -1,6 +1,7 @@
 """Every forward variant at ragged token counts (T = 1, 17, 300 on the DeiT-S bf16 layer), through
 the C ABI, against the float64 oracle: the folded and materialised basis forms, the one-residual-
-matrix form and the MLP router. A single token, a token count below one 16-row routing stage and
+matrix form, the MLP router and the folded input LayerNorm (the forward given y, the oracle run on
+LN(y)). A single token, a token count below one 16-row routing stage and
 one that leaves a partial 256-row tile all run the same kernels as the full layer."""
 import numpy as np
 import pytest
@@ -23,13 +24,14 @@ def _built():
 
 
 @pytest.mark.parametrize("T", [1, 17, 300])
-@pytest.mark.parametrize("form", ["folded", "materialized", "scaled", "mlp"])
+@pytest.mark.parametrize("form", ["folded", "materialized", "scaled", "mlp", "layernorm"])
 def test_variant_ragged(workload, form, T):
     L = workload(synth.DEIT_SMALL_BF16)
     s = L["shape"]
     M = synth.mlp_router(L, act="relu")
     D = synth.to_torch(L | M)
     x = D["x"][:T]
+    y = synth.residual_stream(L["x"], "bf16")[:T]  # the un-normalised stream of the LayerNorm form
     with handle_for(L) as h:
         out = torch.full((T, s.d), float("nan"), device="cuda", dtype=torch.bfloat16)
         if form == "folded":
@@ -43,13 +45,17 @@ def test_variant_ragged(workload, form, T):
         elif form == "scaled":
             cm.clearmoe_ffn_forward_scaled(h.h, x, D["W1"], D["b1"], D["U"], D["S"], D["Vh"], D["R"],
                                            D["scales"], D["Wg"], D["bg"], out)
+        elif form == "layernorm":
+            yd = synth.to_torch({"x": y, "dtype": "bf16"})["x"]
+            cm.clearmoe_ffn_forward_ex(h.h, yd, D["W1"], D["b1"], D["U"], D["S"], D["Vh"], D["residuals"],
+                                       D["Wg"], D["bg"], out, input_layernorm=True)
         else:
             m = cm.mlp_router(D["W_in"], D["b_in"], D["W_out"], D["b_out"], "relu")
             cm.clearmoe_ffn_forward_ex(h.h, x, D["W1"], D["b1"], D["U"], D["S"], D["Vh"], D["residuals"],
                                        None, None, out, mlp=m, E=s.E)
         gr = get_routing(h, T, s.E)
         assert cm.clearmoe_layer_status(h.h) == 0
-    xs = L["x"][:T]
+    xs = O.layer_norm(y) if form == "layernorm" else L["x"][:T]
     if form == "mlp":
         rt = O.route_mlp(xs, M["W_in"], M["b_in"], M["W_out"], M["b_out"], "relu")
     else:
