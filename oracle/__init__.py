@@ -9,6 +9,10 @@ Modules:
   clearmoe -- router, argmax routing, fc1 + GELU, shared basis, residual experts, dense FFN,
               the 12-sublayer stack (numpy float64; a matmul is the only library step)
   brute    -- pure-Python per-element loops on tiny shapes, used to pin `clearmoe`
+  clearmoe_ref.c, ref_c
+           -- the same layer in plain C (float64 loops, libm erf), loaded through ctypes; it
+              shares no code with the other two and is checked against them and the golden
+              values (tests/test_oracle_c.py)
 
 Parity status: every function in `clearmoe` is pinned (tests/test_oracle_pins.py) against
 closed forms, hand-derived golden values (tests/golden/), the brute force and the paper's
