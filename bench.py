@@ -723,6 +723,9 @@ def main():
     roof["frac"] = roof["achieved"] / roof["peak"]
     tr = TRAFFIC.get(dom)
     roof["traffic"] = tr["bytes"] if tr and tr["src"] == source_hash(dom) else None
+    if tr and roof["traffic"] is None:
+        roof["traffic_note"] = ("the kernel's sources changed after its ncu capture "
+                                f"(hash {source_hash(dom)} vs {tr['src']}): not re-captured yet")
     roof["kernel"] = KERNEL_OF_STAGE[dom]
     roof["peak_source"] = f"{pk_src} ({'sustained bf16' if roof['bound'] == 'tensor' else 'HBM copy'})"
 
