@@ -91,7 +91,9 @@ typedef struct {
 typedef struct clearmoe_layer clearmoe_layer;
 
 /* Allocates the handle and its device workspace on the current device (hidden states
- * [max_tokens x hidden], basis coefficients [max_tokens x max_r], routing arrays, status word).
+ * [max_tokens x hidden], basis coefficients [max_tokens x max_r], routing arrays, status word,
+ * and for the folded LayerNorm 8 bytes per token of statistics, fp32 row sums [2 hidden + 16] and,
+ * in bf16 layers, 128 bytes per token and per hidden unit of fc1's augmentation block).
  * Returns EINVAL for a null/invalid desc, EUNSUPPORTED per the tiling limits above, ENOMEM or
  * ECUDA if allocation fails (nothing is leaked). */
 int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out);
