@@ -125,3 +125,28 @@ def test_ties_bad_groups_and_empty_input():
     L = _layer(np.random.default_rng(4), 0, 8, 16, 2, 4)
     y = C.ffn_forward(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], L["residuals"], np.zeros(0, np.int64))
     assert y.shape == (0, 8)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_gpu_check_helper_on_the_numpy_oracle(dtype):
+    """The GPU test's comparison against the C oracle, fed the numpy oracle's routing and output
+    in place of the GPU's: it accepts them (to float64 rounding), and rejects a routing with one
+    token moved to another expert and an output with one element off."""
+    import synth
+    from test_gpu_c_oracle import check_against_c_oracle
+
+    shape = synth.LayerShape(f"tiny_{dtype}", 160, 32, 128, 4, 8, dtype, n_cal=1500)
+    L = synth.make_layer(shape)
+    gr = O.route(L["x"], L["Wg"], L["bg"])
+    y = O.ffn_forward(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], L["residuals"], a=gr["a"],
+                      z_bf16=dtype == "bf16")
+    assert check_against_c_oracle(L, y, gr) <= 1e-9
+    assert check_against_c_oracle(L, y, gr, rows=np.arange(0, 160, 3)) <= 1e-9
+    t = int(np.nonzero(~O.near_ties(L["x"], L["Wg"], L["bg"]))[0][0])
+    moved = dict(gr, a=gr["a"].copy())
+    moved["a"][t] = (moved["a"][t] + 1) % 4
+    with pytest.raises(AssertionError):
+        check_against_c_oracle(L, y, moved)
+    y_bad = y.copy()
+    y_bad[5, 3] += 1.0
+    assert check_against_c_oracle(L, y_bad, gr) > 1e-2
