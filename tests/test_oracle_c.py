@@ -133,7 +133,7 @@ def test_gpu_check_helper_on_the_numpy_oracle(dtype):
     in place of the GPU's: it accepts them (to float64 rounding), and rejects a routing with one
     token moved to another expert and an output with one element off."""
     import synth
-    from test_gpu_c_oracle import check_against_c_oracle
+    from test_gpu_vs_c_oracle import check_against_c_oracle
 
     shape = synth.LayerShape(f"tiny_{dtype}", 160, 32, 128, 4, 8, dtype, n_cal=1500)
     L = synth.make_layer(shape)
