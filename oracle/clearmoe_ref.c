@@ -12,8 +12,9 @@
  *   6. unshuffle and add: y <- h_sh + h_res
  * plus the deployment pieces the library offers: fc2's bias b2 on every row, class tokens on the
  * dense path W2 (group E after the experts), the MLP router, and the per-token LayerNorm of the
- * stacked workload. Shapes: x [T x d], W1 [H x d], b1 [H], U [d x r], S [r], Vh [r x H],
- * residuals [E x d x H], W_g [E x d], b_g [E], W2 [d x H], b2 [d], y [T x d].
+ * stacked workload, and the folded and one-residual-matrix forms. Shapes: x [T x d], W1 [H x d],
+ * b1 [H], U [d x r], S [r], Vh [r x H], residuals [E x d x H], W_g [E x d], b_g [E], W2 [d x H],
+ * b2 [d], y [T x d].
  * Compile with contraction off (-ffp-contract=off) so that x86 and Arm hosts agree bit for bit. */
 #include <math.h>
 #include <stdint.h>
@@ -222,4 +223,42 @@ void cmref_layer_norm(const double* y, int64_t T, int d, double eps, double* x) 
         const double inv = 1.0 / sqrt(var + eps);
         for (int k = 0; k < d; ++k) x[t * d + k] = (yr[k] - mean) * inv;
     }
+}
+
+/* Eq. 2 regrouped: both terms act on the same z, so W_shared z + W_e^res z = W_comb[e] z with
+ * W_comb[e] = W_shared + W_e^res, for every expert e (W_comb [E x d x H]). */
+void cmref_fold_basis(const double* U, const double* S, const double* Vh, const double* residuals, int E, int d,
+                      int r, int H, double* W_comb) {
+    cmref_shared_weight(U, S, Vh, d, r, H, W_comb);  /* W_shared in the first slot */
+    for (int e = E - 1; e >= 0; --e)                  /* the last slot first: slot 0 is read below */
+        for (int64_t i = 0; i < (int64_t)d * H; ++i) W_comb[(int64_t)e * d * H + i] = W_comb[i] + residuals[(int64_t)e * d * H + i];
+}
+
+/* Algorithm 2's residuals are scaled copies of one matrix, W_e^res = s_e R: y_t = W_shared z_t +
+ * s_{a_t} R z_t, with z from fc1 as in cmref_ffn_forward. Returns -1 on a bad expert index or an
+ * allocation failure. */
+int cmref_ffn_forward_scaled(const double* x, int64_t T, int d, int H, const double* W1, const double* b1,
+                             const double* U, const double* S, const double* Vh, int r, const double* R,
+                             const double* s, int E, const int32_t* a, int z_bf16, double* y) {
+    double* z = (double*)malloc(sizeof(double) * (size_t)H);
+    double* Wsh = (double*)malloc(sizeof(double) * (size_t)d * (size_t)H);
+    double* hsh = (double*)malloc(sizeof(double) * (size_t)d);
+    double* hr = (double*)malloc(sizeof(double) * (size_t)d);
+    int rc = -1;
+    if (!z || !Wsh || !hsh || !hr) goto done;
+    cmref_shared_weight(U, S, Vh, d, r, H, Wsh);
+    for (int64_t t = 0; t < T; ++t) {
+        if (a[t] < 0 || a[t] >= E) goto done;
+        cmref_fc1_gelu(x + t * d, 1, d, H, W1, b1, z_bf16, z);
+        matvec(Wsh, z, d, H, hsh);
+        matvec(R, z, d, H, hr);
+        for (int i = 0; i < d; ++i) y[t * d + i] = hsh[i] + s[a[t]] * hr[i];
+    }
+    rc = 0;
+done:
+    free(z);
+    free(Wsh);
+    free(hsh);
+    free(hr);
+    return rc;
 }

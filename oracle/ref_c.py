@@ -39,6 +39,9 @@ _SIGS = {
     "cmref_dense_ffn": (ctypes.c_int, [_D, ctypes.c_int64, ctypes.c_int, ctypes.c_int, _D, _D, _D, _D,
                                        ctypes.c_int, _D]),
     "cmref_layer_norm": (None, [_D, ctypes.c_int64, ctypes.c_int, ctypes.c_double, _D]),
+    "cmref_fold_basis": (None, [_D, _D, _D, _D, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, _D]),
+    "cmref_ffn_forward_scaled": (ctypes.c_int, [_D, ctypes.c_int64, ctypes.c_int, ctypes.c_int, _D, _D, _D, _D,
+                                                _D, ctypes.c_int, _D, _D, ctypes.c_int, _I, ctypes.c_int, _D]),
 }
 
 
@@ -176,3 +179,24 @@ def layer_norm(y, eps: float = 1e-6) -> np.ndarray:
     out = np.empty_like(y)
     lib().cmref_layer_norm(_p(y), T, d, float(eps), _p(out))
     return out
+
+
+def fold_basis(U, S, Vh, residuals) -> np.ndarray:
+    """W_comb[e] = W_shared + W_e^res for every expert."""
+    U, S, Vh, res = (_d(v) for v in (U, S, Vh, residuals))
+    E, d, H = res.shape
+    out = np.empty((E, d, H))
+    lib().cmref_fold_basis(_p(U), _p(S), _p(Vh), _p(res), E, d, S.shape[0], H, _p(out))
+    return out
+
+
+def ffn_forward_scaled(x, W1, b1, U, S, Vh, R, s, a, z_bf16: bool = False) -> np.ndarray:
+    """y_t = W_shared z_t + s_{a_t} R z_t (Algorithm 2's residuals W_e^res = s_e R)."""
+    x, W1, b1, U, S, Vh, R, s = (_d(v) for v in (x, W1, b1, U, S, Vh, R, s))
+    a32 = np.ascontiguousarray(a, dtype=np.int32)
+    T, d = x.shape
+    y = np.empty((T, d))
+    if lib().cmref_ffn_forward_scaled(_p(x), T, d, W1.shape[0], _p(W1), _p(b1), _p(U), _p(S), _p(Vh), S.shape[0],
+                                      _p(R), _p(s), s.shape[0], _pi(a32), int(z_bf16), _p(y)):
+        raise ValueError("bad expert index or allocation failure")
+    return y

@@ -150,3 +150,22 @@ def test_gpu_check_helper_on_the_numpy_oracle(dtype):
     y_bad = y.copy()
     y_bad[5, 3] += 1.0
     assert check_against_c_oracle(L, y_bad, gr) > 1e-2
+
+
+def test_folded_and_scaled_forms_match_numpy_oracle():
+    L = _layer(np.random.default_rng(8), 45, 16, 40, 3, 6)
+    a = C.route(L["x"], L["Wg"], L["bg"])["a"]
+    comb = C.fold_basis(L["U"], L["S"], L["Vh"], L["residuals"])
+    assert _rel(comb, O.fold_basis(L["U"], L["S"], L["Vh"], L["residuals"])) <= 1e-13
+    # the folded weights with a zero basis give the same layer as W_shared + residuals
+    y_fold = C.ffn_forward(L["x"], L["W1"], L["b1"], np.zeros((16, 1)), np.zeros(1), np.zeros((1, 40)), comb, a)
+    assert _rel(y_fold, C.ffn_forward(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], L["residuals"], a)) <= 1e-12
+    R = L["W2"] - C.shared_weight(L["U"], L["S"], L["Vh"])
+    s = np.array([0.5, 1.0, 2.0])
+    y = C.ffn_forward_scaled(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], R, s, a)
+    assert _rel(y, O.ffn_forward_scaled(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], R, s, a=a)) <= 1e-12
+    # with every s_e = 1 the residuals are W2 - W_shared and the layer is the dense FFN
+    y1 = C.ffn_forward_scaled(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], R, np.ones(3), a)
+    assert _rel(y1, C.dense_ffn(L["x"], L["W1"], L["b1"], L["W2"])) <= 1e-12
+    with pytest.raises(ValueError):
+        C.ffn_forward_scaled(L["x"], L["W1"], L["b1"], L["U"], L["S"], L["Vh"], R, s, np.full(45, 3))
