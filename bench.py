@@ -57,14 +57,19 @@ TRAFFIC = {
 def init_replicas(backend="nccl"):
     """One process per GPU (torchrun's RANK / WORLD_SIZE / LOCAL_RANK): (world, rank, local, dist),
     dist None for a single process. Each rank runs an independent replica on its own token shard;
-    the only collectives are the barriers and the max of the rank times."""
+    the only collectives are the barriers and the max of the rank times. A rank that dies between
+    steps is detected by the others at their next collective, which fails with an error within the
+    process group's timeout (CLEARMOE_PG_TIMEOUT_S seconds, default 600) instead of waiting forever."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     dist = None
     if world > 1:
+        import datetime
+
         import torch.distributed as dist
-        dist.init_process_group(backend)
+        timeout = datetime.timedelta(seconds=float(os.environ.get("CLEARMOE_PG_TIMEOUT_S", "600")))
+        dist.init_process_group(backend, timeout=timeout)
     return world, rank, local, dist
 
 

@@ -2,7 +2,9 @@
 over gloo, launched like torchrun launches them (RANK, WORLD_SIZE, LOCAL_RANK, MASTER_ADDR
 127.0.0.1). Each rank builds its own token shard (seed = rank) and routes it independently (the
 oracle stands in for the GPU path here); the only collectives are the barrier, the max of the rank
-times, and, for metrics only, an E-int sum of the expert counts."""
+times, and, for metrics only, an E-int sum of the expert counts. A rank that dies between steps
+makes the survivor's next collective fail with an error (gloo, a 20 s process-group timeout), so the
+job ends instead of hanging."""
 import multiprocessing as mp
 import os
 import socket
@@ -66,3 +68,37 @@ def test_single_process_needs_no_collective(monkeypatch):
     w, r, local, dist = bench.init_replicas("gloo")
     assert (w, r, dist) == (1, 0, None)
     assert bench.max_over_ranks(3.0, None) == 3.0
+
+
+def _dying_rank(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank), CLEARMOE_PG_TIMEOUT_S="20")
+    import time
+
+    import bench
+
+    w, r, local, dist = bench.init_replicas("gloo")
+    if r == 1:
+        os._exit(3)  # dies between steps: no collective of its own in flight
+    t0 = time.time()
+    try:
+        bench.max_over_ranks(1.0, dist, device="cpu")
+        q.put(("completed", time.time() - t0))
+    except Exception as exc:  # the failure reaches the survivor as an error, not a hang
+        q.put((type(exc).__name__, time.time() - t0))
+    os._exit(0)
+
+
+def test_a_dead_rank_fails_the_next_collective():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_dying_rank, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    outcome, waited = q.get(timeout=300)
+    for p in procs:
+        p.join(timeout=60)
+    assert procs[1].exitcode == 3
+    assert outcome != "completed", "the survivor's collective completed without its peer"
+    assert waited < 60, f"the survivor learned of the failure only after {waited:.0f} s"
