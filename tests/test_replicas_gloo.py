@@ -77,15 +77,19 @@ def _dying_rank(rank, world, port, q):
 
     import bench
 
-    w, r, local, dist = bench.init_replicas("gloo")
-    if r == 1:
-        os._exit(3)  # dies between steps: no collective of its own in flight
-    t0 = time.time()
     try:
-        bench.max_over_ranks(1.0, dist, device="cpu")
-        q.put(("completed", time.time() - t0))
-    except Exception as exc:  # the failure reaches the survivor as an error, not a hang
-        q.put((type(exc).__name__, time.time() - t0))
+        w, r, local, dist = bench.init_replicas("gloo")
+        dist.barrier()  # one step completed by both ranks
+        if r == 1:
+            os._exit(3)  # dies between steps: no collective of its own in flight
+        t0 = time.time()
+        try:
+            bench.max_over_ranks(1.0, dist, device="cpu")
+            q.put(("completed", time.time() - t0))
+        except Exception as exc:  # the failure reaches the survivor as an error, not a hang
+            q.put((type(exc).__name__, time.time() - t0))
+    except Exception as exc:
+        q.put((f"setup failed: {exc!r}", -1.0))
     os._exit(0)
 
 
@@ -96,9 +100,15 @@ def test_a_dead_rank_fails_the_next_collective():
     procs = [ctx.Process(target=_dying_rank, args=(r, 2, port, q)) for r in range(2)]
     for p in procs:
         p.start()
-    outcome, waited = q.get(timeout=300)
-    for p in procs:
-        p.join(timeout=60)
+    try:
+        outcome, waited = q.get(timeout=120)
+    finally:
+        for p in procs:
+            p.join(timeout=30)
+            if p.is_alive():  # only this test's own children
+                p.kill()
+                p.join()
+    assert not outcome.startswith("setup failed"), outcome
     assert procs[1].exitcode == 3
     assert outcome != "completed", "the survivor's collective completed without its peer"
     assert waited < 60, f"the survivor learned of the failure only after {waited:.0f} s"
