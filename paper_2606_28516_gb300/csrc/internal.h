@@ -213,6 +213,12 @@ int tc2_pick_bn(int mode, int N);
 cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_tc_gemm(const TcGemmArgs& a, int num_sms, cudaStream_t s);
 
+// cudaFuncSetAttribute(fn, MaxDynamicSharedMemorySize, bytes) once per (current device, fn): the
+// attribute belongs to a device, so a process that launches on several GPUs sets it on each.
+cudaError_t smem_attr_once(const void* fn, int bytes);
+// SM count of the current device, queried once per device (0 on a CUDA error).
+int current_device_sms();
+
 // Encode a 2-D bf16 row-major [rows x cols] tensor map, box {64, box_rows}, 128-byte swizzle.
 int encode_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols,
                      int box_rows);

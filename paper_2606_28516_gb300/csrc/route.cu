@@ -574,27 +574,30 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
     int64_t want = (int64_t)num_sms * (bf16 ? 1 : 2);  // bf16: one CTA per SM owns the ring
     // equal ranges over all CTAs (a range's last 16-row stage may be partial)
     int64_t ch = (T + want - 1) / want;
+    // the shared-memory attribute belongs to a device: set once per device
+    if (smem_attr_once((const void*)route_kernel<true, false>, (int)RT_SMEM_MAX) != cudaSuccess ||
+        smem_attr_once((const void*)route_kernel<true, true>, (int)RT_SMEM_MAX) != cudaSuccess ||
+        smem_attr_once((const void*)route_kernel<false, false>, (int)RT_SMEM_MAX) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return -1;
+    }
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return -1;
+    }
     static std::mutex mu;
     std::lock_guard<std::mutex> lock(mu);
-    static bool attr_set = false;
-    if (!attr_set) {
-            if (cudaFuncSetAttribute((const void*)route_kernel<true, false>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 220 * 1024) != cudaSuccess ||
-            cudaFuncSetAttribute((const void*)route_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 220 * 1024) != cudaSuccess ||
-            cudaFuncSetAttribute((const void*)route_kernel<false, false>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 220 * 1024) != cudaSuccess)
-            return -1;
-        attr_set = true;
-    }
-    // occupancy queries are cached: (dtype, d, E, shared-memory bytes) -> CTAs per SM
-    static struct { int dtype, d, E; size_t smem; int occ; } cache[32];
+    // occupancy queries are cached: (device, dtype, d, E, shared-memory bytes) -> CTAs per SM
+    static struct { int dev, dtype, d, E; size_t smem; int occ; } cache[64];
     static int ncache = 0;
     for (int iter = 0; iter < 4; ++iter) {
         const size_t smem = route_smem(dtype, d, E, (int)ch);
         occ = -1;
         for (int i = 0; i < ncache; ++i)
-            if (cache[i].dtype == dtype && cache[i].d == d && cache[i].E == E && cache[i].smem == smem) occ = cache[i].occ;
+            if (cache[i].dev == dev && cache[i].dtype == dtype && cache[i].d == d && cache[i].E == E &&
+                cache[i].smem == smem)
+                occ = cache[i].occ;
         if (occ < 0) {
             const void* fn = !bf16 ? (const void*)route_kernel<false, false>
                              : route_wreg(dtype, d, E) ? (const void*)route_kernel<true, true>
@@ -602,7 +605,7 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
             cudaError_t err = cudaOccupancyMaxActiveBlocksPerMultiprocessorWithFlags(
                 &occ, fn, bf16 ? RT_BF16_THREADS : RT_THREADS, smem, cudaOccupancyDefault);
             if (err != cudaSuccess) return -1;
-            if (ncache < 32) cache[ncache++] = {dtype, d, E, smem, occ};
+            if (ncache < 64) cache[ncache++] = {dev, dtype, d, E, smem, occ};
         }
         if (occ <= 0) return -2;
         const int64_t maxg = (int64_t)occ * num_sms;

@@ -152,13 +152,8 @@ static int64_t simt_blocks(const SimtGemmArgs& a, int* n_tiles_n) {
 }
 
 cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
-    static int num_sms = 0;
-    if (!num_sms) {
-        int dev = 0;
-        if (cudaGetDevice(&dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-            num_sms = 1;
-    }
+    int num_sms = current_device_sms();  // per device, cached
+    if (num_sms <= 0) num_sms = 1;
     int n64 = 0, n32 = 0;
     const int64_t b64 = simt_blocks<64>(a, &n64), b32 = simt_blocks<32>(a, &n32);
     if (b64 <= 0) return cudaSuccess;

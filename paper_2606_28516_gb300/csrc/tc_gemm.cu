@@ -427,13 +427,8 @@ int tc_pick_bn(int mode, int N) {
 template <int BN, int MODE>
 static cudaError_t launch_one(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     using C = TcCfg<BN>;
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<BN, MODE>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+    const cudaError_t e = smem_attr_once((const void*)tc_gemm_kernel<BN, MODE>, C::SMEM);
+    if (e != cudaSuccess) return e;
     const int n_tiles = a.N / BN;
     int64_t m_tiles = (a.M + TC_BM - 1) / TC_BM;
     if (MODE == TC_GROUPED) m_tiles += a.E;
@@ -471,6 +466,54 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     if (a.mode == TC_GATHER) return launch_mode<TC_GATHER>(a, bn, num_sms, s);
     if (a.mode == TC_GROUPED) return launch_mode<TC_GROUPED>(a, bn, num_sms, s);
     return launch_mode<TC_DENSE>(a, bn, num_sms, s);
+}
+
+namespace {
+constexpr int kMaxDevices = 64;
+struct AttrEntry {
+    int dev;
+    const void* fn;
+    int bytes;
+};
+std::mutex g_attr_mu;
+AttrEntry g_attr[256];
+int g_nattr = 0;
+int g_sms[kMaxDevices] = {};
+}  // namespace
+
+cudaError_t smem_attr_once(const void* fn, int bytes) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(g_attr_mu);
+    for (int i = 0; i < g_nattr; ++i)
+        if (g_attr[i].dev == dev && g_attr[i].fn == fn && g_attr[i].bytes >= bytes) return cudaSuccess;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    for (int i = 0; i < g_nattr; ++i)
+        if (g_attr[i].dev == dev && g_attr[i].fn == fn) {
+            g_attr[i].bytes = bytes;
+            return cudaSuccess;
+        }
+    if (g_nattr < 256) g_attr[g_nattr++] = AttrEntry{dev, fn, bytes};  // else set again on every call
+    return cudaSuccess;
+}
+
+int current_device_sms() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return 0;
+    }
+    std::lock_guard<std::mutex> lock(g_attr_mu);
+    if (dev >= 0 && dev < kMaxDevices && g_sms[dev]) return g_sms[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return 0;
+    }
+    if (dev >= 0 && dev < kMaxDevices) g_sms[dev] = n;
+    return n;
 }
 
 typedef CUresult (*PFN_encodeTiled_t)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,

@@ -611,14 +611,10 @@ int tc2_pick_bn(int mode, int N) {
 template <int BN>
 static cudaError_t launch2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     using C = T2<BN>;
-    static bool attr[3] = {false, false, false};
     const void* fn = a.mode == TC_GROUPED ? (const void*)tc_gemm2_kernel<BN, TC_GROUPED>
                                           : (const void*)tc_gemm2_kernel<BN, TC_DENSE>;
-    if (!attr[a.mode]) {
-        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-        if (e != cudaSuccess) return e;
-        attr[a.mode] = true;
-    }
+    const cudaError_t e = smem_attr_once(fn, C::SMEM);
+    if (e != cudaSuccess) return e;
     const int n_tiles = a.N / BN;
     int64_t m_pairs = (a.M + 2 * C::BM - 1) / (2 * C::BM);
     if (a.mode == TC_GROUPED) m_pairs += a.E;

@@ -90,6 +90,10 @@ def _dying_rank(rank, world, port, q):
             q.put((type(exc).__name__, time.time() - t0))
     except Exception as exc:
         q.put((f"setup failed: {exc!r}", -1.0))
+    # os._exit skips the queue's feeder thread: flush the message to the pipe first, or the
+    # parent may never receive it
+    q.close()
+    q.join_thread()
     os._exit(0)
 
 
