@@ -101,11 +101,13 @@ VIT_BASE_STACK12 = StackShape()
 def round_bf16(a: np.ndarray) -> np.ndarray:
     """Round to the nearest bf16 (ties to even); returns float32 holding bf16 values."""
     f = np.array(a, dtype=np.float32, copy=True, order="C")
-    u = f.view(np.uint32)
-    lsb = (u >> 16) & 1
-    u += np.uint32(0x7FFF)
-    u += lsb
-    u &= np.uint32(0xFFFF0000)
+    u = f.reshape(-1).view(np.uint32)
+    for s in range(0, u.size, 1 << 22):  # in place, in chunks (elementwise: same bits)
+        v = u[s:s + (1 << 22)]
+        lsb = (v >> 16) & 1
+        v += np.uint32(0x7FFF)
+        v += lsb
+        v &= np.uint32(0xFFFF0000)
     return f
 
 
@@ -146,10 +148,16 @@ def residual_stream(x: np.ndarray, dtype: str, seed: int = 7, scale=(0.5, 4.0), 
 
 
 def mixture_tokens(rng: np.random.Generator, centroids: np.ndarray, sizes: np.ndarray,
-                   sigma: float):
+                   sigma: float, chunk: int = 65536):
+    """Tokens mu_label + sigma N(0, I), layer-normalised. Drawn in row chunks: consecutive draws
+    continue the generator's stream, so the values equal one draw of the whole matrix while the
+    temporaries stay small."""
     labels = rng.permutation(np.repeat(np.arange(len(sizes)), sizes))
-    x = centroids[labels] + sigma * rng.standard_normal((labels.size, centroids.shape[1]))
-    return layer_norm(x), labels
+    x = np.empty((labels.size, centroids.shape[1]), dtype=np.float64)
+    for s in range(0, labels.size, chunk):
+        lab = labels[s:s + chunk]
+        x[s:s + chunk] = layer_norm(centroids[lab] + sigma * rng.standard_normal((lab.size, centroids.shape[1])))
+    return x, labels
 
 
 def _gelu32(u: np.ndarray) -> np.ndarray:

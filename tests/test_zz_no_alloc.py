@@ -2,7 +2,9 @@
 (engines that own every device byte, fixed memory budgets, loops that cannot afford cudaMalloc's
 device synchronisation): it keeps its scratch in a static device array instead of a handle's
 workspace. Checked through the C ABI against clearmoe_route, bit-exactly, on two calls in a row
-that reuse the same scratch (the second with a different token count and expert count).
+that reuse the same scratch (the second with a different token count and expert count), on the fp32
+routing kernel with and without a status word; tests/test_gpu_large_tokens.py runs it at 600,000
+tokens, where the per-row words live in the caller's idx between the two kernels.
 This file is collected last on purpose, so a failure here leaves every other test already run."""
 import numpy as np
 import pytest
@@ -43,6 +45,25 @@ def test_route_noalloc_matches_route_twice():
         cm.clearmoe_route_noalloc(x, D["Wg"], D["bg"], *got, status=status)
         torch.cuda.synchronize()
         assert int(status.item()) == 0
+        for g, w, name in zip(got, want, ("idx", "counts", "offsets", "perm")):
+            assert np.array_equal(g.cpu().numpy(), w), name
+
+
+def test_route_noalloc_fp32_and_without_status_word():
+    """The fp32 routing kernel (two CTAs per SM, one token per lane) through the same entry point,
+    once with a status word and once without one (the array's spare word takes the status then),
+    bit for bit against the handle's routing."""
+    import __graft_entry__
+    __graft_entry__.build()
+    L = synth.make_layer(synth.DEIT_TINY_FP32)
+    s = L["shape"]
+    x, D, want = _handle_routing(L, s.T)
+    for status in (torch.full((1,), -7, dtype=torch.int32, device="cuda"), None):
+        got = [torch.full((n,), -7, dtype=torch.int32, device="cuda") for n in (s.T, s.E, s.E + 1, s.T)]
+        cm.clearmoe_route_noalloc(x, D["Wg"], D["bg"], *got, status=status)
+        torch.cuda.synchronize()
+        if status is not None:
+            assert int(status.item()) == 0
         for g, w, name in zip(got, want, ("idx", "counts", "offsets", "perm")):
             assert np.array_equal(g.cpu().numpy(), w), name
 
