@@ -742,8 +742,21 @@ def main():
         return {"value": whole_job_rate(s.T, world, 1, v_ms), "unit": "tokens/s", "ms_per_step": v_ms,
                 "note": note}
 
-    folded = materialized = class_tokens = mlp_router = scaled = layernorm = None
+    folded = materialized = class_tokens = mlp_router = scaled = layernorm = router_in_fc1 = None
     if s.dtype == "bf16" and not args.no_variants:
+        fused = lambda: cm.clearmoe_ffn_forward_ex(h, D["x"], D["W1"], D["b1"], D["U"], D["S"], D["Vh"],
+                                                   D["residuals"], D["Wg"], D["bg"], out, router_in_fc1=True)
+        router_in_fc1 = time_variant(
+            fused, "the router's logits inside fc1 (one 256 x 32 MMA unit per 256-token tile on the x tiles "
+                   "fc1 loads), a slot kernel over 128-token ranges, t stored at the slots, z rows gathered "
+                   "by perm in the grouped GEMM (TMA four-row gathers)")
+        fst = stage_pass(cm, h, fused, min(K, 300), flush)
+        router_in_fc1["stages_us"] = {name: statistics.mean(v) * 1e3 for name, v in
+                                      zip(("fc1_with_router", "slots", "basis", "grouped"), fst.values())}
+        fw = stage_work(s)
+        router_in_fc1["stages_us"]["fc1_with_router_tensor_frac"] = (
+            (fw["fc1_gelu"]["flops"] + fw["route"]["flops"]) / (router_in_fc1["stages_us"]["fc1_with_router"] * 1e-6)
+            / 1e12 / pk["bf16_tflops"])
         W_comb = torch.empty_like(D["residuals"])
         cm.clearmoe_fold_basis(h, D["U"], D["S"], D["Vh"], D["residuals"], W_comb)
         folded = time_variant(
@@ -939,6 +952,7 @@ def main():
         "mlp_router": mlp_router,
         "scaled_residual": scaled,
         "input_layernorm": layernorm,
+        "router_in_fc1": router_in_fc1,
         "configs": configs,
         "wall_s_timed": wall,
     }

@@ -149,13 +149,26 @@ int clearmoe_ffn_forward(clearmoe_layer* layer, const void* x, int64_t T, const 
  *              block's LN affine folds into W1, b1 and the router offline). LN(y) is never
  *              written: one launch forms (mean, rstd) per token and the row sums c = W 1 of W1 and
  *              of the router's first matrix (W_g, or the MLP router's W_in), and the router and fc1
- *              use W LN(y) = rstd (W y - mean c) on their fp32 accumulators. 0: x is the input. */
+ *              use W LN(y) = rstd (W y - mean c) on their fp32 accumulators. 0: x is the input.
+ *  router_in_fc1  non-zero: the linear router's logits (Phase 4 "Linear", Algorithm 3 step 3) are
+ *              computed inside fc1 from the token tiles fc1 has already loaded (one more 256 x 32
+ *              MMA unit per 256-token tile, W_g as its B operand), so the tokens are read from HBM
+ *              once for both; fc1 stores z in token order, a slot kernel forms counts, offsets,
+ *              perm and inv from per-128-token-range counts and ranks, the basis factor stores t at
+ *              each token's slot, and the grouped GEMM gathers z rows by perm (TMA four-row
+ *              gathers). Same results as the default path (expert indices bit-exact outside near
+ *              ties, outputs within the tolerance). bf16 layers with the 2-SM kernels only (H a
+ *              multiple of 128 and <= 4096, d a multiple of 128), the linear router, and neither
+ *              class tokens, the MLP router, input_layernorm nor the materialised basis:
+ *              EUNSUPPORTED otherwise. Works with clearmoe_ffn_forward_ex (factorised basis) and
+ *              clearmoe_ffn_forward_folded_ex. */
 typedef struct {
     const void* b2;
     int64_t cls_stride;
     const void* W2;
     const clearmoe_mlp_router* mlp_router; /* non-NULL: routes with it (router may then be NULL) */
     int32_t input_layernorm;
+    int32_t router_in_fc1;
 } clearmoe_ffn_options;
 
 /* clearmoe_ffn_forward with deployment options (opt may be NULL: then identical to it). With

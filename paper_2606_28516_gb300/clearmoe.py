@@ -39,7 +39,8 @@ class clearmoe_mlp_router(ctypes.Structure):
 
 class clearmoe_ffn_options(ctypes.Structure):
     _fields_ = [("b2", ctypes.c_void_p), ("cls_stride", ctypes.c_int64), ("W2", ctypes.c_void_p),
-                ("mlp_router", ctypes.POINTER(clearmoe_mlp_router)), ("input_layernorm", ctypes.c_int32)]
+                ("mlp_router", ctypes.POINTER(clearmoe_mlp_router)), ("input_layernorm", ctypes.c_int32),
+                ("router_in_fc1", ctypes.c_int32)]
 
 
 ACT_RELU, ACT_GELU = 0, 1
@@ -179,14 +180,16 @@ def clearmoe_ffn_forward(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, 
 
 def clearmoe_ffn_forward_ex(layer: int, x, W1, b1, U_r, S_r, Vh_r, residual_e, Wg, bg, out,
                             b2=None, W2=None, cls_stride: int = 0, mlp: clearmoe_mlp_router | None = None,
-                            E: int | None = None, input_layernorm: bool = False, stream=None) -> None:
+                            E: int | None = None, input_layernorm: bool = False, router_in_fc1: bool = False,
+                            stream=None) -> None:
     """clearmoe_ffn_forward with fc2's bias b2, class tokens (every cls_stride-th token from token 0)
-    on the dense path W2, the MLP router `mlp` (then Wg, bg may be None and E is given), and
-    input_layernorm (x is the un-normalised stream y; the layer's input is LN(y))."""
+    on the dense path W2, the MLP router `mlp` (then Wg, bg may be None and E is given),
+    input_layernorm (x is the un-normalised stream y; the layer's input is LN(y)), and
+    router_in_fc1 (the linear router's logits computed inside fc1)."""
     E = Wg.shape[0] if E is None else E
     res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
     r = _router(Wg, bg) if Wg is not None else None
-    opt = _options(b2, W2, cls_stride, mlp, input_layernorm)
+    opt = _options(b2, W2, cls_stride, mlp, input_layernorm, router_in_fc1)
     _check(lib().clearmoe_ffn_forward_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), _ptr(U_r),
                                          _ptr(S_r), _ptr(Vh_r), res, ctypes.byref(r) if r else None, E,
                                          S_r.shape[0], ctypes.byref(opt), _ptr(out),
@@ -235,18 +238,20 @@ def clearmoe_ffn_forward_scaled(layer: int, x, W1, b1, U_r, S_r, Vh_r, R, s_e, W
            "clearmoe_ffn_forward_scaled")
 
 
-def _options(b2, W2, cls_stride, mlp, input_layernorm=False):
+def _options(b2, W2, cls_stride, mlp, input_layernorm=False, router_in_fc1=False):
     return clearmoe_ffn_options(_ptr(b2), int(cls_stride), _ptr(W2),
-                                ctypes.pointer(mlp) if mlp is not None else None, int(bool(input_layernorm)))
+                                ctypes.pointer(mlp) if mlp is not None else None, int(bool(input_layernorm)),
+                                int(bool(router_in_fc1)))
 
 
 def clearmoe_ffn_forward_folded_ex(layer: int, x, W1, b1, W_comb, Wg, bg, out, b2=None, W2=None,
                                    cls_stride: int = 0, mlp: clearmoe_mlp_router | None = None,
-                                   E: int | None = None, input_layernorm: bool = False, stream=None) -> None:
+                                   E: int | None = None, input_layernorm: bool = False,
+                                   router_in_fc1: bool = False, stream=None) -> None:
     E = Wg.shape[0] if E is None else E
     comb = (ctypes.c_void_p * E)(*[_ptr(W_comb[e]) for e in range(E)])
     r = _router(Wg, bg) if Wg is not None else None
-    opt = _options(b2, W2, cls_stride, mlp, input_layernorm)
+    opt = _options(b2, W2, cls_stride, mlp, input_layernorm, router_in_fc1)
     _check(lib().clearmoe_ffn_forward_folded_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1), comb,
                                                 ctypes.byref(r) if r else None, E, ctypes.byref(opt),
                                                 _ptr(out), _stream(stream)), "clearmoe_ffn_forward_folded_ex")
@@ -255,11 +260,12 @@ def clearmoe_ffn_forward_folded_ex(layer: int, x, W1, b1, W_comb, Wg, bg, out, b
 def clearmoe_ffn_forward_materialized_ex(layer: int, x, W1, b1, W_sh, residual_e, Wg, bg, out, b2=None,
                                          W2=None, cls_stride: int = 0,
                                          mlp: clearmoe_mlp_router | None = None, E: int | None = None,
-                                         input_layernorm: bool = False, stream=None) -> None:
+                                         input_layernorm: bool = False, router_in_fc1: bool = False,
+                                         stream=None) -> None:
     E = Wg.shape[0] if E is None else E
     res = (ctypes.c_void_p * E)(*[_ptr(residual_e[e]) for e in range(E)])
     r = _router(Wg, bg) if Wg is not None else None
-    opt = _options(b2, W2, cls_stride, mlp, input_layernorm)
+    opt = _options(b2, W2, cls_stride, mlp, input_layernorm, router_in_fc1)
     _check(lib().clearmoe_ffn_forward_materialized_ex(layer, _ptr(x), x.shape[0], _ptr(W1), _ptr(b1),
                                                       _ptr(W_sh), res, ctypes.byref(r) if r else None, E,
                                                       ctypes.byref(opt), _ptr(out), _stream(stream)),

@@ -281,7 +281,11 @@ int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out)
         return CLEARMOE_ECUDA;
     }
     const size_t T = (size_t)D.max_tokens;
-    const size_t ncta = (size_t)cm::route_max_ctas(L->num_sms, D.dtype, D.d, D.max_E);
+    // per-range histograms: the routing kernel's ranges, or the 128-row ranges of the router
+    // inside fc1, whichever are more
+    size_t ncta = (size_t)cm::route_max_ctas(L->num_sms, D.dtype, D.d, D.max_E);
+    const size_t nfr = (T + cm::FR_RANGE - 1) / cm::FR_RANGE;
+    if (nfr > ncta) ncta = nfr;
     bool ok = cudaMalloc(&L->z, T * D.hidden * L->esz) == cudaSuccess &&
               cudaMalloc(&L->t, T * D.max_r * L->esz) == cudaSuccess &&
               cudaMalloc((void**)&L->idx, T * 4) == cudaSuccess &&
@@ -342,6 +346,129 @@ int clearmoe_route_mlp(clearmoe_layer* L, const void* x, int64_t T, const clearm
     return do_finalize(L, s);
 }
 
+// The router inside fc1 (clearmoe_ffn_options.router_in_fc1), bf16 layers: fc1 runs in token
+// order and every 256-row pair tile gets one more unit that multiplies the same x tiles by W_g, so
+// the tokens are read once for both; its epilogue writes idx, each token's rank within its 128-row
+// range and every range's expert counts. The slot kernel (route_finalize_kernel over those ranges)
+// forms counts, offsets, perm and inv; the basis factor reads z in token order and stores each t
+// row at its token's slot; the grouped GEMM gathers each expert's z rows by perm (four rows per TMA
+// gather) and scatters its output rows back to token order, as in the default path.
+static int ffn_router_in_fc1(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
+                             const void* U_r, const float* S_r, const void* Vh_r, const void* const* residual_e,
+                             const clearmoe_router* router, int E, int r, const void* b2, void* out,
+                             cudaStream_t s) {
+    const bool factored = U_r != nullptr;
+    const int d = L->desc.d, H = L->desc.hidden;
+    const int p1 = H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;
+    const int p3 = cm::tc2_pick_bn(cm::TC_GROUPED, d);
+    const int p2 = factored ? cm::tc2_pick_bn(cm::TC_DENSE, r) : 0;
+    const int bn2 = factored ? cm::tc_pick_bn(cm::TC_DENSE, r) : 1;
+    if (L->desc.dtype != CLEARMOE_BF16 || !p1 || !p3 || !bn2) return CLEARMOE_EUNSUPPORTED;
+    const int G = (int)((T + cm::FR_RANGE - 1) / cm::FR_RANGE);  // 128-row ranges
+    int rc;
+    mark(L, 0, s);
+    cm::TcGemmArgs g;
+    std::memset(&g, 0, sizeof(g));
+    g.status = L->status;
+    g.wait_limit_ns = L->wait_limit_ns;
+    if (encode_tmap_bf16(&g.tmA0, x, T, d, 128) || encode_tmap_bf16(&g.tmB0, W1, H, d, p1 / 2) ||
+        encode_tmap_bf16(&g.tmR, router->W, E, d, 16))
+        return CLEARMOE_ECUDA;
+    g.mode = cm::TC_DENSE;
+    g.epi = cm::TC_EPI_BIAS_GELU;
+    g.M = T;
+    g.N = H;
+    g.K0 = d;
+    g.bias = b1;
+    g.C = L->z;  // token order
+    g.ldc = H;
+    g.fr_E = E;
+    g.fr_bias = router->b;
+    g.fr_idx = L->idx;
+    g.fr_info = L->tinfo;
+    g.fr_counts = L->cta_counts;
+    g.pdl_wait_role = 0;  // x may be the previous kernel's output
+    if ((rc = cuda_fail(cm::launch_tc_gemm2(g, L->num_sms, s)))) return rc;
+    mark(L, 1, s);
+    cm::RouteArgs& a = L->rt;  // the slots from the 128-row ranges
+    std::memset(&a, 0, sizeof(a));
+    a.T = T;
+    a.d = d;
+    a.E = E;
+    a.dtype = CLEARMOE_BF16;
+    a.idx = L->idx;
+    a.perm = L->perm;
+    a.inv = L->inv;
+    a.counts = L->counts;
+    a.offsets = L->offsets;
+    a.cta_counts = L->cta_counts;
+    a.tinfo = L->tinfo;
+    a.debug_skip = -1;
+    a.wait_limit_ns = L->wait_limit_ns;
+    a.status = L->status;
+    L->rt_grid = G;
+    L->rt_chunk = cm::FR_RANGE;
+    if ((rc = cuda_fail(cm::launch_route_finalize(a, G, cm::FR_RANGE, s)))) return rc;
+    L->last_T = T;
+    L->last_E = E;
+    L->last_groups = E;
+    mark(L, 2, s);
+    if (factored) {  // t = diag(S_r) Vh_r z, z in token order, each t row stored at its slot (inv)
+        cm::TcGemmArgs g2;
+        std::memset(&g2, 0, sizeof(g2));
+        g2.status = L->status;
+        g2.wait_limit_ns = L->wait_limit_ns;
+        if (encode_tmap_bf16(&g2.tmA0, L->z, T, H, 128) || encode_tmap_bf16(&g2.tmB0, Vh_r, r, H, p2 ? p2 / 2 : bn2))
+            return CLEARMOE_ECUDA;
+        g2.mode = cm::TC_DENSE;
+        g2.epi = cm::TC_EPI_SCALE;
+        g2.M = T;
+        g2.N = r;
+        g2.K0 = H;
+        g2.scale = S_r;
+        g2.C = L->t;
+        g2.ldc = r;
+        g2.rows = L->inv;
+        g2.a_evict_first = 1;
+        // z is complete once the slot kernel releases this one (it waits for fc1 first): the loads
+        // and MMAs start at once, the epilogue waits for the slots
+        g2.pdl_wait_role = 1;
+        g2.pdl_trigger_late = 1;
+        rc = cuda_fail(p2 ? cm::launch_tc_gemm2(g2, L->num_sms, s) : cm::launch_tc_gemm(g2, L->num_sms, s));
+        if (rc) return rc;
+    }
+    mark(L, 3, s);
+    cm::TcGemmArgs g3;
+    std::memset(&g3, 0, sizeof(g3));
+    g3.status = L->status;
+    g3.wait_limit_ns = L->wait_limit_ns;
+    const int box3 = p3 / 2;
+    if ((factored && (encode_tmap_bf16(&g3.tmA0, L->t, T, r, 128) || encode_tmap_bf16(&g3.tmB0, U_r, d, r, box3))) ||
+        encode_tmap_bf16(&g3.tmA1, L->z, T, H, 1))  // one-row boxes: the z rows are gathered
+        return CLEARMOE_ECUDA;
+    for (int e = 0; e < E; ++e)
+        if (encode_tmap_bf16(&g3.tmB1[e], residual_e[e], d, H, box3)) return CLEARMOE_ECUDA;
+    g3.out_bias = b2;
+    // after the basis kernel (released once the slots exist) the z segments may start at once; with
+    // no basis kernel the slot kernel precedes this one and every thread waits for it
+    g3.pdl_wait_role = factored ? 2 : 0;
+    g3.mode = cm::TC_GROUPED;
+    g3.epi = cm::TC_EPI_SCATTER;
+    g3.M = T;
+    g3.N = d;
+    g3.K0 = factored ? r : 0;
+    g3.K1 = H;
+    g3.offsets = L->offsets;
+    g3.E = E;
+    g3.rows = L->perm;
+    g3.a1_rows = L->perm;
+    g3.C = out;
+    g3.ldc = d;
+    rc = cuda_fail(cm::launch_tc_gemm2(g3, L->num_sms, s));
+    mark(L, 4, s);
+    return rc;
+}
+
 static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
                     const void* U_r, const float* S_r, const void* Vh_r, const void* W_sh,
                     const void* const* residual_e, const clearmoe_router* router, int E, int r,
@@ -360,6 +487,10 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     const void* b2 = opt ? opt->b2 : nullptr;
     const clearmoe_mlp_router* mlp = opt ? opt->mlp_router : nullptr;
     const bool ln = opt && opt->input_layernorm;  // x is y: LN(y) folded into the router and fc1
+    if (opt && opt->router_in_fc1) {  // the linear router only, no class tokens, no folded LayerNorm
+        if (mlp || cls_stride > 0 || ln || materialized) return CLEARMOE_EUNSUPPORTED;
+        return ffn_router_in_fc1(L, x, T, W1, b1, U_r, S_r, Vh_r, residual_e, router, E, r, b2, out, s);
+    }
     int rc;
     mark(L, 0, s);
     if (ln && (rc = ln_prep(L, x, T, W1, mlp ? mlp->W_in : router->W, mlp ? mlp->hidden : E, s))) return rc;

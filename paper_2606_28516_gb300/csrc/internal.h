@@ -188,7 +188,24 @@ struct TcGemmArgs {
     // with ln_stats set and ln_colsum null the epilogue then only scales by rstd, inside the bias
     // add (BIAS_GELU / BIAS_RELU)
     int ln_aug;
+    // 2-SM dense kernel: the linear router inside fc1 (fr_E > 0, E <= 16). Every 256-row pair tile
+    // gets one more unit whose B is W_g (tmR: [E x K0], boxes of 16 rows, rows past E read as zero)
+    // and whose MMA is 256 x 32 over the same A tiles; its epilogue adds b_g (fr_bias, bf16), takes
+    // the argmax (lowest index on ties) and writes, per token t, fr_idx[t] = e and fr_info[t] =
+    // e | rank << 8 (rank among the earlier tokens of e in t's 128-row range t / 128), and per range
+    // c the expert counts fr_counts[c * CM_MAX_E + e] (ranges c < ceil(M / 128)).
+    CUtensorMap tmR;
+    int fr_E;
+    const void* fr_bias;
+    int32_t* fr_idx;
+    int32_t* fr_info;
+    int32_t* fr_counts;
+    // grouped mode: the z segment's A rows gathered by slot, A row of slot m = a1_rows[m] (perm),
+    // by tile::gather4 loads of four rows each; tmA1 then has boxes one row high
+    const int32_t* a1_rows;
 };
+// Rows of one routing range of the router inside fc1 (a CTA's half of a pair tile).
+constexpr int FR_RANGE = 128;
 // Boundary e of a grouped GEMM's groups: offsets[e], or the single group [0, M) without offsets.
 __host__ __device__ inline int64_t tc_group_off(const TcGemmArgs& a, int e) {
     return a.offsets ? (int64_t)a.offsets[e] : (e == 0 ? 0 : a.M);

@@ -296,7 +296,9 @@ __global__ void __launch_bounds__(MODE == TC_GATHER ? TC_THREADS_GATHER : TC_THR
             tc_fence_after();
             const int r = q * 32 + lane;
             int64_t orow = -1;
-            if (r < t.rows) orow = (a.epi == TC_EPI_SCATTER) ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
+            // rows scattered by the grouped epilogue, or by a dense GEMM given a row map (t at its slot)
+            if (r < t.rows)
+                orow = (a.epi == TC_EPI_SCATTER || (a.mode == TC_DENSE && a.rows)) ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
             const float rsc = (a.group_scale && r < t.rows) ? tc_row_scale(a, t.m0 + r) : 1.f;
             if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;
             // the LayerNorm folded into A: (mean, rstd) of the token whose row this lane holds

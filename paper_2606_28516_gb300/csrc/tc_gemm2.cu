@@ -44,7 +44,8 @@ struct T2 {
     static constexpr int STG_BYTES = NUM_EPI * 32 * STG_ROW;
     static constexpr int BIAS_CAP = TC2_BIAS_CAP;         // fp32 bias / scale staged in shared memory
     static constexpr int TAB_CAP = TC2_TAB_CAP;           // routing prefix table (fused fc1)
-    static constexpr int NBARS = 2 * STAGES + 5;
+    static constexpr int NBARS = 2 * STAGES + 7;  // + 2 for the router inside fc1
+    static constexpr int FR_B_BYTES = 16 * BK * 2;        // the router unit's B box per CTA: 16 rows of W_g
     static constexpr int SMEM =
         1024 + STAGES * STAGE_BYTES + STG_BYTES + BIAS_CAP * 4 + (TAB_CAP + CM_MAX_E) * 4 + NBARS * 8 + 128;
     static constexpr int TMEM_COLS = 2 * BN <= 256 ? 256 : 512;  // two accumulators (a power of 2)
@@ -79,6 +80,16 @@ __device__ __forceinline__ void tma_load_2d_pair_hint(uint32_t dst, const CUtens
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar_cluster), "l"(policy)
         : "memory");
 }
+// Four rows (r0..r3, one row high boxes of 64 bf16 each) of a 2-D tensor into 512 contiguous bytes
+// of shared memory, in the layout a four-row box would have there; completion on the even CTA's barrier.
+__device__ __forceinline__ void tma_gather4_pair(uint32_t dst, const CUtensorMap* map, int32_t c0, int32_t r0,
+                                                 int32_t r1, int32_t r2, int32_t r3, uint32_t bar_cluster) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes.cta_group::2"
+        " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(bar_cluster)
+        : "memory");
+}
 __device__ __forceinline__ uint64_t l2_policy_evict_first() {
     uint64_t p;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
@@ -109,14 +120,22 @@ struct PairTile {
     int64_t hi;  // rows >= hi belong to another expert or lie past T
     int n0;
     int e;
+    bool router;  // the router unit of the pair tile (the router inside fc1)
 };
+
+// Units per 256-row pair tile: the column tiles, plus the router unit when the router runs inside fc1.
+__device__ __forceinline__ int units_per_pair(const TcGemmArgs& a, int n_tiles) {
+    return n_tiles + (a.mode == TC_DENSE && a.fr_E > 0 ? 1 : 0);
+}
 
 template <int BN>
 __device__ __forceinline__ PairTile decode_pair(const TcGemmArgs& a, int unit, int n_tiles, const int* s_prefix) {
     constexpr int BM = T2<BN>::BM;
     PairTile t;
-    const int mp = unit / n_tiles;
-    t.n0 = (unit % n_tiles) * BN;
+    const int nup = units_per_pair(a, n_tiles);
+    const int mp = unit / nup;
+    t.n0 = (unit % nup) * BN;
+    t.router = (unit % nup) == n_tiles;
     if (a.mode == TC_GROUPED) {
         int e = 0;
         while (e + 1 < a.E && s_prefix[e + 1] <= mp) ++e;
@@ -162,6 +181,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
     auto tfull_bar = [&](int i) { return bar0 + 8u * (2 * STAGES + i); };
     auto tempty_bar = [&](int i) { return bar0 + 8u * (2 * STAGES + 2 + i); };
     const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+    // the router inside fc1: the four lane-quarter warps' expert counts of a router unit are
+    // exchanged through shared memory, double-buffered, each buffer guarded by its own barrier
+    auto fr_bar = [&](int i) { return bar0 + 8u * (2 * STAGES + 5 + i); };
+    int* s_frc = s_tab;                                            // [2][4][CM_MAX_E] counts
+    float* s_frb = reinterpret_cast<float*>(s_tab + 8 * CM_MAX_E);  // [CM_MAX_E] b_g
     const uint64_t lim = (uint64_t)a.wait_limit_ns;
 
     const int n_tiles = a.N / BN;
@@ -180,6 +204,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
             mbar_init(tempty_bar(i), 2 * NUM_EPI);  // epilogue warps of both CTAs
         }
         mbar_init(drain_bar, 1);
+        mbar_init(fr_bar(0), 4);  // the quarter warps of the first column group
+        mbar_init(fr_bar(1), 4);
         *abort_flag = 0;
         mbar_fence_init();
     }
@@ -193,6 +219,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         const uint16_t* b = static_cast<const uint16_t*>(a.out_bias);
         for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = __uint_as_float((uint32_t)b[n] << 16);
     }
+    if (MODE == TC_DENSE && a.fr_E > 0 && threadIdx.x < a.fr_E)  // the router's bias (a weight)
+        s_frb[threadIdx.x] = __uint_as_float((uint32_t) static_cast<const uint16_t*>(a.fr_bias)[threadIdx.x] << 16);
     // Tensor memory for the pair: allocated collectively by one warp of each CTA. The two CTAs
     // must see the same base (the even CTA's MMAs name it for both); a mismatch aborts cleanly.
     if (warp == WARP_MMA) {
@@ -302,68 +330,94 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         m_pairs = s_prefix[a.E];
     else
         m_pairs = (int)((a.M + 2 * BM - 1) / (2 * BM));
-    const int num_units = tmem_ok ? m_pairs * n_tiles : 0;
+    const int num_units = tmem_ok ? m_pairs * units_per_pair(a, n_tiles) : 0;
     const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
 
     if (warp == WARP_TMA) {
         // ------------------------------------------------ producers (both CTAs)
-        if (lane == 0) {
-            const uint32_t full_leader0 = map_to_rank(full_bar(0), 0);
-            const uint64_t pol_a = l2_policy_evict_first();
-            bool waited = a.pdl_wait_role != 2;  // role 2: wait before the first t-segment load
-            int stage = 0;
-            uint32_t ph = 0;
-            bool ok = true;
-            for (int u = cid; u < num_units && ok; u += ncl) {
-                const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
-                const int am = (int)(t.m0 + (int64_t)rank * BM);
-                const int bn = t.n0 + (int)rank * BH;
-                const int nkb_t = (MODE == TC_GROUPED && a.dense_last && t.e == a.E - 1) ? nk1 : nkb;
-                for (int kb = 0; kb < nkb_t; ++kb) {
-                    if (!mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim)) {
-                        ok = false;
-                        break;
+        // Lane 0 waits for free stages and issues the tile loads; with the z rows gathered by slot
+        // (a1_rows) every lane issues one four-row gather per stage (32 x 4 = the CTA's 128 rows),
+        // otherwise lane 0 runs alone.
+        const uint32_t full_leader0 = map_to_rank(full_bar(0), 0);
+        const uint64_t pol_a = l2_policy_evict_first();
+        const bool gather = MODE == TC_GROUPED && a.a1_rows != nullptr;
+        bool waited = a.pdl_wait_role != 2;  // role 2: wait before the first t-segment load
+        int stage = 0;
+        uint32_t ph = 0;
+        bool ok = gather || lane == 0;
+        for (int u = cid; u < num_units && ok; u += ncl) {
+            const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
+            const int am = (int)(t.m0 + (int64_t)rank * BM);
+            // the router unit: CTA r supplies W_g rows [16 r, +16) of the 256 x 32 MMA
+            const int bn = (MODE == TC_DENSE && t.router) ? (int)rank * 16 : t.n0 + (int)rank * BH;
+            const uint32_t stage_tx = (MODE == TC_DENSE && t.router) ? 2u * (A_BYTES + C::FR_B_BYTES)
+                                                                     : 2u * STAGE_BYTES;
+            const int nkb_t = (MODE == TC_GROUPED && a.dense_last && t.e == a.E - 1) ? nk1 : nkb;
+            int32_t gr[4] = {0, 0, 0, 0};
+            if (gather) {  // this lane's four slots; slots past M take the last one (their rows are dropped)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    int64_t sl = (int64_t)am + 4 * lane + j;
+                    if (sl > a.M - 1) sl = a.M - 1;
+                    const int32_t tok = a.a1_rows[sl];
+                    gr[j] = (uint32_t)tok < (uint64_t)a.M ? tok : 0;  // only a routing that gave up
+                }
+            }
+            for (int kb = 0; kb < nkb_t; ++kb) {
+                int w_ok = 1;
+                if (lane == 0) w_ok = mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim);
+                if (gather) w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+                if (!w_ok) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t sA = smem_u32(sm + stage * STAGE_BYTES);
+                const uint32_t sB = sA + A_BYTES;
+                const uint32_t fb = full_leader0 + 8u * stage;  // the even CTA's full barrier
+                if (leader && lane == 0) mbar_arrive_expect_tx(full_bar(stage), stage_tx);
+                const CUtensorMap* mA;
+                const CUtensorMap* mB;
+                int kk;
+                bool gathered = false;
+                if (MODE != TC_GROUPED) {  // x x W (or x x W_g), then the augmentation block
+                    mA = kb < nk0 ? &a.tmA0 : &a.tmA1;
+                    mB = t.router ? &a.tmR : kb < nk0 ? &a.tmB0 : &a.tmB1[0];
+                    kk = kb < nk0 ? kb * BK : 0;
+                } else if (kb < nk1) {  // z x W_e^res
+                    mA = &a.tmA1;
+                    mB = &a.tmB1[t.e];
+                    kk = kb * BK;
+                    gathered = gather;
+                } else {  // t x U_r
+                    if (!waited) {
+                        pdl_wait();
+                        waited = true;
                     }
-                    const uint32_t sA = smem_u32(sm + stage * STAGE_BYTES);
-                    const uint32_t sB = sA + A_BYTES;
-                    const uint32_t fb = full_leader0 + 8u * stage;  // the even CTA's full barrier
-                    if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * STAGE_BYTES);
-                    const CUtensorMap* mA;
-                    const CUtensorMap* mB;
-                    int kk;
-                    if (MODE != TC_GROUPED) {  // x x W, then the augmentation block
-                        mA = kb < nk0 ? &a.tmA0 : &a.tmA1;
-                        mB = kb < nk0 ? &a.tmB0 : &a.tmB1[0];
-                        kk = kb < nk0 ? kb * BK : 0;
-                    } else if (kb < nk1) {  // z x W_e^res
-                        mA = &a.tmA1;
-                        mB = &a.tmB1[t.e];
-                        kk = kb * BK;
-                    } else {  // t x U_r
-                        if (!waited) {
-                            pdl_wait();
-                            waited = true;
-                        }
-                        mA = &a.tmA0;
-                        mB = &a.tmB0;
-                        kk = (kb - nk1) * BK;
-                    }
+                    mA = &a.tmA0;
+                    mB = &a.tmB0;
+                    kk = (kb - nk1) * BK;
+                }
+                if (gathered) {
+                    tma_gather4_pair(sA + 512u * lane, mA, kk, gr[0], gr[1], gr[2], gr[3], fb);
+                } else if (lane == 0) {
                     if (a.a_evict_first)
                         tma_load_2d_pair_hint(sA, mA, kk, am, fb, pol_a);
                     else
                         tma_load_2d_pair(sA, mA, kk, am, fb);
-                    tma_load_2d_pair(sB, mB, kk, bn, fb);
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        ph ^= 1;
-                    }
+                }
+                if (lane == 0) tma_load_2d_pair(sB, mB, kk, bn, fb);
+                if (++stage == STAGES) {
+                    stage = 0;
+                    ph ^= 1;
                 }
             }
         }
     } else if (warp == WARP_MMA) {
         // ------------------------------------------------ MMA issuer (even CTA)
         if (leader && lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(2 * BM, BN);
+            const uint32_t idesc_t = idesc_bf16_f32(2 * BM, BN);
+            const uint32_t idesc_r = idesc_bf16_f32(2 * BM, 32);  // the router unit: 256 x 32
+            const int nup = units_per_pair(a, n_tiles);
             // Stage s's descriptors are the stage-0 ones plus the byte offset / 16 in the start
             // address field (every shared address here is below 256 KB, so the field never carries).
             const uint64_t dA0 = sdesc_kmajor_sw128(smem_u32(sm));
@@ -376,6 +430,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                 if (!mbar_wait(tempty_bar(acc), aph ^ 1, abort_flag, a.status, lim)) break;
                 tc_fence_after();
                 const uint32_t dtm = tmem_base + acc * BN;
+                const uint32_t idesc = (MODE == TC_DENSE && u % nup == n_tiles) ? idesc_r : idesc_t;
                 int nkb_t = nkb;  // the dense path's group: the z x W2 segment alone
                 if (MODE == TC_GROUPED && a.dense_last && decode_pair<BN>(a, u, n_tiles, s_prefix).e == a.E - 1)
                     nkb_t = nk1;
@@ -431,6 +486,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         const uint32_t tempty_leader0 = map_to_rank(tempty_bar(0), 0);
         int acc = 0;
         uint32_t aph = 0;
+        int fr_it = 0;  // router units handled so far (the router inside fc1)
         for (int u = cid; u < num_units; u += ncl) {
             const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
             const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
@@ -440,145 +496,200 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
             const float2 ln = (a.ln_stats && mrow < t.hi) ? a.ln_stats[mrow] : make_float2(0.f, 1.f);
             if (!mbar_wait(tfull_bar(acc), aph, abort_flag, a.status, lim)) break;
             tc_fence_after();
-            int64_t orow = -1;
-            if (mrow < t.hi) {
-                if (MODE == TC_DENSE && a.rt_info) {  // the token's routing slot
-                    const uint32_t w = rtw;
-                    const int e = (int)(w & 0xffu);
-                    const int rc = (int)((uint32_t)mrow / (uint32_t)a.rt_chunk);  // T < 2^31
-                    if (a.rt_cls_stride > 0 && (uint32_t)mrow % (uint32_t)a.rt_cls_stride == 0)  // class token
-                        orow = a.M - n_class_tokens(a.M, a.rt_cls_stride) + (uint32_t)mrow / (uint32_t)a.rt_cls_stride;
-                    else if (e < a.rt_E)
-                        orow = (int64_t)s_off[e] + s_tab[rc * a.rt_E + e] + (int)(w >> 8);
-                    if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
-                    if (orow >= 0 && t.n0 == 0 && c_lo == 0) a.rt_perm[orow] = (int32_t)mrow;  // once per token
-                } else {
-                    orow = a.rows ? (int64_t)a.rows[mrow] : mrow;
-                    if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
-                }
-            }
-            const float rsc = (a.group_scale && mrow < t.hi) ? tc_row_scale(a, mrow) : 1.f;
-            // with the mean term in the accumulator (augmentation block) the bias add also scales by
-            // rstd: fma(acc, 1, b) = acc + b exactly, so without the LayerNorm nothing changes
-            const float lns = (a.ln_stats && !a.ln_colsum) ? ln.y : 1.f;
-            const float2 lns2 = make_float2(lns, lns);
-            // this lane stores warp rows 16 h + 8 p + lane / 4 (h, p < 2), 16-byte piece lane % 4 of
-            // each 32-column chunk: their destinations, once per tile
-            uint16_t* dst_row[4];
+            if (MODE == TC_DENSE && t.router) {
+                // The router unit: accumulator columns [0, E) of this lane's row hold W_g x. The four
+                // warps of the first column group (one per lane quarter) add b_g, take the argmax
+                // (lowest index on ties), count each expert's rows of the quarter by ballots, and
+                // exchange the counts through shared memory (a barrier per buffer, bounded waits):
+                // rank = earlier quarters' rows of the expert + earlier lanes' of this quarter.
+                if (c_lo == 0) {
+                    const int E = a.fr_E;
+                    const int rb = fr_it & 1;
+                    int* rc = s_frc + rb * 4 * CM_MAX_E;
+                    uint32_t v[16];
+                    CM_TMEM_LD_X16(tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN, v);
+                    tmem_wait_ld();
+                    int esel = -1;
+                    if (mrow < t.hi) {
+                        float bv = -INFINITY;
+                        int be = 0x7fffffff;
 #pragma unroll
-            for (int hp = 0; hp < 4; ++hp) {
-                const int64_t o = __shfl_sync(0xffffffffu, orow, 8 * hp + lane / 4);
-                dst_row[hp] = o >= 0 ? static_cast<uint16_t*>(a.C) + o * a.ldc + t.n0 + (lane % 4) * 8 : nullptr;
-            }
-            for (int c = c_lo; c < c_lo + WCOLS; c += CW) {
-                uint32_t v[CW];
-                const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
-                CM_TMEM_LD_X16(taddr, v);
-                CM_TMEM_LD_X16(taddr + 16, (v + 16));
-                tmem_wait_ld();
-                float f[CW];
-#pragma unroll
-                for (int j = 0; j < CW; ++j) f[j] = __uint_as_float(v[j]);
-                const int nb = t.n0 + c;
-                if (a.ln_stats && a.ln_colsum) {  // W LN(y) = rstd (W y - mean c), c_n = sum_k W[n, k]
-                    const float4* cp = reinterpret_cast<const float4*>(a.ln_colsum + nb);  // same for all lanes
-#pragma unroll
-                    for (int j4 = 0; j4 < CW / 4; ++j4) {
-                        const float4 c4 = __ldg(cp + j4);
-                        f[4 * j4] = ln.y * fmaf(-ln.x, c4.x, f[4 * j4]);
-                        f[4 * j4 + 1] = ln.y * fmaf(-ln.x, c4.y, f[4 * j4 + 1]);
-                        f[4 * j4 + 2] = ln.y * fmaf(-ln.x, c4.z, f[4 * j4 + 2]);
-                        f[4 * j4 + 3] = ln.y * fmaf(-ln.x, c4.w, f[4 * j4 + 3]);
+                        for (int e = 0; e < 16; ++e) {
+                            if (e < E) {
+                                const float l = __uint_as_float(v[e]) + s_frb[e];
+                                if (l > bv || (l == bv && e < be)) {
+                                    bv = l;
+                                    be = e;
+                                }
+                            }
+                        }
+                        esel = be < E ? be : 0;  // only reachable with non-finite logits
                     }
-                }
-                if (a.epi == TC_EPI_BIAS_GELU) {
-                    const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
-#pragma unroll
-                    for (int j4 = 0; j4 < CW / 4; ++j4) {
-                        const float4 b = bp[j4];
-                        const float2 g0 = gelu_pair_as(
-                            __ffma2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), lns2, make_float2(b.x, b.y)));
-                        const float2 g1 = gelu_pair_as(
-                            __ffma2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), lns2, make_float2(b.z, b.w)));
-                        f[4 * j4] = g0.x;
-                        f[4 * j4 + 1] = g0.y;
-                        f[4 * j4 + 2] = g1.x;
-                        f[4 * j4 + 3] = g1.y;
+                    int rk = 0;
+                    for (int e = 0; e < E; ++e) {
+                        const unsigned mk = __ballot_sync(0xffffffffu, esel == e);
+                        if (lane == 0) rc[q * CM_MAX_E + e] = __popc(mk);
+                        if (esel == e) rk = __popc(mk & ((1u << lane) - 1u));
                     }
-                } else if (a.epi == TC_EPI_BIAS_RELU) {
-                    const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
-#pragma unroll
-                    for (int j4 = 0; j4 < CW / 4; ++j4) {
-                        const float4 b = bp[j4];
-                        f[4 * j4] = fmaxf(fmaf(f[4 * j4], lns, b.x), 0.f);
-                        f[4 * j4 + 1] = fmaxf(fmaf(f[4 * j4 + 1], lns, b.y), 0.f);
-                        f[4 * j4 + 2] = fmaxf(fmaf(f[4 * j4 + 2], lns, b.z), 0.f);
-                        f[4 * j4 + 3] = fmaxf(fmaf(f[4 * j4 + 3], lns, b.w), 0.f);
-                    }
-                } else if (a.out_bias) {
-                    const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
-#pragma unroll
-                    for (int j4 = 0; j4 < CW / 4; ++j4) {
-                        const float4 b = bp[j4];
-                        const float2 p0 = __fadd2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), make_float2(b.x, b.y));
-                        const float2 p1 = __fadd2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), make_float2(b.z, b.w));
-                        f[4 * j4] = p0.x;
-                        f[4 * j4 + 1] = p0.y;
-                        f[4 * j4 + 2] = p1.x;
-                        f[4 * j4 + 3] = p1.y;
-                    }
-                } else if (a.epi == TC_EPI_SCALE) {
-                    const float4* sp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
-#pragma unroll
-                    for (int j4 = 0; j4 < CW / 4; ++j4) {
-                        const float4 sc = sp[j4];
-                        const float2 p0 = __fmul2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), make_float2(sc.x, sc.y));
-                        const float2 p1 = __fmul2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), make_float2(sc.z, sc.w));
-                        f[4 * j4] = p0.x;
-                        f[4 * j4 + 1] = p0.y;
-                        f[4 * j4 + 2] = p1.x;
-                        f[4 * j4 + 3] = p1.y;
-                    }
-                }
-                if (a.group_scale) {
-#pragma unroll
-                    for (int j2 = 0; j2 < CW / 2; ++j2) {
-                        const float2 p2 = __fmul2_rn(make_float2(f[2 * j2], f[2 * j2 + 1]), make_float2(rsc, rsc));
-                        f[2 * j2] = p2.x;
-                        f[2 * j2 + 1] = p2.y;
-                    }
-                }
-                if (a.c_f32) {  // fp32 output: each lane stores its row's 32 values as computed
-                    if (orow >= 0) {
-                        float4* dstf = reinterpret_cast<float4*>(static_cast<float*>(a.C) + orow * a.ldc + nb);
-#pragma unroll
-                        for (int j4 = 0; j4 < CW / 4; ++j4)
-                            dstf[j4] = make_float4(f[4 * j4], f[4 * j4 + 1], f[4 * j4 + 2], f[4 * j4 + 3]);
-                    }
-                    continue;
-                }
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    if ((lane >> 4) == h) {
-                        const int rw = lane & 15;
-                        unsigned char* dst = wstg + rw * 64;
-#pragma unroll
-                        for (int j8 = 0; j8 < 4; ++j8) {
-                            const float* g = f + 8 * j8;
-                            *reinterpret_cast<uint4*>(dst + ((j8 ^ ((rw >> 1) & 3)) << 4)) =
-                                make_uint4(pack_bf16(g[0], g[1]), pack_bf16(g[2], g[3]), pack_bf16(g[4], g[5]),
-                                           pack_bf16(g[6], g[7]));
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(fr_bar(rb));
+                    if (mbar_wait(fr_bar(rb), (uint32_t)(fr_it >> 1) & 1u, abort_flag, a.status, lim)) {
+                        if (esel >= 0) {
+                            int base = 0;
+                            for (int qq = 0; qq < q; ++qq) base += rc[qq * CM_MAX_E + esel];
+                            a.fr_idx[mrow] = esel;
+                            a.fr_info[mrow] = esel | ((base + rk) << 8);
+                        }
+                        const int64_t rng = t.m0 / FR_RANGE + rank;  // this CTA's 128-row range
+                        if (q == 0 && lane < E && rng * FR_RANGE < a.M) {
+                            int c = 0;
+                            for (int qq = 0; qq < 4; ++qq) c += rc[qq * CM_MAX_E + lane];
+                            a.fr_counts[rng * CM_MAX_E + lane] = c;
                         }
                     }
-                    __syncwarp();
-#pragma unroll
-                    for (int p = 0; p < 2; ++p) {
-                        const int rr = 8 * p + lane / 4;  // row of the half
-                        const int ch = (lane % 4) ^ ((rr >> 1) & 3);
-                        const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * 64 + ch * 16);
-                        if (dst_row[2 * h + p]) *reinterpret_cast<uint4*>(dst_row[2 * h + p] + c) = val;
+                }
+                ++fr_it;
+            } else {
+                int64_t orow = -1;
+                if (mrow < t.hi) {
+                    if (MODE == TC_DENSE && a.rt_info) {  // the token's routing slot
+                        const uint32_t w = rtw;
+                        const int e = (int)(w & 0xffu);
+                        const int rc = (int)((uint32_t)mrow / (uint32_t)a.rt_chunk);  // T < 2^31
+                        if (a.rt_cls_stride > 0 && (uint32_t)mrow % (uint32_t)a.rt_cls_stride == 0)  // class token
+                            orow = a.M - n_class_tokens(a.M, a.rt_cls_stride) + (uint32_t)mrow / (uint32_t)a.rt_cls_stride;
+                        else if (e < a.rt_E)
+                            orow = (int64_t)s_off[e] + s_tab[rc * a.rt_E + e] + (int)(w >> 8);
+                        if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
+                        if (orow >= 0 && t.n0 == 0 && c_lo == 0) a.rt_perm[orow] = (int32_t)mrow;  // once per token
+                    } else {
+                        orow = a.rows ? (int64_t)a.rows[mrow] : mrow;
+                        if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
                     }
-                    __syncwarp();
+                }
+                const float rsc = (a.group_scale && mrow < t.hi) ? tc_row_scale(a, mrow) : 1.f;
+                // with the mean term in the accumulator (augmentation block) the bias add also scales by
+                // rstd: fma(acc, 1, b) = acc + b exactly, so without the LayerNorm nothing changes
+                const float lns = (a.ln_stats && !a.ln_colsum) ? ln.y : 1.f;
+                const float2 lns2 = make_float2(lns, lns);
+                // this lane stores warp rows 16 h + 8 p + lane / 4 (h, p < 2), 16-byte piece lane % 4 of
+                // each 32-column chunk: their destinations, once per tile
+                uint16_t* dst_row[4];
+    #pragma unroll
+                for (int hp = 0; hp < 4; ++hp) {
+                    const int64_t o = __shfl_sync(0xffffffffu, orow, 8 * hp + lane / 4);
+                    dst_row[hp] = o >= 0 ? static_cast<uint16_t*>(a.C) + o * a.ldc + t.n0 + (lane % 4) * 8 : nullptr;
+                }
+                for (int c = c_lo; c < c_lo + WCOLS; c += CW) {
+                    uint32_t v[CW];
+                    const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
+                    CM_TMEM_LD_X16(taddr, v);
+                    CM_TMEM_LD_X16(taddr + 16, (v + 16));
+                    tmem_wait_ld();
+                    float f[CW];
+    #pragma unroll
+                    for (int j = 0; j < CW; ++j) f[j] = __uint_as_float(v[j]);
+                    const int nb = t.n0 + c;
+                    if (a.ln_stats && a.ln_colsum) {  // W LN(y) = rstd (W y - mean c), c_n = sum_k W[n, k]
+                        const float4* cp = reinterpret_cast<const float4*>(a.ln_colsum + nb);  // same for all lanes
+    #pragma unroll
+                        for (int j4 = 0; j4 < CW / 4; ++j4) {
+                            const float4 c4 = __ldg(cp + j4);
+                            f[4 * j4] = ln.y * fmaf(-ln.x, c4.x, f[4 * j4]);
+                            f[4 * j4 + 1] = ln.y * fmaf(-ln.x, c4.y, f[4 * j4 + 1]);
+                            f[4 * j4 + 2] = ln.y * fmaf(-ln.x, c4.z, f[4 * j4 + 2]);
+                            f[4 * j4 + 3] = ln.y * fmaf(-ln.x, c4.w, f[4 * j4 + 3]);
+                        }
+                    }
+                    if (a.epi == TC_EPI_BIAS_GELU) {
+                        const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
+    #pragma unroll
+                        for (int j4 = 0; j4 < CW / 4; ++j4) {
+                            const float4 b = bp[j4];
+                            const float2 g0 = gelu_pair_as(
+                                __ffma2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), lns2, make_float2(b.x, b.y)));
+                            const float2 g1 = gelu_pair_as(
+                                __ffma2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), lns2, make_float2(b.z, b.w)));
+                            f[4 * j4] = g0.x;
+                            f[4 * j4 + 1] = g0.y;
+                            f[4 * j4 + 2] = g1.x;
+                            f[4 * j4 + 3] = g1.y;
+                        }
+                    } else if (a.epi == TC_EPI_BIAS_RELU) {
+                        const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
+    #pragma unroll
+                        for (int j4 = 0; j4 < CW / 4; ++j4) {
+                            const float4 b = bp[j4];
+                            f[4 * j4] = fmaxf(fmaf(f[4 * j4], lns, b.x), 0.f);
+                            f[4 * j4 + 1] = fmaxf(fmaf(f[4 * j4 + 1], lns, b.y), 0.f);
+                            f[4 * j4 + 2] = fmaxf(fmaf(f[4 * j4 + 2], lns, b.z), 0.f);
+                            f[4 * j4 + 3] = fmaxf(fmaf(f[4 * j4 + 3], lns, b.w), 0.f);
+                        }
+                    } else if (a.out_bias) {
+                        const float4* bp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
+    #pragma unroll
+                        for (int j4 = 0; j4 < CW / 4; ++j4) {
+                            const float4 b = bp[j4];
+                            const float2 p0 = __fadd2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), make_float2(b.x, b.y));
+                            const float2 p1 = __fadd2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), make_float2(b.z, b.w));
+                            f[4 * j4] = p0.x;
+                            f[4 * j4 + 1] = p0.y;
+                            f[4 * j4 + 2] = p1.x;
+                            f[4 * j4 + 3] = p1.y;
+                        }
+                    } else if (a.epi == TC_EPI_SCALE) {
+                        const float4* sp = reinterpret_cast<const float4*>(s_bias + nb);  // same for all lanes
+    #pragma unroll
+                        for (int j4 = 0; j4 < CW / 4; ++j4) {
+                            const float4 sc = sp[j4];
+                            const float2 p0 = __fmul2_rn(make_float2(f[4 * j4], f[4 * j4 + 1]), make_float2(sc.x, sc.y));
+                            const float2 p1 = __fmul2_rn(make_float2(f[4 * j4 + 2], f[4 * j4 + 3]), make_float2(sc.z, sc.w));
+                            f[4 * j4] = p0.x;
+                            f[4 * j4 + 1] = p0.y;
+                            f[4 * j4 + 2] = p1.x;
+                            f[4 * j4 + 3] = p1.y;
+                        }
+                    }
+                    if (a.group_scale) {
+    #pragma unroll
+                        for (int j2 = 0; j2 < CW / 2; ++j2) {
+                            const float2 p2 = __fmul2_rn(make_float2(f[2 * j2], f[2 * j2 + 1]), make_float2(rsc, rsc));
+                            f[2 * j2] = p2.x;
+                            f[2 * j2 + 1] = p2.y;
+                        }
+                    }
+                    if (a.c_f32) {  // fp32 output: each lane stores its row's 32 values as computed
+                        if (orow >= 0) {
+                            float4* dstf = reinterpret_cast<float4*>(static_cast<float*>(a.C) + orow * a.ldc + nb);
+    #pragma unroll
+                            for (int j4 = 0; j4 < CW / 4; ++j4)
+                                dstf[j4] = make_float4(f[4 * j4], f[4 * j4 + 1], f[4 * j4 + 2], f[4 * j4 + 3]);
+                        }
+                        continue;
+                    }
+    #pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        if ((lane >> 4) == h) {
+                            const int rw = lane & 15;
+                            unsigned char* dst = wstg + rw * 64;
+    #pragma unroll
+                            for (int j8 = 0; j8 < 4; ++j8) {
+                                const float* g = f + 8 * j8;
+                                *reinterpret_cast<uint4*>(dst + ((j8 ^ ((rw >> 1) & 3)) << 4)) =
+                                    make_uint4(pack_bf16(g[0], g[1]), pack_bf16(g[2], g[3]), pack_bf16(g[4], g[5]),
+                                               pack_bf16(g[6], g[7]));
+                            }
+                        }
+                        __syncwarp();
+    #pragma unroll
+                        for (int p = 0; p < 2; ++p) {
+                            const int rr = 8 * p + lane / 4;  // row of the half
+                            const int ch = (lane % 4) ^ ((rr >> 1) & 3);
+                            const uint4 val = *reinterpret_cast<const uint4*>(wstg + rr * 64 + ch * 16);
+                            if (dst_row[2 * h + p]) *reinterpret_cast<uint4*>(dst_row[2 * h + p] + c) = val;
+                        }
+                        __syncwarp();
+                    }
                 }
             }
             tc_fence_before();
@@ -618,7 +729,7 @@ static cudaError_t launch2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     const int n_tiles = a.N / BN;
     int64_t m_pairs = (a.M + 2 * C::BM - 1) / (2 * C::BM);
     if (a.mode == TC_GROUPED) m_pairs += a.E;
-    const int64_t units = m_pairs * n_tiles;
+    const int64_t units = m_pairs * (n_tiles + (a.mode == TC_DENSE && a.fr_E > 0 ? 1 : 0));
     int64_t clusters = units < num_sms / 2 ? units : num_sms / 2;
     if (clusters <= 0) return cudaSuccess;
     cudaLaunchConfig_t cfg = {};
@@ -646,6 +757,12 @@ cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     const bool bias_epi = a.epi == TC_EPI_BIAS_GELU || a.epi == TC_EPI_BIAS_RELU;
     if (a.ln_aug && (a.mode != TC_DENSE || !bias_epi || !a.ln_stats || a.ln_colsum)) return cudaErrorInvalidValue;
     if (a.ln_stats && !a.ln_colsum && !a.ln_aug) return cudaErrorInvalidValue;
+    // the router inside fc1: dense mode, fc1's own epilogue, token order, none of the other row maps
+    if (a.fr_E > 0 && (a.mode != TC_DENSE || a.fr_E > CM_MAX_E || a.epi != TC_EPI_BIAS_GELU || a.ln_aug ||
+                       a.ln_stats || a.rt_info || a.rows || a.c_f32 || a.group_scale || !a.fr_bias || !a.fr_idx ||
+                       !a.fr_info || !a.fr_counts))
+        return cudaErrorInvalidValue;
+    if (a.a1_rows && a.mode != TC_GROUPED) return cudaErrorInvalidValue;
     if (bn == 256) return launch2<256>(a, num_sms, s);
     if (bn == 192) return launch2<192>(a, num_sms, s);
     return launch2<128>(a, num_sms, s);
