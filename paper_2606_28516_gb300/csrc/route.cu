@@ -28,7 +28,7 @@
 namespace cm {
 
 constexpr int RT_THREADS = 256;                 // fp32 router: 8 warps
-constexpr int RT_BF16_THREADS = 320;            // bf16 router: up to 9 consumer warps + 1 producer warp
+constexpr int RT_BF16_THREADS = 288;            // bf16 router: 8 consumer warps + 1 producer warp
 constexpr int RT_MAX_WARPS = RT_BF16_THREADS / 32;
 constexpr int RT_STAGE_ROWS = 16;               // rows per ring stage (one MMA row group)
 
@@ -68,54 +68,33 @@ __host__ __device__ inline size_t frag_bytes(int dtype, int d, int E) {
     return (size_t)E * d * 4;
 }
 
-// W_g's B fragments held in registers (bf16, E <= 8, d <= RT_WREG_D): 4 registers per 32 columns
-constexpr int RT_WREG_D = 768;
-__host__ __device__ inline bool route_wreg(int dtype, int d, int E) {
-    return dtype == CLEARMOE_BF16 && E <= 8 && d <= RT_WREG_D;
-}
-
-// Dynamic shared memory: [router weights] [bf16: ring of S stages] [bf16: 2 S + 2 mbarriers]
+// Dynamic shared memory: [router weights] [bf16: ring of S stages] [bf16: 2 S + 1 mbarriers]
 // [per-row word: expert | local rank << 8, when chunk words fit; else that word lives in idx in
 // global memory (the CTA's own rows, visible block-wide after __syncthreads) until phase 2
 // rewrites idx with the expert alone], so the footprint does not grow with T.
-// The ring has one slot per consumer warp (S = 9, 8, or 4 when eight stages do not fit): consumer
+// The ring has one slot per consumer warp (S = 8, or 4 when eight stages do not fit): consumer
 // warp w alone reads slot w, for stages w, w + S, ..., so each of its mbarrier waits is for the
 // phase right after the one it last consumed (a parity wait cannot tell phases two apart).
-// Nine slots when W_g's fragments live in registers and everything fits: the ninth slot lies on
-// top of W_g's rows, which the consumers have copied into registers (they signal that on the last
-// barrier) before the producer first fills it. The stream is bound by the bytes in flight per SM,
-// so the ninth slot buys about an eighth more bandwidth.
 constexpr size_t RT_SMEM_MAX = 220 * 1024;
 struct RouteLayout {
-    size_t frag, ring, bars, sidx, scnt, total;
+    size_t ring, bars, sidx, scnt, total;
     int S, stage_bytes;
-    bool sidx_in_smem, wslot;
+    bool sidx_in_smem;
 };
 __host__ __device__ inline RouteLayout route_layout(int dtype, int d, int E, int chunk) {
     RouteLayout L;
     const size_t frag = (frag_bytes(dtype, d, E) + 127) & ~(size_t)127;
     L.stage_bytes = RT_STAGE_ROWS * d * 2;
+    L.S = 0;
+    L.ring = frag;
+    if (dtype == CLEARMOE_BF16)  // eight slots when they fit beside W_g and the barriers, else four
+        L.S = (L.ring + 8 * (size_t)L.stage_bytes + 17 * 8 <= RT_SMEM_MAX) ? 8 : 4;
+    L.bars = (L.ring + (size_t)L.S * L.stage_bytes + 15) & ~(size_t)15;
+    L.sidx = L.bars + (size_t)(2 * L.S + 1) * 8;  // bf16: ring barriers + the W_g barrier
     // expert ids of the CTA's rows: in shared memory when they fit, else read back from idx
     // per row a 4-byte word; bf16 also keeps each 16-row stage's per-expert counts (2 bytes each)
     const size_t rows_bytes =
         (size_t)chunk * 4 + (dtype == CLEARMOE_BF16 ? (size_t)((chunk + 15) / 16) * CM_MAX_E * 2 : 0);
-    const size_t nbars9 = (size_t)(2 * 9 + 2) * 8;
-    if (route_wreg(dtype, d, E) && frag <= (size_t)L.stage_bytes &&
-        9 * (size_t)L.stage_bytes + nbars9 + rows_bytes <= RT_SMEM_MAX) {
-        L.S = 9;
-        L.wslot = true;
-        L.ring = 0;
-        L.frag = 8 * (size_t)L.stage_bytes;  // slot 8
-    } else {
-        L.wslot = false;
-        L.frag = 0;
-        L.ring = frag;
-        L.S = 0;
-        if (dtype == CLEARMOE_BF16)  // eight slots when they fit beside W_g and the barriers, else four
-            L.S = (L.ring + 8 * (size_t)L.stage_bytes + 18 * 8 <= RT_SMEM_MAX) ? 8 : 4;
-    }
-    L.bars = (L.ring + (size_t)L.S * L.stage_bytes + 15) & ~(size_t)15;
-    L.sidx = L.bars + (size_t)(2 * L.S + 2) * 8;  // bf16: ring barriers, W_g landed, W_g copied out
     L.scnt = L.sidx + (size_t)chunk * 4;
     L.sidx_in_smem = L.sidx + rows_bytes <= RT_SMEM_MAX;
     L.total = L.sidx + (L.sidx_in_smem ? rows_bytes : 0);
@@ -129,11 +108,15 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
                  : "memory");
 }
 
+// W_g's B fragments held in registers (bf16, E <= 8, d <= RT_WREG_D): 4 registers per 32 columns
+constexpr int RT_WREG_D = 768;
+inline bool route_wreg(int dtype, int d, int E) { return dtype == CLEARMOE_BF16 && E <= 8 && d <= RT_WREG_D; }
+
 template <bool BF16, bool WREG>
 __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_kernel(const RouteArgs a, const int chunk) {
     constexpr int NTHREADS = BF16 ? RT_BF16_THREADS : RT_THREADS;
     constexpr int NWARPS = NTHREADS / 32;
-    constexpr int NCONS_MAX = 9;  // warps computing logits (bf16: the first S warps); the next one produces
+    constexpr int NCONS_MAX = 8;  // warps computing logits (bf16: the first S warps)
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ int s_count[CM_MAX_E];
     __shared__ int s_run[CM_MAX_E];
@@ -176,7 +159,6 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         // their own barrier) and then streams the stages.
         const bool producer = tid == NCONS_MAX * 32;
         const uint32_t wbar = bar0 + 8u * (2 * S);
-        const uint32_t wdone = bar0 + 8u * (2 * S + 1);  // every consumer holds W_g in registers
         const int WRB = wrow_bytes(d);
         if (producer) {
             for (int s = 0; s < S; ++s) {
@@ -184,15 +166,13 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 mbar_init(empty_bar(s), 1);
             }
             mbar_init(wbar, 1);
-            mbar_init(wdone, S);
             mbar_fence_init();
         }
         __syncthreads();  // barriers initialised
         if (producer) {
             mbar_arrive_expect_tx(wbar, (uint32_t)E * d * 2);
             const unsigned char* Wb = static_cast<const unsigned char*>(a.Wg);
-            for (int e = 0; e < E; ++e)
-                bulk_g2s(smem_u32(smem + lay.frag) + e * WRB, Wb + (size_t)e * d * 2, d * 2, wbar);
+            for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(smem) + e * WRB, Wb + (size_t)e * d * 2, d * 2, wbar);
         }
         pdl_wait();  // from here on the previous kernel's results (x) are read and outputs written
         // the next kernel may start now (its CTAs set up, and may read x, while this one streams):
@@ -205,9 +185,6 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
                 for (; k < nstages; ++k) {
                     const int s = k % S;
                     if (!mbar_wait(empty_bar(s), ((k / S) & 1) ^ 1, abort_flag, a.status, (uint64_t)a.wait_limit_ns))
-                        break;
-                    // the slot on top of W_g's rows: first filled once every consumer has copied them out
-                    if (lay.wslot && k == 8 && !mbar_wait(wdone, 0, abort_flag, a.status, (uint64_t)a.wait_limit_ns))
                         break;
                     if (k == a.debug_skip && blockIdx.x == 0) continue;  // fault injection: withhold a stage
                     const int rows = min(RT_STAGE_ROWS, nrows - k * RT_STAGE_ROWS);
@@ -232,7 +209,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt)
                 wfr[nt] = (nt < NT && nt * 8 + g < E)
-                              ? reinterpret_cast<const uint4*>(smem + lay.frag + (size_t)(nt * 8 + g) * WRB + tig * 16)
+                              ? reinterpret_cast<const uint4*>(smem + (size_t)(nt * 8 + g) * WRB + tig * 16)
                               : nullptr;
             const bool w_ok = nstages == 0 || mbar_wait(wbar, 0, abort_flag, a.status, (uint64_t)a.wait_limit_ns);
             constexpr int NWC = WREG ? RT_WREG_D / 32 : 1;  // register copy of the fragments (WREG)
@@ -240,10 +217,6 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
             if constexpr (WREG) {
 #pragma unroll
                 for (int c = 0; c < NWC; ++c) wreg[c] = (c < nchunk && wfr[0] && w_ok) ? wfr[0][4 * c] : zero;
-            }
-            if (lay.wslot) {  // W_g's rows are no longer read: their space may take a stage
-                __syncwarp();
-                if (lane == 0) mbar_arrive(wdone);
             }
             for (int k = warp; w_ok && k < nstages; k += S) {
                 const int s = warp;

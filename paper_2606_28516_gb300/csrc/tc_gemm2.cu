@@ -123,19 +123,25 @@ struct PairTile {
     bool router;  // the router unit of the pair tile (the router inside fc1)
 };
 
+// Kernel variants: the plain dense and grouped GEMMs, the dense GEMM with the router unit (the
+// router inside fc1), and the grouped GEMM whose z rows are gathered by slot. Each variant is its own
+// instantiation, so the plain kernels carry none of the others' code.
+enum Tc2Var { TC2_PLAIN = 0, TC2_ROUTER = 1, TC2_GATHER = 2 };
+
 // Units per 256-row pair tile: the column tiles, plus the router unit when the router runs inside fc1.
-__device__ __forceinline__ int units_per_pair(const TcGemmArgs& a, int n_tiles) {
-    return n_tiles + (a.mode == TC_DENSE && a.fr_E > 0 ? 1 : 0);
+template <int VAR>
+__device__ __forceinline__ int units_per_pair(int n_tiles) {
+    return n_tiles + (VAR == TC2_ROUTER ? 1 : 0);
 }
 
-template <int BN>
+template <int BN, int VAR>
 __device__ __forceinline__ PairTile decode_pair(const TcGemmArgs& a, int unit, int n_tiles, const int* s_prefix) {
     constexpr int BM = T2<BN>::BM;
     PairTile t;
-    const int nup = units_per_pair(a, n_tiles);
+    const int nup = units_per_pair<VAR>(n_tiles);
     const int mp = unit / nup;
     t.n0 = (unit % nup) * BN;
-    t.router = (unit % nup) == n_tiles;
+    t.router = VAR == TC2_ROUTER && (unit % nup) == n_tiles;
     if (a.mode == TC_GROUPED) {
         int e = 0;
         while (e + 1 < a.E && s_prefix[e + 1] <= mp) ++e;
@@ -150,7 +156,7 @@ __device__ __forceinline__ PairTile decode_pair(const TcGemmArgs& a, int unit, i
     return t;
 }
 
-template <int BN_, int MODE>
+template <int BN_, int MODE, int VAR>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
     tc_gemm2_kernel(const __grid_constant__ TcGemmArgs a) {
     using C = T2<BN_>;
@@ -219,7 +225,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         const uint16_t* b = static_cast<const uint16_t*>(a.out_bias);
         for (int n = threadIdx.x; n < a.N; n += NUM_EPI * 32) s_bias[n] = __uint_as_float((uint32_t)b[n] << 16);
     }
-    if (MODE == TC_DENSE && a.fr_E > 0 && threadIdx.x < a.fr_E)  // the router's bias (a weight)
+    if (VAR == TC2_ROUTER && threadIdx.x < a.fr_E)  // the router's bias (a weight)
         s_frb[threadIdx.x] = __uint_as_float((uint32_t) static_cast<const uint16_t*>(a.fr_bias)[threadIdx.x] << 16);
     // Tensor memory for the pair: allocated collectively by one warp of each CTA. The two CTAs
     // must see the same base (the even CTA's MMAs name it for both); a mismatch aborts cleanly.
@@ -330,7 +336,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         m_pairs = s_prefix[a.E];
     else
         m_pairs = (int)((a.M + 2 * BM - 1) / (2 * BM));
-    const int num_units = tmem_ok ? m_pairs * units_per_pair(a, n_tiles) : 0;
+    const int num_units = tmem_ok ? m_pairs * units_per_pair<VAR>(n_tiles) : 0;
     const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
 
     if (warp == WARP_TMA) {
@@ -340,18 +346,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         // otherwise lane 0 runs alone.
         const uint32_t full_leader0 = map_to_rank(full_bar(0), 0);
         const uint64_t pol_a = l2_policy_evict_first();
-        const bool gather = MODE == TC_GROUPED && a.a1_rows != nullptr;
+        constexpr bool gather = VAR == TC2_GATHER;
         bool waited = a.pdl_wait_role != 2;  // role 2: wait before the first t-segment load
         int stage = 0;
         uint32_t ph = 0;
         bool ok = gather || lane == 0;
         for (int u = cid; u < num_units && ok; u += ncl) {
-            const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
+            const PairTile t = decode_pair<BN, VAR>(a, u, n_tiles, s_prefix);
             const int am = (int)(t.m0 + (int64_t)rank * BM);
             // the router unit: CTA r supplies W_g rows [16 r, +16) of the 256 x 32 MMA
-            const int bn = (MODE == TC_DENSE && t.router) ? (int)rank * 16 : t.n0 + (int)rank * BH;
-            const uint32_t stage_tx = (MODE == TC_DENSE && t.router) ? 2u * (A_BYTES + C::FR_B_BYTES)
-                                                                     : 2u * STAGE_BYTES;
+            const int bn = t.router ? (int)rank * 16 : t.n0 + (int)rank * BH;
+            const uint32_t stage_tx = t.router ? 2u * (A_BYTES + C::FR_B_BYTES) : 2u * STAGE_BYTES;
             const int nkb_t = (MODE == TC_GROUPED && a.dense_last && t.e == a.E - 1) ? nk1 : nkb;
             int32_t gr[4] = {0, 0, 0, 0};
             if (gather) {  // this lane's four slots; slots past M take the last one (their rows are dropped)
@@ -366,7 +371,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
             for (int kb = 0; kb < nkb_t; ++kb) {
                 int w_ok = 1;
                 if (lane == 0) w_ok = mbar_wait(empty_bar(stage), ph ^ 1, abort_flag, a.status, lim);
-                if (gather) w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+                if constexpr (gather) w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
                 if (!w_ok) {
                     ok = false;
                     break;
@@ -417,7 +422,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         if (leader && lane == 0) {
             const uint32_t idesc_t = idesc_bf16_f32(2 * BM, BN);
             const uint32_t idesc_r = idesc_bf16_f32(2 * BM, 32);  // the router unit: 256 x 32
-            const int nup = units_per_pair(a, n_tiles);
+            const int nup = units_per_pair<VAR>(n_tiles);
             // Stage s's descriptors are the stage-0 ones plus the byte offset / 16 in the start
             // address field (every shared address here is below 256 KB, so the field never carries).
             const uint64_t dA0 = sdesc_kmajor_sw128(smem_u32(sm));
@@ -430,9 +435,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                 if (!mbar_wait(tempty_bar(acc), aph ^ 1, abort_flag, a.status, lim)) break;
                 tc_fence_after();
                 const uint32_t dtm = tmem_base + acc * BN;
-                const uint32_t idesc = (MODE == TC_DENSE && u % nup == n_tiles) ? idesc_r : idesc_t;
+                const uint32_t idesc = (VAR == TC2_ROUTER && u % nup == n_tiles) ? idesc_r : idesc_t;
                 int nkb_t = nkb;  // the dense path's group: the z x W2 segment alone
-                if (MODE == TC_GROUPED && a.dense_last && decode_pair<BN>(a, u, n_tiles, s_prefix).e == a.E - 1)
+                if (MODE == TC_GROUPED && a.dense_last && decode_pair<BN, VAR>(a, u, n_tiles, s_prefix).e == a.E - 1)
                     nkb_t = nk1;
                 for (int kb = 0; kb < nkb_t; ++kb) {
                     if (!mbar_wait(full_bar(stage), ph, abort_flag, a.status, lim)) {
@@ -488,7 +493,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
         uint32_t aph = 0;
         int fr_it = 0;  // router units handled so far (the router inside fc1)
         for (int u = cid; u < num_units; u += ncl) {
-            const PairTile t = decode_pair<BN>(a, u, n_tiles, s_prefix);
+            const PairTile t = decode_pair<BN, VAR>(a, u, n_tiles, s_prefix);
             const int64_t mrow = t.m0 + (int64_t)rank * BM + q * 32 + lane;
             // the token's routing word, loaded before the accumulator wait so that the wait hides it
             const uint32_t rtw = (MODE == TC_DENSE && a.rt_info && mrow < t.hi) ? (uint32_t)a.rt_info[mrow] : 0u;
@@ -496,7 +501,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
             const float2 ln = (a.ln_stats && mrow < t.hi) ? a.ln_stats[mrow] : make_float2(0.f, 1.f);
             if (!mbar_wait(tfull_bar(acc), aph, abort_flag, a.status, lim)) break;
             tc_fence_after();
-            if (MODE == TC_DENSE && t.router) {
+            if (VAR == TC2_ROUTER && t.router) {
                 // The router unit: accumulator columns [0, E) of this lane's row hold W_g x. The four
                 // warps of the first column group (one per lane quarter) add b_g, take the argmax
                 // (lowest index on ties), count each expert's rows of the quarter by ballots, and
@@ -719,17 +724,16 @@ int tc2_pick_bn(int mode, int N) {
     return 0;
 }
 
-template <int BN>
+template <int BN, int MODE, int VAR>
 static cudaError_t launch2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     using C = T2<BN>;
-    const void* fn = a.mode == TC_GROUPED ? (const void*)tc_gemm2_kernel<BN, TC_GROUPED>
-                                          : (const void*)tc_gemm2_kernel<BN, TC_DENSE>;
+    const void* fn = (const void*)tc_gemm2_kernel<BN, MODE, VAR>;
     const cudaError_t e = smem_attr_once(fn, C::SMEM);
     if (e != cudaSuccess) return e;
     const int n_tiles = a.N / BN;
     int64_t m_pairs = (a.M + 2 * C::BM - 1) / (2 * C::BM);
     if (a.mode == TC_GROUPED) m_pairs += a.E;
-    const int64_t units = m_pairs * (n_tiles + (a.mode == TC_DENSE && a.fr_E > 0 ? 1 : 0));
+    const int64_t units = m_pairs * (n_tiles + (VAR == TC2_ROUTER ? 1 : 0));
     int64_t clusters = units < num_sms / 2 ? units : num_sms / 2;
     if (clusters <= 0) return cudaSuccess;
     cudaLaunchConfig_t cfg = {};
@@ -742,8 +746,14 @@ static cudaError_t launch2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     attr_pdl[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr_pdl;
     cfg.numAttrs = 1;
-    if (a.mode == TC_GROUPED) return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<BN, TC_GROUPED>, a);
-    return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<BN, TC_DENSE>, a);
+    return cudaLaunchKernelEx(&cfg, tc_gemm2_kernel<BN, MODE, VAR>, a);
+}
+
+template <int BN>
+static cudaError_t launch2_var(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
+    if (a.mode == TC_GROUPED)
+        return a.a1_rows ? launch2<BN, TC_GROUPED, TC2_GATHER>(a, num_sms, s) : launch2<BN, TC_GROUPED, TC2_PLAIN>(a, num_sms, s);
+    return a.fr_E > 0 ? launch2<BN, TC_DENSE, TC2_ROUTER>(a, num_sms, s) : launch2<BN, TC_DENSE, TC2_PLAIN>(a, num_sms, s);
 }
 
 cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
@@ -763,9 +773,9 @@ cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
                        !a.fr_info || !a.fr_counts))
         return cudaErrorInvalidValue;
     if (a.a1_rows && a.mode != TC_GROUPED) return cudaErrorInvalidValue;
-    if (bn == 256) return launch2<256>(a, num_sms, s);
-    if (bn == 192) return launch2<192>(a, num_sms, s);
-    return launch2<128>(a, num_sms, s);
+    if (bn == 256) return launch2_var<256>(a, num_sms, s);
+    if (bn == 192) return launch2_var<192>(a, num_sms, s);
+    return launch2_var<128>(a, num_sms, s);
 }
 
 }  // namespace cm
