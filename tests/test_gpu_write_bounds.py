@@ -3,9 +3,9 @@
 Every output buffer here has 64 extra rows (entries) after the T it is called with, filled with a
 sentinel; after the call the first T rows must be finite and the tail must still hold the sentinel,
 bit for bit. Covered: the forward in its forms (factorised, folded, materialised, one residual
-matrix, the folded input LayerNorm, class tokens with b2), the dense FFN, the LayerNorm and the
-routing copies, at T = 1, 17 and 300 on the bf16 DeiT-S layer and at T = 17 on the fp32 DeiT-T
-layer."""
+matrix, the folded input LayerNorm, class tokens with b2, the router inside fc1 on the factorised
+and folded forms), the dense FFN, the LayerNorm and the routing copies, at T = 1, 17 and 300 on the
+bf16 DeiT-S layer and at T = 17 on the fp32 DeiT-T layer."""
 import numpy as np
 import pytest
 import torch
@@ -68,18 +68,25 @@ def test_outputs_stay_within_T(workload, shape, T):
             calls["scaled"] = lambda o: cm.clearmoe_ffn_forward_scaled(h.h, x, D["W1"], D["b1"], D["U"], D["S"],
                                                                        D["Vh"], D["R"], D["scales"], D["Wg"],
                                                                        D["bg"], o)
+            calls["router in fc1"] = lambda o: cm.clearmoe_ffn_forward_ex(h.h, x, *args, o, router_in_fc1=True)
+            calls["router in fc1, folded"] = lambda o: cm.clearmoe_ffn_forward_folded_ex(
+                h.h, x, D["W1"], D["b1"], comb, D["Wg"], D["bg"], o, router_in_fc1=True)
         for what, call in calls.items():
             buf = _padded(T, shape.d, dt)
             call(buf[:T])
             _check(buf, T, what)
-        cm.clearmoe_ffn_forward(h.h, x, *args, _padded(T, shape.d, dt)[:T])
-        idx, perm = (torch.full((T + PAD,), -7, dtype=torch.int32, device="cuda") for _ in range(2))
-        counts = torch.full((shape.E + PAD,), -7, dtype=torch.int32, device="cuda")
-        offsets = torch.full((shape.E + 1 + PAD,), -7, dtype=torch.int32, device="cuda")
-        cm.clearmoe_get_routing(h.h, idx, counts, offsets, perm)
-        torch.cuda.synchronize()
-        assert cm.clearmoe_layer_status(h.h) == 0
-    for buf, n, what in ((idx, T, "idx"), (perm, T, "perm"), (counts, shape.E, "counts"),
-                         (offsets, shape.E + 1, "offsets")):
-        b = buf.cpu().numpy()
-        assert np.all(b[:n] >= 0) and np.all(b[n:] == -7), f"{what}: wrote past its {n} entries"
+        routing = []  # the routing copies after the default forward and after the router inside fc1
+        for fused in ((False, True) if shape.dtype == "bf16" else (False,)):
+            cm.clearmoe_ffn_forward_ex(h.h, x, *args, _padded(T, shape.d, dt)[:T], router_in_fc1=fused)
+            idx, perm = (torch.full((T + PAD,), -7, dtype=torch.int32, device="cuda") for _ in range(2))
+            counts = torch.full((shape.E + PAD,), -7, dtype=torch.int32, device="cuda")
+            offsets = torch.full((shape.E + 1 + PAD,), -7, dtype=torch.int32, device="cuda")
+            cm.clearmoe_get_routing(h.h, idx, counts, offsets, perm)
+            torch.cuda.synchronize()
+            assert cm.clearmoe_layer_status(h.h) == 0
+            routing.append((fused, idx, perm, counts, offsets))
+    for fused, idx, perm, counts, offsets in routing:
+        for buf, n, what in ((idx, T, "idx"), (perm, T, "perm"), (counts, shape.E, "counts"),
+                             (offsets, shape.E + 1, "offsets")):
+            b = buf.cpu().numpy()
+            assert np.all(b[:n] >= 0) and np.all(b[n:] == -7), f"{what} (router in fc1: {fused}): wrote past its {n} entries"
