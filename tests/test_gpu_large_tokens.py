@@ -6,9 +6,9 @@ DeiT-B width (d = 768, bf16, E = 8) that space holds about 2,620 rows per CTA, s
 tokens (152 CTAs) the words go to idx in global memory and the ranks come from the match-mask loop
 instead of the per-stage ballots (Algorithm 3, "sort z by a": the same stable order either way).
 This file runs that path at T = 600,000 (3,948 rows per CTA): routing bit-exact against the oracle
-on every token outside near ties, outputs on a seeded sample plus the whole smallest expert, and
-the handle-free routing entry point at the same size, whose idx then carries the packed words
-between its two kernels."""
+on every token outside near ties, outputs on a seeded sample plus the whole smallest expert, the
+handle-free routing entry point at the same size, whose idx then carries the packed words between
+its two kernels, and the router inside fc1, whose slot kernel then spans 4,688 ranges."""
 import numpy as np
 import pytest
 import torch
@@ -68,3 +68,22 @@ def test_route_noalloc_at_600k_tokens(large_layer):
     assert int(status.item()) == 0
     gr = {k: g.cpu().numpy().astype(np.int64) for k, g in zip(("a", "counts", "offsets", "perm"), got)}
     check_routing(gr, L["x"], L["Wg"], L["bg"])
+
+
+def test_router_in_fc1_at_600k_tokens(large_layer):
+    """The router inside fc1 at the same size: 4,688 ranges of 128 tokens for its slot kernel, routing
+    bit-exact on every token outside near ties, outputs on a seeded sample plus the smallest expert."""
+    L = large_layer
+    s = L["shape"]
+    D = synth.to_torch(L)
+    with handle_for(L) as h:
+        out = torch.full((s.T, s.d), float("nan"), device="cuda", dtype=torch.bfloat16)
+        cm.clearmoe_ffn_forward_ex(h.h, D["x"], D["W1"], D["b1"], D["U"], D["S"], D["Vh"], D["residuals"],
+                                   D["Wg"], D["bg"], out, router_in_fc1=True)
+        gr = get_routing(h, s.T, s.E)
+        assert cm.clearmoe_layer_status(h.h) == 0
+    check_routing(gr, L["x"], L["Wg"], L["bg"])
+    rows = sample_rows(gr, s.T, n=4096, seed=13)
+    y = oracle_rows(L, rows, gr["a"][rows])
+    err = out_error(out[torch.from_numpy(rows).cuda()], y, "bf16")
+    assert err <= tol("bf16"), f"{s.name} router in fc1: {err:.3e}"
