@@ -151,3 +151,16 @@ def test_unsupported_combinations(workload):
             cm.clearmoe_ffn_forward_ex(h.h, Dt["x"][:50], Dt["W1"], Dt["b1"], Dt["U"], Dt["S"], Dt["Vh"],
                                        Dt["residuals"], Dt["Wg"], Dt["bg"], out, router_in_fc1=True)
         assert e.value.code == cm.EUNSUPPORTED
+
+
+def test_single_expert_is_token_order():
+    """E = 1: every token takes expert 0 and the permutation is the identity."""
+    L = synth.make_layer(synth.DEIT_SMALL_BF16.with_(T=777, E=1, n_cal=2000))
+    gr = _check(L)
+    assert np.array_equal(gr["perm"], np.arange(777)) and np.all(gr["a"] == 0)
+
+
+def test_widest_layer():
+    """d = 1,024 (16 K blocks in the router unit) and H = 4,096 (the widest fc1 the 2-SM kernel
+    stages a bias for)."""
+    _check(synth.make_layer(synth.LayerShape("d1024_bf16", 3000, 1024, 4096, 4, 128, "bf16", n_cal=4000)))
