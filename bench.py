@@ -46,7 +46,7 @@ NOMINAL_PEAKS = {"hbm_gbs": 7900.0, "bf16_tflops": 2250.0}
 # fp32 CUDA-core peak of the fp32 layer: 152 SMs x 128 fp32 lanes x 2 FLOP (FMA) x 2.07 GHz
 FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 STAGES = ("route", "fc1_gelu", "basis", "grouped")
-KERNEL_OF_STAGE = {"route": "cm::route_kernel<1, 1>",
+KERNEL_OF_STAGE = {"route": "cm::route_tc_kernel",
                    "fc1_gelu": "cm::tc_gemm2_kernel<256, 0, 0> (2-SM dense, rows stored at their routing slots)",
                    "basis": "cm::tc_gemm2_kernel<128, 0, 0> (2-SM dense, column scale)",
                    "grouped": "cm::tc_gemm2_kernel<256, 2, 0> (2-SM grouped, rows stored at perm[slot])"}

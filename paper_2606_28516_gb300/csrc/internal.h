@@ -239,5 +239,11 @@ int current_device_sms();
 // Encode a 2-D bf16 row-major [rows x cols] tensor map, box {64, box_rows}, 128-byte swizzle.
 int encode_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols,
                      int box_rows);
+// The same [rows x cols] matrix (cols % 64 == 0) viewed as {64 columns, rows, cols / 64 chunks}
+// with boxes of 64 x box_rows x box_chunks, 128-byte swizzle: a box lands in shared memory as
+// box_chunks consecutive [box_rows x 64] tiles (one K block each) and reads box_chunks x 128
+// contiguous bytes of each of its rows.
+int encode_tmap_bf16_chunks(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows,
+                            int box_chunks);
 
 }  // namespace cm

@@ -2,22 +2,27 @@
 //   logits = W_g x + b_g (linear router), a = argmax (lowest index on ties),
 //   per-expert histogram, exclusive prefix sum, and the stable permutation perm[slot] = token.
 //
-// route_kernel: CTA b owns a contiguous range of `chunk` tokens and never waits for another CTA.
-//   phase 1: stream x once from HBM, router logits and argmax per token, the range's histogram.
-//            bf16: one CTA per SM; a producer thread copies the CTA's rows, 16 at a time, into a
-//            ring of shared-memory stages with 1-D bulk copies (mbarrier-tracked, so the bytes in
-//            flight cost no registers) and eight consumer warps take one 16-row stage each;
-//   then:    the histogram row goes to cta_counts, and each token's rank among the range's
-//            earlier tokens of its expert (warp match masks) to tinfo, packed with the expert.
-// The slot of token t in range c is offsets[e] + (tokens of e in ranges before c) + its rank, in
-// token order within each expert, which makes the sort stable. It is formed by the consumer of
-// the routing: the fc1 epilogue of the 2-SM GEMM (which then stores z rows at their slots and
-// writes perm), or route_finalize_kernel (perm and inv ahead of the other paths).
-// bf16 tokens: the d x E contraction runs on the legacy warp MMA (m16n8k16, fp32 accumulate):
-// x fragments from the shared-memory stage, W_g fragments staged once in shared memory (reading
-// them through L1 in the inner loop was measured slower), and the K order of each fragment is
-// permuted identically for x and W_g, which leaves every dot product unchanged.
-// fp32 tokens: fp32 FMA on the CUDA cores (an fp32 router decision needs fp32 products).
+// Every routing kernel gives CTA b a contiguous range of `chunk` tokens, and no CTA ever waits for
+// another: each writes its range's histogram to cta_counts and, per token, (expert | rank among the
+// range's earlier tokens of that expert << 8) to tinfo. The slot of token t in range c is
+// offsets[e] + (tokens of e in ranges before c) + its rank, in token order within each expert,
+// which makes the sort stable. It is formed by the consumer of the routing: the fc1 epilogue of
+// the 2-SM GEMM (which then stores z rows at their slots and writes perm), or route_finalize_kernel
+// (perm and inv ahead of the other paths).
+//
+// bf16 tokens (route_tc_kernel): the d x E contraction runs on the tensor cores. One CTA per SM
+//   streams its range as 128-row blocks into a ring of shared-memory stages, each stage nkc K blocks
+//   (64 columns) of a block, loaded as 16 TMA boxes of 8 rows x nkc K blocks (128-byte swizzle), so
+//   that every box reads nkc x 128 contiguous bytes of each of its rows (a box of 128 rows x 64
+//   columns, 128 bytes per row, kept DRAM 45 % busy); W_g sits in shared memory as the B operand (16
+//   rows, rows past E read as zero). One thread issues tcgen05.mma (M = 128, N = 16, K = 16, fp32
+//   accumulator in tensor memory, two accumulators); four epilogue warps, one per TMEM lane quarter,
+//   read their 32 rows' logits with tcgen05.ld, take the argmax per row (one row per lane, no
+//   shuffles) and the ranks by one ballot per expert, exchanging the four warps' counts through
+//   shared memory, and write idx and the final per-token word. A range's last, partial block loads
+//   only the boxes that hold its rows, so that at most 7 rows past the range are read.
+// fp32 tokens (route_f32_kernel): fp32 FMA on the CUDA cores (an fp32 router decision needs fp32
+//   products), one row per lane, then the ranks from warp match masks.
 // Class tokens (cls_stride > 0, t % cls_stride == 0) skip the router: idx = E, no histogram entry
 // and no rank; their slots T - n_cls + t / cls_stride follow the experts' (the dense path).
 #include <mutex>
@@ -27,29 +32,6 @@
 
 namespace cm {
 
-constexpr int RT_THREADS = 256;                 // fp32 router: 8 warps
-constexpr int RT_BF16_THREADS = 288;            // bf16 router: 8 consumer warps + 1 producer warp
-constexpr int RT_MAX_WARPS = RT_BF16_THREADS / 32;
-constexpr int RT_STAGE_ROWS = 16;               // rows per ring stage (one MMA row group)
-
-__device__ __forceinline__ uint4 ldg_nc_v4(const uint4* p) {
-    uint4 v;
-    asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
-    return v;
-}
-
-__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1,
-                                               uint32_t a2, uint32_t a3, uint32_t b0,
-                                               uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-        "{%8,%9}, {%0,%1,%2,%3};"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
 // better (value, index) with the lower index winning exact ties
 __device__ __forceinline__ void arg_better(float& bv, int& be, float v, int e) {
     if (v > bv || (v == bv && e < be)) {
@@ -58,388 +40,373 @@ __device__ __forceinline__ void arg_better(float& bv, int& be, float v, int e) {
     }
 }
 
-// bf16: W_g rows in shared memory with a 64-byte pad, so that the 16-byte B-fragment reads of a
-// quarter warp (two rows, four 16-byte column groups each) hit all 32 banks once. Token stages
-// stay contiguous (one bulk copy per 16 rows, 2-way conflicts on the A-fragment reads): neither
-// per-row copies into padded rows nor a 128-byte-swizzled tensor copy was measured faster.
-__host__ __device__ inline int wrow_bytes(int d) { return d * 2 + 64; }
-__host__ __device__ inline size_t frag_bytes(int dtype, int d, int E) {
-    if (dtype == CLEARMOE_BF16) return (size_t)E * wrow_bytes(d);
-    return (size_t)E * d * 4;
-}
+// ------------------------------------------------------------------ bf16: tcgen05 router
+constexpr int RTC_THREADS = 192;  // warps 0-3: epilogue (TMEM lane quarters), 4: producer, 5: MMA
+constexpr int RTC_BM = 128;       // rows per block (the MMA's M)
+constexpr int RTC_BK = 64;        // columns per K block (128 bytes)
+constexpr int RTC_BOX_ROWS = 8;   // rows per TMA box: one 128-byte swizzle atom per K block
+constexpr int RTC_WBOX_BYTES = 16 * RTC_BK * 2;  // W_g's box per K block: 16 rows, 2 KB
+constexpr int RTC_MAX_STAGES = 16;
+constexpr int RTC_TMEM_COLS = 32;  // two 16-column accumulators
+#ifndef RTC_NKC_MAX
+#define RTC_NKC_MAX 6  // K blocks per stage at most (6 x 128 contiguous bytes of each row per box)
+#endif
+// dynamic shared memory: the 227 KB a CTA may hold, less the kernel's static arrays and a margin
+constexpr size_t RTC_SMEM_CAP = 227 * 1024 - 1024 - 256;
 
-// Dynamic shared memory: [router weights] [bf16: ring of S stages] [bf16: 2 S + 1 mbarriers]
-// [per-row word: expert | local rank << 8, when chunk words fit; else that word lives in idx in
-// global memory (the CTA's own rows, visible block-wide after __syncthreads) until phase 2
-// rewrites idx with the expert alone], so the footprint does not grow with T.
-// The ring has one slot per consumer warp (S = 8, or 4 when eight stages do not fit): consumer
-// warp w alone reads slot w, for stages w, w + S, ..., so each of its mbarrier waits is for the
-// phase right after the one it last consumed (a parity wait cannot tell phases two apart).
-constexpr size_t RT_SMEM_MAX = 220 * 1024;
-struct RouteLayout {
-    size_t ring, bars, sidx, scnt, total;
-    int S, stage_bytes;
-    bool sidx_in_smem;
+struct RouteTcArgs {
+    RouteArgs r;
+    CUtensorMap tmX;  // x [T x d] as {64, T, d / 64}: boxes of 64 x 8 rows x nkc K blocks
+    CUtensorMap tmW;  // W_g [E x d]: boxes of 64 columns x 16 rows (rows past E read as zero)
+    int chunk;
 };
-__host__ __device__ inline RouteLayout route_layout(int dtype, int d, int E, int chunk) {
-    RouteLayout L;
-    const size_t frag = (frag_bytes(dtype, d, E) + 127) & ~(size_t)127;
-    L.stage_bytes = RT_STAGE_ROWS * d * 2;
-    L.S = 0;
-    L.ring = frag;
-    if (dtype == CLEARMOE_BF16)  // eight slots when they fit beside W_g and the barriers, else four
-        L.S = (L.ring + 8 * (size_t)L.stage_bytes + 17 * 8 <= RT_SMEM_MAX) ? 8 : 4;
-    L.bars = (L.ring + (size_t)L.S * L.stage_bytes + 15) & ~(size_t)15;
-    L.sidx = L.bars + (size_t)(2 * L.S + 1) * 8;  // bf16: ring barriers + the W_g barrier
-    // expert ids of the CTA's rows: in shared memory when they fit, else read back from idx
-    // per row a 4-byte word; bf16 also keeps each 16-row stage's per-expert counts (2 bytes each)
-    const size_t rows_bytes =
-        (size_t)chunk * 4 + (dtype == CLEARMOE_BF16 ? (size_t)((chunk + 15) / 16) * CM_MAX_E * 2 : 0);
-    L.scnt = L.sidx + (size_t)chunk * 4;
-    L.sidx_in_smem = L.sidx + rows_bytes <= RT_SMEM_MAX;
-    L.total = L.sidx + (L.sidx_in_smem ? rows_bytes : 0);
+
+// A stage holds nkc K blocks of a 128-row block: 16 boxes of 8 rows, box b at b * nkc KB, its K
+// block c at + c KB (an 8 x 128-byte swizzle atom), so the MMA reads K block c of the 128 rows
+// with 8-row atoms nkc KB apart. Each box reads nkc x 128 contiguous bytes of each of its rows.
+// Dynamic shared memory: [W_g: d / 64 boxes of 2 KB] [ring: S stages] [2 S + 6 mbarriers] [TMEM
+// base]; the base is aligned to 1024 bytes in the kernel (the swizzle atom). nkc is the largest
+// divisor of d / 64 up to RTC_NKC_MAX that leaves room for two stages.
+struct RouteTcLayout {
+    int nkc, S;
+    size_t stage_bytes, w_bytes, ring, bars, total;
+};
+__host__ __device__ inline RouteTcLayout route_tc_layout(int d) {
+    RouteTcLayout L;
+    const int nk = d / RTC_BK;
+    L.w_bytes = (size_t)nk * RTC_WBOX_BYTES;
+    L.ring = L.w_bytes;
+    const size_t avail = RTC_SMEM_CAP - 1024 - L.w_bytes - (2 * RTC_MAX_STAGES + 6) * 8 - 16;
+    L.nkc = 1;
+    L.S = 1;
+    for (int c = 1; c <= RTC_NKC_MAX && c <= nk; ++c) {
+        if (nk % c) continue;
+        int S = (int)(avail / ((size_t)RTC_BM * c * RTC_BK * 2));
+        if (S > RTC_MAX_STAGES) S = RTC_MAX_STAGES;
+        if (S < 2) continue;
+        L.nkc = c;
+        L.S = S;
+    }
+    L.stage_bytes = (size_t)RTC_BM * L.nkc * RTC_BK * 2;
+    L.bars = L.ring + (size_t)L.S * L.stage_bytes;
+    L.total = 1024 + L.bars + (size_t)(2 * L.S + 6) * 8 + 16;
     return L;
 }
-static size_t route_smem(int dtype, int d, int E, int chunk) { return route_layout(dtype, d, E, chunk).total; }
 
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-                 "l"(src), "r"(bytes), "r"(bar)
-                 : "memory");
+__global__ void __launch_bounds__(RTC_THREADS, 1) route_tc_kernel(const __grid_constant__ RouteTcArgs A) {
+    const RouteArgs& a = A.r;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    __shared__ int s_cnt[2][4][CM_MAX_E];  // per block (double-buffered): each quarter warp's expert counts
+    __shared__ float s_b[CM_MAX_E], s_g[CM_MAX_E];
+    __shared__ int s_abort;
+    const uint32_t raw = smem_u32(smem_raw);
+    unsigned char* sm = smem_raw + ((1024 - (raw & 1023)) & 1023);
+    const RouteTcLayout lay = route_tc_layout(a.d);
+    const int S = lay.S;
+    const uint32_t w_u32 = smem_u32(sm);
+    const uint32_t ring_u32 = w_u32 + (uint32_t)lay.ring;
+    const uint32_t bar0 = w_u32 + (uint32_t)lay.bars;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + lay.bars + (size_t)(2 * S + 6) * 8);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
+    const uint32_t wbar = bar0 + 8u * (2 * S);
+    auto tfull_bar = [&](int i) { return bar0 + 8u * (2 * S + 1 + i); };
+    auto tempty_bar = [&](int i) { return bar0 + 8u * (2 * S + 3 + i); };
+    const uint32_t drain_bar = bar0 + 8u * (2 * S + 5);
+    volatile int* abort_flag = &s_abort;
+    const uint64_t lim = (uint64_t)a.wait_limit_ns;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int E = a.E, nk = a.d / RTC_BK, nkc = lay.nkc, nh = nk / nkc;
+    const uint32_t stage_bytes = (uint32_t)lay.stage_bytes, box_bytes = (uint32_t)nkc * RTC_BOX_ROWS * RTC_BK * 2;
+    const int64_t row0 = (int64_t)blockIdx.x * A.chunk;
+    const int nrows = (int)max((int64_t)0, min((int64_t)A.chunk, a.T - row0));
+    const int nblk = (nrows + RTC_BM - 1) / RTC_BM;
+    const bool producer = warp == 4 && lane == 0, issuer = warp == 5 && lane == 0;
+
+    if (tid == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full_bar(s), 1);   // the producer's arrive + the stage's bytes
+            mbar_init(empty_bar(s), 1);  // one commit once the stage's MMAs have read it
+        }
+        mbar_init(wbar, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(tfull_bar(i), 1);   // one commit per block
+            mbar_init(tempty_bar(i), 4);  // the four epilogue warps
+        }
+        mbar_init(drain_bar, 1);
+        s_abort = 0;
+        mbar_fence_init();
+    }
+    if (warp == 5) tmem_alloc(smem_u32(tmem_slot), RTC_TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    // W_g (a weight, not written by the previous kernel) is requested before the launch-overlap wait
+    if (producer && nblk > 0) {
+        mbar_arrive_expect_tx(wbar, (uint32_t)(nk * RTC_WBOX_BYTES));
+        for (int kc = 0; kc < nk; ++kc) tma_load_2d(w_u32 + kc * RTC_WBOX_BYTES, &A.tmW, kc * RTC_BK, 0, wbar);
+    }
+    pdl_wait();  // from here on the previous kernel's results (x) are read and outputs written
+    // the next kernel may start now (its CTAs set up, and may read x, while this one streams):
+    // released only after the wait, so every kernel before this one has completed by then
+    pdl_launch_dependents();
+    if (tid < CM_MAX_E) {
+        s_b[tid] = tid < E ? bf16_to_f32(static_cast<const uint16_t*>(a.bg)[tid]) : 0.f;
+        s_g[tid] = (a.ln_stats && tid < E) ? a.ln_wsum[tid] : 0.f;
+    }
+    __syncthreads();
+    const uint32_t tmem = *tmem_slot;
+
+    if (producer) {
+        // stage k = K blocks [h nkc, +nkc) of block j, with j = k / nh and h = k % nh; ring slot k % S
+        int k = 0;
+        bool ok = true;
+        for (int j = 0; j < nblk && ok; ++j) {
+            const int rows = min(RTC_BM, nrows - j * RTC_BM);
+            const int r = (int)(row0 + (int64_t)j * RTC_BM);  // T <= 2^30
+            const int nbox = (rows + RTC_BOX_ROWS - 1) / RTC_BOX_ROWS;  // the last block may be partial
+            const uint32_t bytes = (uint32_t)nbox * box_bytes;
+            for (int h = 0; h < nh; ++h, ++k) {
+                const int s = k % S;
+                if (!mbar_wait(empty_bar(s), ((k / S) & 1) ^ 1, abort_flag, a.status, lim)) {
+                    ok = false;
+                    break;
+                }
+                if (k == a.debug_skip && blockIdx.x == 0) continue;  // fault injection: withhold a stage
+                const uint32_t dst = ring_u32 + (uint32_t)s * stage_bytes;
+                mbar_arrive_expect_tx(full_bar(s), bytes);
+                for (int b = 0; b < nbox; ++b)
+                    tma_load_3d(dst + (uint32_t)b * box_bytes, &A.tmX, 0, r + b * RTC_BOX_ROWS, h * nkc, full_bar(s));
+            }
+        }
+        if (!ok)  // gave up: let the copies in flight land before the CTA moves on
+            for (int j = max(0, k - S); j < k; ++j)
+                mbar_wait(full_bar(j % S), (j / S) & 1, nullptr, a.status, 10000000ull);
+        if (nblk > 0) mbar_wait(wbar, 0, nullptr, a.status, 10000000ull);  // W_g's boxes have landed too
+    } else if (issuer) {
+        const uint32_t idesc = idesc_bf16_f32(RTC_BM, 16);
+        // a K block's descriptor is the ring base's plus the byte offset / 16 (addresses stay below
+        // 256 KB): 8-row atoms nkc KB apart in x's stages, 1 KB apart in W_g's boxes
+        const uint64_t dA0 = sdesc_kmajor_sw128_sbo(ring_u32, (uint32_t)nkc * 1024u);
+        const uint64_t dW0 = sdesc_kmajor_sw128(w_u32);
+        bool ok = nblk == 0 || mbar_wait(wbar, 0, abort_flag, a.status, lim);
+        int k = 0;
+        for (int j = 0; j < nblk && ok; ++j) {
+            const int acc = j & 1;
+            if (!mbar_wait(tempty_bar(acc), ((j >> 1) & 1) ^ 1, abort_flag, a.status, lim)) break;
+            tc_fence_after();
+            const uint32_t dtm = tmem + (uint32_t)acc * 16;
+            for (int h = 0; h < nh; ++h, ++k) {
+                const int s = k % S;
+                if (!mbar_wait(full_bar(s), (k / S) & 1, abort_flag, a.status, lim)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                for (int c = 0; c < nkc; ++c) {
+                    const uint64_t da = dA0 + (uint64_t)((s * stage_bytes + c * 1024u) >> 4);
+                    const uint64_t dw = dW0 + (uint64_t)(((h * nkc + c) * RTC_WBOX_BYTES) >> 4);
+#pragma unroll
+                    for (int kk = 0; kk < RTC_BK / 16; ++kk)  // 16 columns = 32 bytes = 2 descriptor units
+                        umma_bf16(dtm, da + 2 * kk, dw + 2 * kk, idesc, (h > 0 || c > 0 || kk > 0) ? 1u : 0u);
+                }
+                umma_commit(empty_bar(s));
+            }
+            if (!ok) break;
+            umma_commit(tfull_bar(acc));
+        }
+        umma_commit(drain_bar);  // every MMA issued has completed before tensor memory is released
+        mbar_wait(drain_bar, 0, nullptr, a.status, 10000000ull);
+    } else if (warp < 4) {
+        // epilogue: warp q reads TMEM lanes [32 q, +32) = rows 32 q .. 32 q + 31 of each block. Every
+        // warp runs all nblk iterations (a wait that gave up only skips the work), so the named
+        // barrier below is reached the same number of times by all four.
+        const int q = warp;
+        const unsigned below = (1u << lane) - 1u;
+        const bool lnf = a.ln_stats != nullptr;
+        float bias[CM_MAX_E], gsum[CM_MAX_E];  // b_g and, with the LayerNorm folded, W_g's row sums
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e) {
+            bias[e] = s_b[e];
+            gsum[e] = s_g[e];
+        }
+        int run = 0;  // lane e < E: expert e's rows of the range in the blocks so far
+        for (int j = 0; j < nblk; ++j) {
+            const int acc = j & 1;
+            const int i = j * RTC_BM + q * 32 + lane;  // row within the range
+            const bool valid = i < nrows;
+            const int64_t row = row0 + i;
+            const float2 ln = (lnf && valid) ? a.ln_stats[row] : make_float2(0.f, 1.f);
+            // the warp agrees on the outcome, so that its tcgen05.ld runs on all lanes or none
+            const bool ok = __all_sync(0xffffffffu, mbar_wait(tfull_bar(acc), (j >> 1) & 1, abort_flag, a.status, lim));
+            int esel = -1;  // this lane's expert (E: a class token; -1: no row)
+            if (ok) {
+                tc_fence_after();
+                uint32_t v[16];
+                CM_TMEM_LD_X16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)acc * 16, v);
+                tmem_wait_ld();
+                if (valid) {
+                    float bv = -INFINITY;
+                    int be = 0x7fffffff;
+#pragma unroll
+                    for (int e = 0; e < CM_MAX_E; ++e) {
+                        if (e < E) {
+                            float l = __uint_as_float(v[e]);
+                            if (lnf) l = ln.y * fmaf(-ln.x, gsum[e], l);  // W_g LN(y) = rstd (W_g y - mean g)
+                            arg_better(bv, be, l + bias[e], e);
+                        }
+                    }
+                    esel = be < E ? be : 0;  // only reachable with non-finite logits
+                    if (a.cls_stride > 0 && row % a.cls_stride == 0) esel = E;  // a class token
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty_bar(acc));  // the accumulator may be overwritten
+            // ranks: earlier blocks' rows of the expert + earlier quarters' + earlier lanes'. The lanes
+            // that picked the same expert form one match group; its first lane records the group's size.
+            const unsigned same = __match_any_sync(0xffffffffu, esel);
+            const int rk = __popc(same & below);
+            int* cw = &s_cnt[j & 1][q][0];
+            if (lane < CM_MAX_E) cw[lane] = 0;
+            __syncwarp();
+            if (esel >= 0 && esel < E && rk == 0) cw[esel] = __popc(same);
+            const int* cb = &s_cnt[j & 1][0][0];
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            // lane e: expert e's rows before this warp's (earlier blocks and quarters), and in the block
+            int pre = run, tot = 0;
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) {
+                const int c = lane < CM_MAX_E ? cb[qq * CM_MAX_E + lane] : 0;
+                if (qq < q) pre += c;
+                tot += c;
+            }
+            run += tot;
+            const int base = __shfl_sync(0xffffffffu, pre, (esel >= 0 && esel < E) ? esel : 0);
+            if (ok && valid) {
+                if (a.tinfo != a.idx) a.idx[row] = esel;
+                a.tinfo[row] = esel < E ? esel | ((base + rk) << 8) : E;
+            }
+        }
+        if (q == 0 && lane < E) a.cta_counts[(size_t)blockIdx.x * CM_MAX_E + lane] = run;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 5) tmem_dealloc(tmem, RTC_TMEM_COLS);
 }
 
-// W_g's B fragments held in registers (bf16, E <= 8, d <= RT_WREG_D): 4 registers per 32 columns
-constexpr int RT_WREG_D = 768;
-inline bool route_wreg(int dtype, int d, int E) { return dtype == CLEARMOE_BF16 && E <= 8 && d <= RT_WREG_D; }
+// ------------------------------------------------------------------ fp32 router
+constexpr int RT_THREADS = 256;  // 8 warps
+constexpr size_t RT_F32_SMEM_MAX = 220 * 1024;
 
-template <bool BF16, bool WREG>
-__global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_kernel(const RouteArgs a, const int chunk) {
-    constexpr int NTHREADS = BF16 ? RT_BF16_THREADS : RT_THREADS;
+// Dynamic shared memory: [W_g as fp32] [per-row word: expert | local rank << 8, when chunk words
+// fit; else that word lives in idx in global memory (the CTA's own rows, visible block-wide after
+// __syncthreads) until the finalize kernel rewrites idx with the expert alone], so the footprint
+// does not grow with T.
+struct RouteF32Layout {
+    size_t sidx, total;
+    bool sidx_in_smem;
+};
+__host__ __device__ inline RouteF32Layout route_f32_layout(int d, int E, int chunk) {
+    RouteF32Layout L;
+    L.sidx = ((size_t)E * d * 4 + 127) & ~(size_t)127;
+    L.sidx_in_smem = L.sidx + (size_t)chunk * 4 <= RT_F32_SMEM_MAX;
+    L.total = L.sidx + (L.sidx_in_smem ? (size_t)chunk * 4 : 0);
+    return L;
+}
+
+__global__ void __launch_bounds__(RT_THREADS) route_f32_kernel(const RouteArgs a, const int chunk) {
+    constexpr int NTHREADS = RT_THREADS;
     constexpr int NWARPS = NTHREADS / 32;
-    constexpr int NCONS_MAX = 8;  // warps computing logits (bf16: the first S warps)
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ int s_count[CM_MAX_E];
     __shared__ int s_run[CM_MAX_E];
-    __shared__ int s_wc[RT_MAX_WARPS][CM_MAX_E];
-    __shared__ int s_abort;
+    __shared__ int s_wc[NWARPS][CM_MAX_E];
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int E = a.E, d = a.d;
     const int64_t row0 = (int64_t)blockIdx.x * chunk;
     const int nrows = (int)max((int64_t)0, min((int64_t)chunk, a.T - row0));
-    const int nchunk = d / 32;
-    const int NT = (E + 7) / 8;
-    const RouteLayout lay = route_layout(BF16 ? CLEARMOE_BF16 : CLEARMOE_F32, d, E, chunk);
-    // per-row expert after phase 1: in shared memory when it fits, else read back from idx
+    const RouteF32Layout lay = route_f32_layout(d, E, chunk);
+    // per-row expert after the first pass: in shared memory when it fits, else read back from idx
     uint32_t* sinfo = lay.sidx_in_smem ? reinterpret_cast<uint32_t*>(smem + lay.sidx) : nullptr;
     auto info_of = [&](int i) -> uint32_t { return sinfo ? sinfo[i] : (uint32_t)__ldcg(a.idx + row0 + i); };
-    // bf16 with the words in shared memory: ranks within 16-row stages during phase 1 (scnt holds
-    // each stage's per-expert counts), so that only a scan over stages remains afterwards
-    uint16_t* scnt = (BF16 && sinfo) ? reinterpret_cast<uint16_t*>(smem + lay.scnt) : nullptr;
-    auto record = [&](int i, int e, int rank) {  // phase 1 result of row i: idx, its word, histogram
+    auto record = [&](int i, int e) {  // first-pass result of row i: idx, its word, histogram
         a.idx[row0 + i] = e;
-        if (sinfo) sinfo[i] = (uint32_t)e | ((uint32_t)rank << 8);
+        if (sinfo) sinfo[i] = (uint32_t)e;
         if (e < E) atomicAdd(&s_count[e], 1);  // e == E: a class token
     };
-
     if (tid < CM_MAX_E) s_count[tid] = 0;
-    if (tid == 0) s_abort = 0;
 
-    // ---------------- phase 1: router logits + argmax for this CTA's rows
-    if constexpr (BF16) {
-        const int S = lay.S, SB = lay.stage_bytes;
-        const uint32_t ring = smem_u32(smem + lay.ring);
-        const uint32_t bar0 = smem_u32(smem + lay.bars);
-        auto full_bar = [&](int s) { return bar0 + 8u * s; };
-        auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
-        const int nstages = (nrows + RT_STAGE_ROWS - 1) / RT_STAGE_ROWS;
-        volatile int* abort_flag = &s_abort;
-        // ---- producer: stage k = rows [16 k, 16 k + 16) of this CTA, ring slot k % S. Its thread
-        // initialises the barriers, copies W_g's rows into shared memory (first in its queue, on
-        // their own barrier) and then streams the stages.
-        const bool producer = tid == NCONS_MAX * 32;
-        const uint32_t wbar = bar0 + 8u * (2 * S);
-        const int WRB = wrow_bytes(d);
-        if (producer) {
-            for (int s = 0; s < S; ++s) {
-                mbar_init(full_bar(s), 1);
-                mbar_init(empty_bar(s), 1);
-            }
-            mbar_init(wbar, 1);
-            mbar_fence_init();
-        }
-        __syncthreads();  // barriers initialised
-        if (producer) {
-            mbar_arrive_expect_tx(wbar, (uint32_t)E * d * 2);
-            const unsigned char* Wb = static_cast<const unsigned char*>(a.Wg);
-            for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(smem) + e * WRB, Wb + (size_t)e * d * 2, d * 2, wbar);
-        }
-        pdl_wait();  // from here on the previous kernel's results (x) are read and outputs written
-        // the next kernel may start now (its CTAs set up, and may read x, while this one streams):
-        // released only after the wait, so every kernel before this one has completed by then
-        pdl_launch_dependents();
-        if (warp == NCONS_MAX) {
-            if (producer) {
-                const unsigned char* xb = static_cast<const unsigned char*>(a.x) + row0 * d * 2;
-                int k = 0;
-                for (; k < nstages; ++k) {
-                    const int s = k % S;
-                    if (!mbar_wait(empty_bar(s), ((k / S) & 1) ^ 1, abort_flag, a.status, (uint64_t)a.wait_limit_ns))
-                        break;
-                    if (k == a.debug_skip && blockIdx.x == 0) continue;  // fault injection: withhold a stage
-                    const int rows = min(RT_STAGE_ROWS, nrows - k * RT_STAGE_ROWS);
-                    const uint32_t bytes = (uint32_t)rows * d * 2;
-                    mbar_arrive_expect_tx(full_bar(s), bytes);
-                    bulk_g2s(ring + s * SB, xb + (size_t)k * SB, bytes, full_bar(s));
-                }
-                if (k < nstages) {  // gave up: let the copies in flight land before moving on
-                    for (int j = max(0, k - S); j < k; ++j)
-                        mbar_wait(full_bar(j % S), (j / S) & 1, nullptr, a.status, 10000000ull);
-                }
-                mbar_wait(wbar, 0, nullptr, a.status, 10000000ull);  // W_g's rows have landed too
-            }
-        } else if (warp < S) {
-            // ---- consumers: warp w owns slot w and takes stages w, w + S, w + 2 S, ...
-            const uint16_t* bgp = static_cast<const uint16_t*>(a.bg);
-            const int g = lane >> 2, tig = lane & 3;
-            const uint4 zero = make_uint4(0, 0, 0, 0);
-            // B fragment of n-tile nt, 32-column chunk c: 8 consecutive bf16 of W_g row nt*8 + g,
-            // columns c*32 + tig*8 (rows past E are zero)
-            const uint4* wfr[2];
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-                wfr[nt] = (nt < NT && nt * 8 + g < E)
-                              ? reinterpret_cast<const uint4*>(smem + (size_t)(nt * 8 + g) * WRB + tig * 16)
-                              : nullptr;
-            const bool w_ok = nstages == 0 || mbar_wait(wbar, 0, abort_flag, a.status, (uint64_t)a.wait_limit_ns);
-            constexpr int NWC = WREG ? RT_WREG_D / 32 : 1;  // register copy of the fragments (WREG)
-            uint4 wreg[NWC];
-            if constexpr (WREG) {
-#pragma unroll
-                for (int c = 0; c < NWC; ++c) wreg[c] = (c < nchunk && wfr[0] && w_ok) ? wfr[0][4 * c] : zero;
-            }
-            for (int k = warp; w_ok && k < nstages; k += S) {
-                const int s = warp;
-                if (!mbar_wait(full_bar(s), (k / S) & 1, abort_flag, a.status, (uint64_t)a.wait_limit_ns)) break;
-                const int rows = min(RT_STAGE_ROWS, nrows - k * RT_STAGE_ROWS);
-                const bool vA = g < rows, vB = g + 8 < rows;
-                const unsigned char* st = smem + lay.ring + (size_t)s * SB;
-                const uint4* pA = reinterpret_cast<const uint4*>(st + (size_t)g * d * 2) + tig;
-                const uint4* pB = reinterpret_cast<const uint4*>(st + (size_t)(g + 8) * d * 2) + tig;
-                // four independent accumulator chains (K steps 4j + q go to chain q), summed at the end
-                float part[2][4][4];
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) part[nt][q][i] = 0.f;
-                if constexpr (WREG) {
-#pragma unroll
-                    for (int c = 0; c < NWC; c += 2) {  // one n-tile, fragments in registers
-                        if (c < nchunk) {
-                            const uint4 xa0 = vA ? pA[4 * c] : zero, xa1 = vA ? pA[4 * c + 4] : zero;
-                            const uint4 xb0 = vB ? pB[4 * c] : zero, xb1 = vB ? pB[4 * c + 4] : zero;
-                            const uint4 w0 = wreg[c], w1 = wreg[c + 1];
-                            mma_bf16_16816(part[0][0], xa0.x, xb0.x, xa0.y, xb0.y, w0.x, w0.y);
-                            mma_bf16_16816(part[0][1], xa0.z, xb0.z, xa0.w, xb0.w, w0.z, w0.w);
-                            mma_bf16_16816(part[0][2], xa1.x, xb1.x, xa1.y, xb1.y, w1.x, w1.y);
-                            mma_bf16_16816(part[0][3], xa1.z, xb1.z, xa1.w, xb1.w, w1.z, w1.w);
-                        }
-                    }
-                } else {
-                    for (int c = 0; c < nchunk; c += 2) {  // d % 64 == 0: nchunk is even
-                        const uint4 xa0 = vA ? pA[4 * c] : zero, xa1 = vA ? pA[4 * c + 4] : zero;
-                        const uint4 xb0 = vB ? pB[4 * c] : zero, xb1 = vB ? pB[4 * c + 4] : zero;
-#pragma unroll
-                        for (int nt = 0; nt < 2; ++nt) {
-                            if (nt < NT) {
-                                const uint4 w0 = wfr[nt] ? wfr[nt][4 * c] : zero;
-                                const uint4 w1 = wfr[nt] ? wfr[nt][4 * c + 4] : zero;
-                                mma_bf16_16816(part[nt][0], xa0.x, xb0.x, xa0.y, xb0.y, w0.x, w0.y);
-                                mma_bf16_16816(part[nt][1], xa0.z, xb0.z, xa0.w, xb0.w, w0.z, w0.w);
-                                mma_bf16_16816(part[nt][2], xa1.x, xb1.x, xa1.y, xb1.y, w1.x, w1.y);
-                                mma_bf16_16816(part[nt][3], xa1.z, xb1.z, xa1.w, xb1.w, w1.z, w1.w);
-                            }
-                        }
-                    }
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(empty_bar(s));  // the stage is no longer read
-                float acc[2][4];
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        acc[nt][i] = (part[nt][0][i] + part[nt][1][i]) + (part[nt][2][i] + part[nt][3][i]);
-                // D fragment: acc[nt][0..1] = row g, experts nt*8 + 2*tig + {0,1}; [2..3] = row g+8
-                float2 lnA = make_float2(0.f, 1.f), lnB = make_float2(0.f, 1.f);  // (mean, rstd)
-                if (a.ln_stats) {
-                    const int64_t tA = row0 + (int64_t)k * RT_STAGE_ROWS + g;
-                    if (vA) lnA = a.ln_stats[tA];
-                    if (vB) lnB = a.ln_stats[tA + 8];
-                }
-                float bA = -INFINITY, bB = -INFINITY;
-                int eA = 0x7fffffff, eB = 0x7fffffff;
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt) {
-#pragma unroll
-                    for (int j = 0; j < 2; ++j) {
-                        const int e = nt * 8 + 2 * tig + j;
-                        if (nt < NT && e < E) {
-                            const uint16_t bb = bgp[e];
-                            const float bias = __uint_as_float((uint32_t)bb << 16);
-                            float lA = acc[nt][j], lB = acc[nt][2 + j];
-                            if (a.ln_stats) {  // W_g LN(y) = rstd (W_g y - mean g)
-                                const float ge = a.ln_wsum[e];
-                                lA = lnA.y * fmaf(-lnA.x, ge, lA);
-                                lB = lnB.y * fmaf(-lnB.x, ge, lB);
-                            }
-                            arg_better(bA, eA, lA + bias, e);
-                            arg_better(bB, eB, lB + bias, e);
-                        }
-                    }
-                }
-#pragma unroll
-                for (int off = 1; off <= 2; off <<= 1) {
-                    const float ovA = __shfl_xor_sync(0xffffffffu, bA, off);
-                    const int oeA = __shfl_xor_sync(0xffffffffu, eA, off);
-                    const float ovB = __shfl_xor_sync(0xffffffffu, bB, off);
-                    const int oeB = __shfl_xor_sync(0xffffffffu, eB, off);
-                    arg_better(bA, eA, ovA, oeA);
-                    arg_better(bB, eB, ovB, oeB);
-                }
-                if (eA > E - 1) eA = 0;  // only reachable with non-finite logits
-                if (eB > E - 1) eB = 0;
-                if (a.cls_stride > 0) {  // class tokens: group E, outside every expert's ballot
-                    const int64_t tA = row0 + (int64_t)k * RT_STAGE_ROWS + g;
-                    if (tA % a.cls_stride == 0) eA = E;
-                    if ((tA + 8) % a.cls_stride == 0) eB = E;
-                }
-                int rankA = 0, rankB = 0;
-                if (scnt) {
-                    // rank of each row among the stage's earlier rows of its expert, from one ballot
-                    // per expert over the lanes holding rows 0-7 (eA) and rows 8-15 (eB)
-                    unsigned selAA = 0, selBA = 0, selBB = 0;
-                    for (int e = 0; e < E; ++e) {
-                        const unsigned mA = __ballot_sync(0xffffffffu, tig == 0 && vA && eA == e);
-                        const unsigned mB = __ballot_sync(0xffffffffu, tig == 0 && vB && eB == e);
-                        if (eA == e) selAA = mA;
-                        if (eB == e) {
-                            selBA = mA;
-                            selBB = mB;
-                        }
-                        if (lane == 0) scnt[k * CM_MAX_E + e] = (uint16_t)(__popc(mA) + __popc(mB));
-                    }
-                    const unsigned below = (1u << (4 * g)) - 1u;  // lanes of rows before row g
-                    rankA = __popc(selAA & below);
-                    rankB = __popc(selBA) + __popc(selBB & below);
-                }
-                if (tig == 0) {
-                    const int iA = k * RT_STAGE_ROWS + g, iB = iA + 8;
-                    if (vA) record(iA, eA, rankA);
-                    if (vB) record(iB, eB, rankB);
-                }
-            }
-        }
+    // ---------------- router logits + argmax for this CTA's rows
+    float* Wf = reinterpret_cast<float*>(smem);
+    if (a.w_bf16) {  // bf16 router weights on fp32 tokens: widened exactly
+        const uint16_t* W = static_cast<const uint16_t*>(a.Wg);
+        for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = bf16_to_f32(W[i]);
     } else {
-        float* Wf = reinterpret_cast<float*>(smem);
-        if (a.w_bf16) {  // bf16 router weights on fp32 tokens: widened exactly
-            const uint16_t* W = static_cast<const uint16_t*>(a.Wg);
-            for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = bf16_to_f32(W[i]);
-        } else {
-            const float* W = static_cast<const float*>(a.Wg);
-            for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = W[i];
-        }
-        pdl_wait();
-        pdl_launch_dependents();
-        __syncthreads();
-        auto bias_of = [&](int e) -> float {
-            return a.w_bf16 ? bf16_to_f32(static_cast<const uint16_t*>(a.bg)[e]) : static_cast<const float*>(a.bg)[e];
-        };
-        // one row per lane: each lane streams its row in 16-float chunks (float4 loads; the L1
-        // merges the 32 rows' sectors) against W_g broadcast from shared memory, fp32 FMA in k
-        // order, so a warp routes 32 rows with no cross-lane reduction (d % 4 == 0)
-        const float* X = static_cast<const float*>(a.x);
-        for (int b0 = warp * 32; b0 < nrows; b0 += NWARPS * 32) {
-            const int i = b0 + lane;
-            const bool valid = i < nrows;
-            const float4* xr = reinterpret_cast<const float4*>(X + (row0 + (valid ? i : 0)) * d);
-            float acc[CM_MAX_E];
+        const float* W = static_cast<const float*>(a.Wg);
+        for (int i = tid; i < E * d; i += NTHREADS) Wf[i] = W[i];
+    }
+    pdl_wait();
+    pdl_launch_dependents();
+    __syncthreads();
+    auto bias_of = [&](int e) -> float {
+        return a.w_bf16 ? bf16_to_f32(static_cast<const uint16_t*>(a.bg)[e]) : static_cast<const float*>(a.bg)[e];
+    };
+    // one row per lane: each lane streams its row in 16-float chunks (float4 loads; the L1
+    // merges the 32 rows' sectors) against W_g broadcast from shared memory, fp32 FMA in k
+    // order, so a warp routes 32 rows with no cross-lane reduction (d % 4 == 0)
+    const float* X = static_cast<const float*>(a.x);
+    for (int b0 = warp * 32; b0 < nrows; b0 += NWARPS * 32) {
+        const int i = b0 + lane;
+        const bool valid = i < nrows;
+        const float4* xr = reinterpret_cast<const float4*>(X + (row0 + (valid ? i : 0)) * d);
+        float acc[CM_MAX_E];
 #pragma unroll
-            for (int e = 0; e < CM_MAX_E; ++e) acc[e] = 0.f;
-            for (int k4 = 0; k4 < d / 4; k4 += 4) {
-                float4 xv[4];
+        for (int e = 0; e < CM_MAX_E; ++e) acc[e] = 0.f;
+        for (int k4 = 0; k4 < d / 4; k4 += 4) {
+            float4 xv[4];
 #pragma unroll
-                for (int j = 0; j < 4; ++j) xv[j] = (k4 + j < d / 4) ? xr[k4 + j] : make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int j = 0; j < 4; ++j) xv[j] = (k4 + j < d / 4) ? xr[k4 + j] : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    if (k4 + j < d / 4) {
+            for (int j = 0; j < 4; ++j) {
+                if (k4 + j < d / 4) {
 #pragma unroll
-                        for (int e = 0; e < CM_MAX_E; ++e) {
-                            if (e < E) {
-                                const float4 w = reinterpret_cast<const float4*>(Wf + (size_t)e * d)[k4 + j];
-                                acc[e] = fmaf(xv[j].x, w.x, acc[e]);
-                                acc[e] = fmaf(xv[j].y, w.y, acc[e]);
-                                acc[e] = fmaf(xv[j].z, w.z, acc[e]);
-                                acc[e] = fmaf(xv[j].w, w.w, acc[e]);
-                            }
+                    for (int e = 0; e < CM_MAX_E; ++e) {
+                        if (e < E) {
+                            const float4 w = reinterpret_cast<const float4*>(Wf + (size_t)e * d)[k4 + j];
+                            acc[e] = fmaf(xv[j].x, w.x, acc[e]);
+                            acc[e] = fmaf(xv[j].y, w.y, acc[e]);
+                            acc[e] = fmaf(xv[j].z, w.z, acc[e]);
+                            acc[e] = fmaf(xv[j].w, w.w, acc[e]);
                         }
                     }
                 }
             }
-            if (a.ln_stats) {  // W_g LN(y) = rstd (W_g y - mean g)
-                const float2 st = valid ? a.ln_stats[row0 + i] : make_float2(0.f, 1.f);
-#pragma unroll
-                for (int e = 0; e < CM_MAX_E; ++e)
-                    if (e < E) acc[e] = st.y * fmaf(-st.x, a.ln_wsum[e], acc[e]);
-            }
-            float bv = -INFINITY;
-            int be = 0x7fffffff;
+        }
+        if (a.ln_stats) {  // W_g LN(y) = rstd (W_g y - mean g)
+            const float2 st = valid ? a.ln_stats[row0 + i] : make_float2(0.f, 1.f);
 #pragma unroll
             for (int e = 0; e < CM_MAX_E; ++e)
-                if (e < E) arg_better(bv, be, acc[e] + bias_of(e), e);
-            if (be > E - 1) be = 0;  // only reachable with non-finite logits
-            if (a.cls_stride > 0 && (row0 + i) % a.cls_stride == 0) be = E;  // a class token
-            if (valid) record(i, be, 0);
+                if (e < E) acc[e] = st.y * fmaf(-st.x, a.ln_wsum[e], acc[e]);
         }
+        float bv = -INFINITY;
+        int be = 0x7fffffff;
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e)
+            if (e < E) arg_better(bv, be, acc[e] + bias_of(e), e);
+        if (be > E - 1) be = 0;  // only reachable with non-finite logits
+        if (a.cls_stride > 0 && (row0 + i) % a.cls_stride == 0) be = E;  // a class token
+        if (valid) record(i, be);
     }
     __syncthreads();
 
     // ---------------- this CTA's histogram, and each row's rank among the CTA's earlier rows of
     // its expert (warp match masks, then a per-expert prefix over warps and over passes), which
-    // makes the final order stable. The slots themselves are assigned by the consumer of the
-    // routing (the fc1 epilogue, or route_finalize_kernel): no CTA ever waits for another.
+    // makes the final order stable.
     if (tid < E) a.cta_counts[(size_t)blockIdx.x * CM_MAX_E + tid] = s_count[tid];
-    if (scnt) {
-        // per expert, an exclusive scan of the stage counts (one warp per expert, 32 stages a
-        // step), then rank = the stage's prefix + the rank within the stage
-        const int nst = (nrows + RT_STAGE_ROWS - 1) / RT_STAGE_ROWS;
-        for (int e = warp; e < E; e += NWARPS) {
-            int carry = 0;
-            for (int k0 = 0; k0 < nst; k0 += 32) {
-                const int k = k0 + lane;
-                const int v = k < nst ? scnt[k * CM_MAX_E + e] : 0;
-                int incl = v;
-#pragma unroll
-                for (int off = 1; off < 32; off <<= 1) {
-                    const int o = __shfl_up_sync(0xffffffffu, incl, off);
-                    if (lane >= off) incl += o;
-                }
-                if (k < nst) scnt[k * CM_MAX_E + e] = (uint16_t)(carry + incl - v);
-                carry += __shfl_sync(0xffffffffu, incl, 31);
-            }
-        }
-        __syncthreads();
-        for (int i = tid; i < nrows; i += NTHREADS) {
-            const uint32_t w = sinfo[i];
-            const int e = (int)(w & 0xffu);
-            // class tokens (e == E) and rows a launch that gave up never routed take no slot here
-            a.tinfo[row0 + i] =
-                e < E ? e | ((scnt[(i / RT_STAGE_ROWS) * CM_MAX_E + e] + (int)((w >> 8) & 0xffu)) << 8) : E;
-        }
-        return;
-    }
     const unsigned lt = (1u << lane) - 1u;
     if (tid < CM_MAX_E) s_run[tid] = 0;
     for (int i0 = 0; i0 < nrows; i0 += NTHREADS) {
@@ -470,6 +437,7 @@ __global__ void __launch_bounds__(BF16 ? RT_BF16_THREADS : RT_THREADS) route_ker
         if (warp == NWARPS - 1 && lane < E) s_run[lane] = pre + own;
     }
 }
+
 
 // Slots of one routing range (the same ranges as route_kernel: CTA b owns rows [b chunk, +chunk)):
 // the per-expert sums of the G ranges' histograms before this one and over all (thread b reads row
@@ -572,12 +540,11 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
     const bool bf16 = dtype == CLEARMOE_BF16;
     int occ = 0;
     int64_t want = (int64_t)num_sms * (bf16 ? 1 : 2);  // bf16: one CTA per SM owns the ring
-    // equal ranges over all CTAs (a range's last 16-row stage may be partial)
+    // equal ranges over all CTAs (a range's last block may be partial)
     int64_t ch = (T + want - 1) / want;
     // the shared-memory attribute belongs to a device: set once per device
-    if (smem_attr_once((const void*)route_kernel<true, false>, (int)RT_SMEM_MAX) != cudaSuccess ||
-        smem_attr_once((const void*)route_kernel<true, true>, (int)RT_SMEM_MAX) != cudaSuccess ||
-        smem_attr_once((const void*)route_kernel<false, false>, (int)RT_SMEM_MAX) != cudaSuccess) {
+    if (smem_attr_once((const void*)route_tc_kernel, (int)RTC_SMEM_CAP) != cudaSuccess ||
+        smem_attr_once((const void*)route_f32_kernel, (int)RT_F32_SMEM_MAX) != cudaSuccess) {
         (void)cudaGetLastError();
         return -1;
     }
@@ -592,18 +559,16 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
     static struct { int dev, dtype, d, E; size_t smem; int occ; } cache[64];
     static int ncache = 0;
     for (int iter = 0; iter < 4; ++iter) {
-        const size_t smem = route_smem(dtype, d, E, (int)ch);
+        const size_t smem = bf16 ? route_tc_layout(d).total : route_f32_layout(d, E, (int)ch).total;
         occ = -1;
         for (int i = 0; i < ncache; ++i)
             if (cache[i].dev == dev && cache[i].dtype == dtype && cache[i].d == d && cache[i].E == E &&
                 cache[i].smem == smem)
                 occ = cache[i].occ;
         if (occ < 0) {
-            const void* fn = !bf16 ? (const void*)route_kernel<false, false>
-                             : route_wreg(dtype, d, E) ? (const void*)route_kernel<true, true>
-                                                       : (const void*)route_kernel<true, false>;
+            const void* fn = bf16 ? (const void*)route_tc_kernel : (const void*)route_f32_kernel;
             cudaError_t err = cudaOccupancyMaxActiveBlocksPerMultiprocessorWithFlags(
-                &occ, fn, bf16 ? RT_BF16_THREADS : RT_THREADS, smem, cudaOccupancyDefault);
+                &occ, fn, bf16 ? RTC_THREADS : RT_THREADS, smem, cudaOccupancyDefault);
             if (err != cudaSuccess) return -1;
             if (ncache < 64) cache[ncache++] = {dev, dtype, d, E, smem, occ};
         }
@@ -622,20 +587,29 @@ int route_grid(int64_t T, int d, int E, int dtype, int num_sms, int* grid, int* 
 
 cudaError_t launch_route(const RouteArgs& a, int grid, int chunk, cudaStream_t s) {
     const bool bf16 = a.dtype == CLEARMOE_BF16;
-    const size_t smem = route_smem(a.dtype, a.d, a.E, chunk);  // the attribute is set by route_grid
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(bf16 ? RT_BF16_THREADS : RT_THREADS);
-    cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (!bf16) return cudaLaunchKernelEx(&cfg, route_kernel<false, false>, a, chunk);
-    if (route_wreg(a.dtype, a.d, a.E)) return cudaLaunchKernelEx(&cfg, route_kernel<true, true>, a, chunk);
-    return cudaLaunchKernelEx(&cfg, route_kernel<true, false>, a, chunk);
+    if (!bf16) {  // the attribute is set by route_grid
+        cfg.blockDim = dim3(RT_THREADS);
+        cfg.dynamicSmemBytes = route_f32_layout(a.d, a.E, chunk).total;
+        return cudaLaunchKernelEx(&cfg, route_f32_kernel, a, chunk);
+    }
+    if (a.d % RTC_BK != 0 || a.E > CM_MAX_E || a.T > ((int64_t)1 << 30)) return cudaErrorInvalidValue;
+    RouteTcArgs t;
+    t.r = a;
+    t.chunk = chunk;
+    if (encode_tmap_bf16_chunks(&t.tmX, a.x, a.T, a.d, RTC_BOX_ROWS, route_tc_layout(a.d).nkc) ||
+        encode_tmap_bf16(&t.tmW, a.Wg, a.E, a.d, 16))
+        return cudaErrorInvalidValue;
+    cfg.blockDim = dim3(RTC_THREADS);
+    cfg.dynamicSmemBytes = route_tc_layout(a.d).total;
+    return cudaLaunchKernelEx(&cfg, route_tc_kernel, t);
 }
 
 cudaError_t launch_route_finalize(const RouteArgs& a, int grid, int chunk, cudaStream_t s) {

@@ -523,13 +523,13 @@ typedef CUresult (*PFN_encodeTiled_t)(CUtensorMap*, CUtensorMapDataType, cuuint3
                                       const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                       CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-// Encoded maps are cached by (base, rows, cols, box rows), which determine them entirely: a forward
-// encodes up to ~20 maps, and the driver call costs microseconds each on the host.
+// Encoded maps are cached by (base, rows, cols, box rows, box chunks), which determine them
+// entirely: a forward encodes up to ~20 maps, and the driver call costs microseconds each on the host.
 namespace {
 struct TmapEntry {
     const void* base;
     int64_t rows, cols;
-    int box_rows;
+    int box_rows, box_chunks;
     bool valid;
     CUtensorMap map;
 };
@@ -539,27 +539,41 @@ int g_tmap_next = 0;
 std::mutex g_tmap_mu;
 }  // namespace
 
-static int encode_tmap_bf16_uncached(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows);
+static int encode_tmap_uncached(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows,
+                                int box_chunks);
 
-int encode_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
+static int encode_tmap_cached(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows,
+                              int box_chunks) {
     std::lock_guard<std::mutex> lock(g_tmap_mu);
     for (int i = 0; i < TMAP_CACHE; ++i) {
         const TmapEntry& c = g_tmaps[i];
-        if (c.valid && c.base == base && c.rows == rows && c.cols == cols && c.box_rows == box_rows) {
+        if (c.valid && c.base == base && c.rows == rows && c.cols == cols && c.box_rows == box_rows &&
+            c.box_chunks == box_chunks) {
             *map = c.map;
             return 0;
         }
     }
-    const int rc = encode_tmap_bf16_uncached(map, base, rows, cols, box_rows);
+    const int rc = encode_tmap_uncached(map, base, rows, cols, box_rows, box_chunks);
     if (rc == 0) {
         TmapEntry& c = g_tmaps[g_tmap_next];
-        c = TmapEntry{base, rows, cols, box_rows, true, *map};
+        c = TmapEntry{base, rows, cols, box_rows, box_chunks, true, *map};
         g_tmap_next = (g_tmap_next + 1) % TMAP_CACHE;
     }
     return rc;
 }
 
-static int encode_tmap_bf16_uncached(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
+int encode_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
+    return encode_tmap_cached(map, base, rows, cols, box_rows, 0);
+}
+
+int encode_tmap_bf16_chunks(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows,
+                            int box_chunks) {
+    if (box_chunks < 1 || cols % TC_BK != 0 || box_chunks > cols / TC_BK) return -2;
+    return encode_tmap_cached(map, base, rows, cols, box_rows, box_chunks);
+}
+
+static int encode_tmap_uncached(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows,
+                                int box_chunks) {
     static PFN_encodeTiled_t fn = nullptr;
     if (!fn) {
         void* p = nullptr;
@@ -570,13 +584,24 @@ static int encode_tmap_bf16_uncached(CUtensorMap* map, const void* base, int64_t
             return -1;
         fn = reinterpret_cast<PFN_encodeTiled_t>(p);
     }
-    const cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    const cuuint64_t gstride[1] = {(cuuint64_t)cols * 2};
-    const cuuint32_t box[2] = {(cuuint32_t)TC_BK, (cuuint32_t)box_rows};
-    const cuuint32_t es[2] = {1, 1};
-    const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride, box, es,
-                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    CUresult r;
+    if (box_chunks == 0) {  // [rows x cols]: boxes of 64 columns x box_rows rows
+        const cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+        const cuuint64_t gstride[1] = {(cuuint64_t)cols * 2};
+        const cuuint32_t box[2] = {(cuuint32_t)TC_BK, (cuuint32_t)box_rows};
+        const cuuint32_t es[2] = {1, 1};
+        r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    } else {  // the same matrix as {64 columns, rows, cols / 64 chunks}: boxes of 64 x box_rows x box_chunks
+        const cuuint64_t gdim[3] = {(cuuint64_t)TC_BK, (cuuint64_t)rows, (cuuint64_t)(cols / TC_BK)};
+        const cuuint64_t gstride[2] = {(cuuint64_t)cols * 2, (cuuint64_t)TC_BK * 2};
+        const cuuint32_t box[3] = {(cuuint32_t)TC_BK, (cuuint32_t)box_rows, (cuuint32_t)box_chunks};
+        const cuuint32_t es[3] = {1, 1, 1};
+        r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), gdim, gstride, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    }
     return r == CUDA_SUCCESS ? 0 : -2;
 }
 

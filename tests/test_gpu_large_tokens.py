@@ -1,14 +1,13 @@
-"""GPU parity at a token count where the routing kernel keeps its per-row words in global memory.
+"""GPU parity at a token count where every routing range spans many 128-row blocks.
 
-The routing kernel stores each of its rows' words (expert | rank in the range) and per-stage
-expert counts in shared memory while they fit beside W_g and the eight-stage copy ring. At the
-DeiT-B width (d = 768, bf16, E = 8) that space holds about 2,620 rows per CTA, so above ~398 K
-tokens (152 CTAs) the words go to idx in global memory and the ranks come from the match-mask loop
-instead of the per-stage ballots (Algorithm 3, "sort z by a": the same stable order either way).
-This file runs that path at T = 600,000 (3,948 rows per CTA): routing bit-exact against the oracle
-on every token outside near ties, outputs on a seeded sample plus the whole smallest expert, the
-handle-free routing entry point at the same size, whose idx then carries the packed words between
-its two kernels, and the router inside fc1, whose slot kernel then spans 4,688 ranges."""
+The bf16 routing kernel gives each of its 152 CTAs an equal range of tokens and walks it in
+128-row blocks, carrying each expert's running count from block to block; a token's word is
+expert | rank in the range << 8 (Algorithm 3, "sort z by a": the rank makes the order stable). At
+T = 600,000 a range holds 3,948 rows, i.e. 30 full blocks and a partial one, and the ranks run far
+past one byte. This file checks: routing bit-exact against the oracle on every token outside near
+ties, outputs on a seeded sample plus the whole smallest expert, the handle-free routing entry
+point at the same size, whose idx then carries the packed words between its two kernels, and the
+router inside fc1, whose slot kernel then spans 4,688 ranges."""
 import numpy as np
 import pytest
 import torch
@@ -31,15 +30,11 @@ def large_layer():
     return synth.make_layer(synth.DEIT_BASE_BF16.with_(T=T_LARGE, n_cal=2000, seed=5))
 
 
-def test_rows_per_cta_exceed_shared_memory():
-    """The shape of this file is past the shared-memory limit of the per-row words: 152 equal
-    ranges of 3,948 rows need 3,948 x 4 bytes of words and 247 stages x 16 experts x 2 bytes of
-    stage counts, beyond the 15,736 bytes that W_g's padded rows (8 x 1,600), eight 24 KB stages
-    and 17 barriers leave below the kernel's 220 KB."""
+def test_ranges_span_many_blocks():
+    """The shape of this file: 152 equal ranges of 3,948 rows, 30 full 128-row blocks and a last
+    block of 108 rows (14 boxes of 8 rows, 4 of them past the range's end read and ignored)."""
     chunk = -(-T_LARGE // 152)
-    fixed = 8 * (768 * 2 + 64) + 8 * 16 * 768 * 2 + 17 * 8
-    words = chunk * 4 + -(-chunk // 16) * 16 * 2
-    assert chunk == 3948 and fixed + words > 220 * 1024
+    assert chunk == 3948 and chunk // 128 == 30 and chunk % 128 == 108 and -(-108 // 8) * 8 - 108 == 4
 
 
 def test_forward_at_600k_tokens(large_layer):

@@ -1,9 +1,9 @@
 """GPU parity at the limits of the shapes the library accepts, through the C ABI.
 
-E = 16 experts (the largest; the routing kernel then runs two 8-expert MMA column tiles and the
+E = 16 experts (the largest; the routing kernel's MMA then uses all of its N = 16 columns and the
 fused fc1 epilogue's prefix table is full at 152 ranges x 16), d = 1,024 (the largest bf16 width;
-the routing kernel keeps W_g's fragments in shared memory instead of registers above d = 768, and
-H = 4,096 fills fc1's staged bias), and T = max_tokens of the handle. Routing bit-exact outside
+the routing kernel's stages then hold four 64-column K blocks, three stages beside W_g's 32 KB,
+and H = 4,096 fills fc1's staged bias), and T = max_tokens of the handle. Routing bit-exact outside
 near ties, outputs within the bf16 tolerance against the float64 oracle on every row."""
 import numpy as np
 import pytest
