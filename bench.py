@@ -54,10 +54,10 @@ KERNEL_OF_STAGE = {"route": "cm::route_tc_kernel",
 # capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel's sources
 # it was taken on (source_hash); a different hash means the kernel changed and the figure is void.
 TRAFFIC = {
-    "route": {"bytes": 78.328320e6, "src": "219e320a5465ccec"},
-    "fc1_gelu": {"bytes": 337.895168e6, "src": "ecded5355f57aa4f"},
-    "basis": {"bytes": 315.816192e6, "src": "ecded5355f57aa4f"},
-    "grouped": {"bytes": 426.702848e6, "src": "ecded5355f57aa4f"},
+    "route": {"bytes": 78.880768e6, "src": "81624f31b9fa81cb"},
+    "fc1_gelu": {"bytes": 337.621760e6, "src": "d801f22810b8c94f"},
+    "basis": {"bytes": 316.358912e6, "src": "d801f22810b8c94f"},
+    "grouped": {"bytes": 426.954240e6, "src": "d801f22810b8c94f"},
 }
 
 
