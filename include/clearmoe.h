@@ -281,9 +281,10 @@ int clearmoe_layer_status(clearmoe_layer* layer);
 
 /* Fault injection for tests of the bounded waits: every device-side wait of the routing kernel
  * gives up after wait_limit_ns nanoseconds (default 1e9) and, when phantom_arrivals > 0, the
- * routing withholds the copy of one 16-token stage (in its first CTA), so the wait for it runs
- * out and the call reports CLEARMOE_ETIMEOUT through clearmoe_layer_status; nothing is left in
- * flight and the layer stays usable. phantom_arrivals = 0 restores normal use. */
+ * bf16 routing withholds the copy of its first stage (the first K blocks of its first 128-row block,
+ * in its first CTA), so the MMA thread's wait for it runs out and the call reports
+ * CLEARMOE_ETIMEOUT through clearmoe_layer_status; the kernel lets its other copies in flight land
+ * before it exits, and the layer stays usable. phantom_arrivals = 0 restores normal use. */
 int clearmoe_debug_set_wait(clearmoe_layer* layer, int64_t wait_limit_ns, int32_t phantom_arrivals);
 
 /* Per-stage timing: when n >= 5, clearmoe_ffn_forward records events[0] before its first kernel

@@ -151,10 +151,10 @@ def test_deterministic_and_token_split(workload):
 
 
 def test_bounded_wait_reports_timeout(workload):
-    """The routing kernel's producer withholds one 16-token stage copy on purpose
-    (clearmoe_debug_set_wait), so the bounded mbarrier wait of the consumer warp that owns that
-    stage runs out after 20 ms with nothing in flight: the call reports CLEARMOE_ETIMEOUT through
-    the status word, and the handle computes correct results afterwards."""
+    """The routing kernel's producer withholds its first stage copy on purpose
+    (clearmoe_debug_set_wait), so the MMA thread's bounded mbarrier wait for it runs out after
+    20 ms; the producer lets its other copies land before the CTA exits. The call reports
+    CLEARMOE_ETIMEOUT through the status word, and the handle computes correct results afterwards."""
     L = workload(synth.DEIT_SMALL_BF16)
     D = synth.to_torch(L)
     with handle_for(L) as h:
