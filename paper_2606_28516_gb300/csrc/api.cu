@@ -614,6 +614,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         // x and W1 are ready before the routing (which releases fc1 only after its own wait): the
         // operand loads and MMAs start at once; the epilogue waits for the routing's results
         g.pdl_wait_role = 1;
+        g.epi12 = p1 == 256 && d <= cm::TC2_EPI12_MAX_K;  // short K: the GELU epilogue bounds a tile
         rc = cuda_fail(cm::launch_tc_gemm2(g, L->num_sms, s));
     } else {
         if (encode_tmap_bf16(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
@@ -848,6 +849,7 @@ int clearmoe_ffn_forward_scaled(clearmoe_layer* L, const void* x, int64_t T, con
         g.bias = b1;
         g.C = L->z;
         g.ldc = H;
+        g.epi12 = p1 == 256 && d <= cm::TC2_EPI12_MAX_K;  // short K: the GELU epilogue bounds a tile
         if ((rc = cuda_fail(p1 ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s))))
             return rc;
         mark(L, 2, s);
@@ -1010,6 +1012,7 @@ static int dense_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W
     g.ln_stats = lns;
     g.ln_colsum = lnc;  // the 1-SM kernel: the column sums in the epilogue
     if (ln && pair1 && (rc = ln_fc1_aug(L, g, T, pair1 / 2))) return rc;  // 2-SM: the augmentation block
+    g.epi12 = pair1 == 256 && d <= cm::TC2_EPI12_MAX_K;  // short K: the GELU epilogue bounds a tile
     if ((rc = cuda_fail(pair1 ? cm::launch_tc_gemm2(g, L->num_sms, s) : cm::launch_tc_gemm(g, L->num_sms, s))))
         return rc;
     mark(L, 1, s);

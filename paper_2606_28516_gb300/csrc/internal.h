@@ -203,7 +203,13 @@ struct TcGemmArgs {
     // grouped mode: the z segment's A rows gathered by slot, A row of slot m = a1_rows[m] (perm),
     // by tile::gather4 loads of four rows each; tmA1 then has boxes one row high
     const int32_t* a1_rows;
+    // 2-SM dense mode at 256-wide tiles: 12 epilogue warps (three per TMEM lane quarter) and a 160 KB
+    // operand ring instead of 8 warps and 192 KB, for short K where the epilogue bounds a tile
+    int epi12;
 };
+// fc1 takes the 12-epilogue-warp kernel up to this K (d): there a 256 x 256 tile's MMAs are short
+// beside its bias + GELU epilogue
+constexpr int TC2_EPI12_MAX_K = 512;
 // Rows of one routing range of the router inside fc1 (a CTA's half of a pair tile).
 constexpr int FR_RANGE = 128;
 // Boundary e of a grouped GEMM's groups: offsets[e], or the single group [0, M) without offsets.

@@ -21,8 +21,9 @@
 #include "internal.h"
 
 namespace cm {
-// Tile configuration by pair-tile width BN (256, 192 or 128 columns).
-template <int BN_>
+// Tile configuration by pair-tile width BN (256, 192 or 128 columns) and epilogue warps NEPI (8,
+// or 12 for short K, where the epilogue rather than the MMA bounds a tile).
+template <int BN_, int NEPI_ = 8>
 struct T2 {
     static constexpr int BM = 128;                        // rows per CTA; the pair covers 256
     static constexpr int BN = BN_;                        // columns per pair tile
@@ -31,12 +32,15 @@ struct T2 {
     static constexpr int A_BYTES = BM * BK * 2;           // 16 KB
     static constexpr int B_BYTES = BH * BK * 2;           // 16 KB (BN 256), 12 KB (192), 8 KB (128)
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES = 192 * 1024 / STAGE_BYTES;  // at most 192 KB of operands: 6 / 6 / 8
-    static constexpr int NUM_EPI = 8;                     // two per TMEM lane quarter
+    // at most 192 KB of operands (6 / 6 / 8 stages); 160 KB with 12 epilogue warps (their staging)
+    static constexpr int STAGES = (NEPI_ == 8 ? 192 : 160) * 1024 / STAGE_BYTES;
+    static constexpr int NUM_EPI = NEPI_;                 // two or three per TMEM lane quarter
     static constexpr int WARP_MMA = NUM_EPI, WARP_TMA = NUM_EPI + 1;
     static constexpr int THREADS = 32 * (WARP_TMA + 1);
-    static constexpr int WCOLS = BN / (NUM_EPI / 4);      // columns per epilogue warp
     static constexpr int CW = 32;                         // columns per tensor-memory read
+    static constexpr int NCH = BN / CW;                   // 32-column chunks per tile
+    // chunks of the tile of epilogue warp group g (the warps g * 4 .. g * 4 + 3): [g NCH / G, (g + 1) NCH / G)
+    static constexpr int GROUPS = NUM_EPI / 4;
     static constexpr int SW = 16;                         // columns per staged store pass
     // Staging: 32-byte rows (16 bf16); the two 16-byte chunks of row r swap places when bit 2 of r
     // is set, which makes both the row-wise writes and the 2-lanes-per-row reads conflict-free.
@@ -126,7 +130,11 @@ struct PairTile {
 // Kernel variants: the plain dense and grouped GEMMs, the dense GEMM with the router unit (the
 // router inside fc1), and the grouped GEMM whose z rows are gathered by slot. Each variant is its own
 // instantiation, so the plain kernels carry none of the others' code.
-enum Tc2Var { TC2_PLAIN = 0, TC2_ROUTER = 1, TC2_GATHER = 2 };
+enum Tc2Var { TC2_PLAIN = 0, TC2_ROUTER = 1, TC2_GATHER = 2, TC2_EPI12 = 3 };
+// TC2_EPI12: the plain dense GEMM with 12 epilogue warps (three per TMEM lane quarter) and a 160 KB
+// operand ring, for short K (fc1 at d <= 512), where the epilogue's GELU bounds a tile.
+template <int BN, int VAR>
+using T2v = T2<BN, VAR == TC2_EPI12 ? 12 : 8>;
 
 // Units per 256-row pair tile: the column tiles, plus the router unit when the router runs inside fc1.
 template <int VAR>
@@ -157,12 +165,12 @@ __device__ __forceinline__ PairTile decode_pair(const TcGemmArgs& a, int unit, i
 }
 
 template <int BN_, int MODE, int VAR>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2v<BN_, VAR>::THREADS, 1)
     tc_gemm2_kernel(const __grid_constant__ TcGemmArgs a) {
-    using C = T2<BN_>;
+    using C = T2v<BN_, VAR>;
     constexpr int BM = C::BM, BN = C::BN, BH = C::BH, BK = C::BK, A_BYTES = C::A_BYTES;
     constexpr int STAGE_BYTES = C::STAGE_BYTES, STAGES = C::STAGES, NUM_EPI = C::NUM_EPI;
-    constexpr int WARP_MMA = C::WARP_MMA, WARP_TMA = C::WARP_TMA, WCOLS = C::WCOLS, CW = C::CW, SW = C::SW;
+    constexpr int WARP_MMA = C::WARP_MMA, WARP_TMA = C::WARP_TMA, CW = C::CW;
     constexpr int STG_ROW = C::STG_ROW, STG_BYTES = C::STG_BYTES, BIAS_CAP = C::BIAS_CAP, NBARS = C::NBARS;
     constexpr int TMEM_COLS = C::TMEM_COLS;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -481,7 +489,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
     } else if (warp < NUM_EPI) {
         // ------------------------------------------------ epilogue (both CTAs, own 128 rows)
         const int q = warp & 3;  // a warp reads the TMEM lanes of its index mod 4
-        const int c_lo = (warp >> 2) * WCOLS;
+        // this warp's columns of every tile: chunks [grp NCH / GROUPS, (grp + 1) NCH / GROUPS)
+        const int grp = warp >> 2;
+        const int c_lo = CW * (grp * C::NCH / C::GROUPS), c_hi = CW * ((grp + 1) * C::NCH / C::GROUPS);
         unsigned char* wstg = stg + warp * 32 * STG_ROW;
         // Staging by half warps: the 16 rows of lanes 16 h .. 16 h + 15 as 64-byte rows (a 32-column
         // chunk), 16-byte piece j of row r at piece j ^ ((r >> 1) & 3) (conflict-free for the
@@ -585,7 +595,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T2<BN_>::THREADS, 1)
                     const int64_t o = __shfl_sync(0xffffffffu, orow, 8 * hp + lane / 4);
                     dst_row[hp] = o >= 0 ? static_cast<uint16_t*>(a.C) + o * a.ldc + t.n0 + (lane % 4) * 8 : nullptr;
                 }
-                for (int c = c_lo; c < c_lo + WCOLS; c += CW) {
+                for (int c = c_lo; c < c_hi; c += CW) {
                     uint32_t v[CW];
                     const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c;
                     CM_TMEM_LD_X16(taddr, v);
@@ -726,7 +736,7 @@ int tc2_pick_bn(int mode, int N) {
 
 template <int BN, int MODE, int VAR>
 static cudaError_t launch2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
-    using C = T2<BN>;
+    using C = T2v<BN, VAR>;
     const void* fn = (const void*)tc_gemm2_kernel<BN, MODE, VAR>;
     const cudaError_t e = smem_attr_once(fn, C::SMEM);
     if (e != cudaSuccess) return e;
@@ -753,6 +763,9 @@ template <int BN>
 static cudaError_t launch2_var(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
     if (a.mode == TC_GROUPED)
         return a.a1_rows ? launch2<BN, TC_GROUPED, TC2_GATHER>(a, num_sms, s) : launch2<BN, TC_GROUPED, TC2_PLAIN>(a, num_sms, s);
+    if constexpr (BN == 256) {
+        if (a.epi12) return launch2<BN, TC_DENSE, TC2_EPI12>(a, num_sms, s);
+    }
     return a.fr_E > 0 ? launch2<BN, TC_DENSE, TC2_ROUTER>(a, num_sms, s) : launch2<BN, TC_DENSE, TC2_PLAIN>(a, num_sms, s);
 }
 
@@ -773,6 +786,8 @@ cudaError_t launch_tc_gemm2(const TcGemmArgs& a, int num_sms, cudaStream_t s) {
                        !a.fr_info || !a.fr_counts))
         return cudaErrorInvalidValue;
     if (a.a1_rows && a.mode != TC_GROUPED) return cudaErrorInvalidValue;
+    // twelve epilogue warps: the plain dense GEMM at 256-wide tiles (short-K fc1)
+    if (a.epi12 && (a.mode != TC_DENSE || bn != 256 || a.fr_E > 0)) return cudaErrorInvalidValue;
     if (bn == 256) return launch2_var<256>(a, num_sms, s);
     if (bn == 192) return launch2_var<192>(a, num_sms, s);
     return launch2_var<128>(a, num_sms, s);
