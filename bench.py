@@ -54,10 +54,10 @@ KERNEL_OF_STAGE = {"route": "cm::route_tc_kernel",
 # capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel's sources
 # it was taken on (source_hash); a different hash means the kernel changed and the figure is void.
 TRAFFIC = {
-    "route": {"bytes": 78.880768e6, "src": "81624f31b9fa81cb"},
-    "fc1_gelu": {"bytes": 337.621760e6, "src": "d801f22810b8c94f"},
-    "basis": {"bytes": 316.358912e6, "src": "d801f22810b8c94f"},
-    "grouped": {"bytes": 426.954240e6, "src": "d801f22810b8c94f"},
+    "route": {"bytes": 78.790400e6, "src": "9be00256fafa440d"},
+    "fc1_gelu": {"bytes": 338.251008e6, "src": "24b63d4c739bc1af"},
+    "basis": {"bytes": 315.580416e6, "src": "24b63d4c739bc1af"},
+    "grouped": {"bytes": 427.535104e6, "src": "24b63d4c739bc1af"},
 }
 
 
