@@ -27,6 +27,8 @@ struct clearmoe_layer {
     float* ln_sums;    // [2 hidden + CM_MAX_E]  row sums of W1, then of the router's first matrix
     uint16_t* ln_aug_x;  // bf16 layers: [max_tokens x LN_AUG_K]  fc1's augmentation block, token side
     uint16_t* ln_aug_w;  // bf16 layers: [hidden x LN_AUG_K]      and W1's side
+    float* simt_ws;      // fp32 layers: the SIMT GEMMs' split-K partial tiles [simt_ws_floats]
+    int* simt_cnt;       // fp32 layers: their per-tile counters [simt_cnt_len], zero between launches
     int64_t wait_limit_ns;
     int32_t phantom;  // fault injection: > 0 makes the routing withhold one stage copy
     cm::RouteArgs rt;  // the last routing launch (its consumers reuse the shape)
@@ -50,10 +52,19 @@ int cuda_fail(cudaError_t e) {
     return CLEARMOE_ECUDA;
 }
 
+// The fp32 layers' SIMT GEMMs, with the handle's split-K workspace.
+int launch_simt(clearmoe_layer* L, cm::SimtGemmArgs& g, cudaStream_t s) {
+    g.ws = L->simt_ws;
+    g.ws_floats = L->simt_ws ? cm::simt_ws_floats(L->num_sms) : 0;
+    g.cnt = L->simt_cnt;
+    g.cnt_len = L->simt_cnt ? cm::simt_cnt_len(L->num_sms) : 0;
+    return cuda_fail(cm::launch_simt_gemm(g, s));
+}
+
 void free_ws(clearmoe_layer* L) {
     void* ptrs[] = {L->z,     L->t,          L->idx,   L->perm,   L->inv,     L->counts,
                     L->offsets, L->cta_counts, L->tinfo, L->status, L->ln_stats, L->ln_sums,
-                    L->ln_aug_x, L->ln_aug_w};
+                    L->ln_aug_x, L->ln_aug_w, L->simt_ws, L->simt_cnt};
     for (void* p : ptrs)
         if (p) cudaFree(p);
 }
@@ -89,7 +100,7 @@ int mlp_hidden(clearmoe_layer* L, const void* x, int64_t T, const clearmoe_mlp_r
         g.ldc = nh;
         g.ln_stats = lns;
         g.ln_colsum = lnc;
-        return cuda_fail(cm::launch_simt_gemm(g, s));
+        return launch_simt(L, g, s);
     }
     cm::TcGemmArgs g;
     std::memset(&g, 0, sizeof(g));
@@ -300,7 +311,11 @@ int clearmoe_layer_create(const clearmoe_layer_desc* desc, clearmoe_layer** out)
               cudaMalloc((void**)&L->ln_sums, (2 * (size_t)D.hidden + CM_MAX_E) * 4) == cudaSuccess &&
               (D.dtype != CLEARMOE_BF16 ||
                (cudaMalloc((void**)&L->ln_aug_x, T * cm::LN_AUG_K * 2) == cudaSuccess &&
-                cudaMalloc((void**)&L->ln_aug_w, (size_t)D.hidden * cm::LN_AUG_K * 2) == cudaSuccess));
+                cudaMalloc((void**)&L->ln_aug_w, (size_t)D.hidden * cm::LN_AUG_K * 2) == cudaSuccess)) &&
+              (D.dtype != CLEARMOE_F32 ||
+               (cudaMalloc((void**)&L->simt_ws, (size_t)cm::simt_ws_floats(L->num_sms) * 4) == cudaSuccess &&
+                cudaMalloc((void**)&L->simt_cnt, (size_t)cm::simt_cnt_len(L->num_sms) * 4) == cudaSuccess &&
+                cudaMemset(L->simt_cnt, 0, (size_t)cm::simt_cnt_len(L->num_sms) * 4) == cudaSuccess));
     if (ok) {
         // index workspaces start at zero (valid rows), so no launch ever reads garbage indices
         ok = cudaMemset(L->status, 0, 4) == cudaSuccess && cudaMemset(L->perm, 0, T * 4) == cudaSuccess &&
@@ -520,7 +535,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
             g.ln_stats = L->ln_stats;
             g.ln_colsum = L->ln_sums;
         }
-        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        if ((rc = launch_simt(L, g, s))) return rc;
         mark(L, 2, s);
         if (factored) {  // t = diag(S_r) Vh_r z
             std::memset(&g, 0, sizeof(g));
@@ -533,7 +548,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
             g.scale = S_r;
             g.C = static_cast<float*>(L->t);
             g.ldc = r;
-            if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+            if ((rc = launch_simt(L, g, s))) return rc;
         }
         mark(L, 3, s);
         // out[perm[slot]] = U_r t + W_e^res z per expert sub-batch (folded: W_e^comb z)
@@ -565,7 +580,7 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
         g.c_rows = L->perm;
         g.offsets = L->offsets;
         g.E = G;
-        rc = cuda_fail(cm::launch_simt_gemm(g, s));
+        rc = launch_simt(L, g, s);
         mark(L, 4, s);
         return rc;
     }
@@ -794,7 +809,7 @@ int clearmoe_ffn_forward_scaled(clearmoe_layer* L, const void* x, int64_t T, con
         g.gelu = 1;
         g.C = static_cast<float*>(L->z);
         g.ldc = H;
-        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        if ((rc = launch_simt(L, g, s))) return rc;
         mark(L, 2, s);
         std::memset(&g, 0, sizeof(g));  // t' = diag(S_r) Vh_r z / s_a
         g.A0 = static_cast<const float*>(L->z);
@@ -810,7 +825,7 @@ int clearmoe_ffn_forward_scaled(clearmoe_layer* L, const void* x, int64_t T, con
         g.row_scale_inv = 1;
         g.C = static_cast<float*>(L->t);
         g.ldc = r;
-        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        if ((rc = launch_simt(L, g, s))) return rc;
         mark(L, 3, s);
         std::memset(&g, 0, sizeof(g));  // out = s_a (U_r t' + R z)
         g.A0 = static_cast<const float*>(L->t);
@@ -828,7 +843,7 @@ int clearmoe_ffn_forward_scaled(clearmoe_layer* L, const void* x, int64_t T, con
         g.scale_groups = E;
         g.C = static_cast<float*>(out);
         g.ldc = d;
-        rc = cuda_fail(cm::launch_simt_gemm(g, s));
+        rc = launch_simt(L, g, s);
     } else {
         const int p1 = H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;
         const int p2 = cm::tc2_pick_bn(cm::TC_DENSE, r), p3 = cm::tc2_pick_bn(cm::TC_GROUPED, d);
@@ -975,7 +990,7 @@ static int dense_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W
         g.ldc = H;
         g.ln_stats = lns;
         g.ln_colsum = lnc;
-        if ((rc = cuda_fail(cm::launch_simt_gemm(g, s)))) return rc;
+        if ((rc = launch_simt(L, g, s))) return rc;
         mark(L, 1, s);
         std::memset(&g, 0, sizeof(g));
         g.A0 = static_cast<const float*>(L->z);
@@ -987,7 +1002,7 @@ static int dense_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W
         g.N = d;
         g.C = static_cast<float*>(out);
         g.ldc = d;
-        rc = cuda_fail(cm::launch_simt_gemm(g, s));
+        rc = launch_simt(L, g, s);
         mark(L, 2, s);
         return rc;
     }

@@ -93,7 +93,19 @@ struct SimtGemmArgs {
     // the bias, with (mean, rstd) = ln_stats[A0's row] and c_n = ln_colsum[n] = sum_k B0[n, k]
     const float2* ln_stats;
     const float* ln_colsum;
+    // split K for launches with too few tiles to fill the GPU: the K chain of each tile is cut into
+    // up to SIMT_MAX_SPLIT ranges run by separate blocks, which write fp32 partial tiles to ws
+    // (ws_floats floats); the last block of a tile (counter cnt[tile], cnt_len counters, zero
+    // between launches) adds them in split order and runs the epilogue. Nullable: no split.
+    float* ws;
+    int64_t ws_floats;
+    int* cnt;
+    int cnt_len;
 };
+constexpr int SIMT_MAX_SPLIT = 8;
+// Workspace of the split K: partial tiles of up to 4 blocks per SM of 64 x 64 outputs, and counters.
+inline int64_t simt_ws_floats(int num_sms) { return (int64_t)4 * num_sms * 64 * 64; }
+inline int simt_cnt_len(int num_sms) { return 4 * num_sms; }
 cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s);
 
 cudaError_t launch_layer_norm(const void* y, void* x, int64_t T, int d, int dtype, cudaStream_t s);

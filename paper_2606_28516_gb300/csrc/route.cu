@@ -22,7 +22,8 @@
 //   shared memory, and write idx and the final per-token word. A range's last, partial block loads
 //   only the boxes that hold its rows, so that at most 7 rows past the range are read.
 // fp32 tokens (route_f32_kernel): fp32 FMA on the CUDA cores (an fp32 router decision needs fp32
-//   products), one row per lane, then the ranks from warp match masks.
+//   products), one row per lane, or a row split over up to 32 lanes when a CTA's range is short,
+//   then the ranks from warp match masks.
 // Class tokens (cls_stride > 0, t % cls_stride == 0) skip the router: idx = E, no histogram entry
 // and no rank; their slots T - n_cls + t / cls_stride follow the experts' (the dense path).
 #include <mutex>
@@ -355,28 +356,36 @@ __global__ void __launch_bounds__(RT_THREADS) route_f32_kernel(const RouteArgs a
     auto bias_of = [&](int e) -> float {
         return a.w_bf16 ? bf16_to_f32(static_cast<const uint16_t*>(a.bg)[e]) : static_cast<const float*>(a.bg)[e];
     };
-    // one row per lane: each lane streams its row in 16-float chunks (float4 loads; the L1
-    // merges the 32 rows' sectors) against W_g broadcast from shared memory, fp32 FMA in k
-    // order, so a warp routes 32 rows with no cross-lane reduction (d % 4 == 0)
+    // Lanes per row: with few rows per CTA (small T), each row is split over tpr lanes (a power of
+    // two, tpr x rows <= the CTA's threads), which take its float4 columns in turn and add their
+    // partial logits by shuffles; with many rows, one row per lane (tpr = 1), fp32 FMA in k order
+    // and no cross-lane step. W_g is broadcast from shared memory (d % 4 == 0).
+    int tpr = 1;
+    while (tpr < 32 && nrows * tpr * 2 <= NTHREADS) tpr *= 2;
+    const int rpw = 32 / tpr;  // rows per warp per pass
+    const int sub = lane & (tpr - 1);
     const float* X = static_cast<const float*>(a.x);
-    for (int b0 = warp * 32; b0 < nrows; b0 += NWARPS * 32) {
-        const int i = b0 + lane;
+    const int d4 = d / 4;
+    for (int b0 = warp * rpw; b0 < nrows; b0 += NWARPS * rpw) {
+        const int i = b0 + lane / tpr;
         const bool valid = i < nrows;
         const float4* xr = reinterpret_cast<const float4*>(X + (row0 + (valid ? i : 0)) * d);
         float acc[CM_MAX_E];
 #pragma unroll
         for (int e = 0; e < CM_MAX_E; ++e) acc[e] = 0.f;
-        for (int k4 = 0; k4 < d / 4; k4 += 4) {
+        for (int k4 = sub; k4 < d4; k4 += 4 * tpr) {
             float4 xv[4];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) xv[j] = (k4 + j < d / 4) ? xr[k4 + j] : make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int j = 0; j < 4; ++j)
+                xv[j] = (k4 + j * tpr < d4) ? xr[k4 + j * tpr] : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                if (k4 + j < d / 4) {
+                const int kk = k4 + j * tpr;
+                if (kk < d4) {
 #pragma unroll
                     for (int e = 0; e < CM_MAX_E; ++e) {
                         if (e < E) {
-                            const float4 w = reinterpret_cast<const float4*>(Wf + (size_t)e * d)[k4 + j];
+                            const float4 w = reinterpret_cast<const float4*>(Wf + (size_t)e * d)[kk];
                             acc[e] = fmaf(xv[j].x, w.x, acc[e]);
                             acc[e] = fmaf(xv[j].y, w.y, acc[e]);
                             acc[e] = fmaf(xv[j].z, w.z, acc[e]);
@@ -385,6 +394,11 @@ __global__ void __launch_bounds__(RT_THREADS) route_f32_kernel(const RouteArgs a
                     }
                 }
             }
+        }
+        for (int off = tpr >> 1; off > 0; off >>= 1) {  // every lane of the row ends with the sums
+#pragma unroll
+            for (int e = 0; e < CM_MAX_E; ++e)
+                if (e < E) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], off);
         }
         if (a.ln_stats) {  // W_g LN(y) = rstd (W_g y - mean g)
             const float2 st = valid ? a.ln_stats[row0 + i] : make_float2(0.f, 1.f);
@@ -399,7 +413,7 @@ __global__ void __launch_bounds__(RT_THREADS) route_f32_kernel(const RouteArgs a
             if (e < E) arg_better(bv, be, acc[e] + bias_of(e), e);
         if (be > E - 1) be = 0;  // only reachable with non-finite logits
         if (a.cls_stride > 0 && (row0 + i) % a.cls_stride == 0) be = E;  // a class token
-        if (valid) record(i, be);
+        if (valid && sub == 0) record(i, be);
     }
     __syncthreads();
 

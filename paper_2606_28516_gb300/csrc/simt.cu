@@ -10,6 +10,9 @@
 // bias, GELU or ReLU, per-column scale and per-row scale, and an optional row scatter of C (the
 // unshuffle, step 6). With the LayerNorm folded into A0 (rows of the un-normalised stream y) the
 // epilogue first forms rstd (acc - mean c_n), c_n = sum_k B0[n, k], since W LN(y) = rstd (W y - mean W 1).
+// Launches with too few tiles to fill the GPU split each tile's K chain over several blocks, whose
+// partial sums the tile's last block adds in a fixed order: results are deterministic for a given
+// shape, and the order of the fp32 sum depends on the number of tiles (so on T).
 #include "common.cuh"
 #include "internal.h"
 
@@ -62,13 +65,22 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
     // operand tiles; the next step's values are loaded into registers while this step computes.
     const int kk = tid % SG_K, r0 = tid / SG_K;
     constexpr int RS = 256 / SG_K;
+    // the tile's K chain in SG_K steps (the dense path's group has no first segment), and this
+    // block's range of it: split blockIdx.y of gridDim.y equal parts
+    const bool seg0_on = a.A0 != nullptr && a.K0 > 0 && !(a.offsets && a.dense_last && e == a.E - 1);
+    const int st0 = seg0_on ? (a.K0 + SG_K - 1) / SG_K : 0;
+    const int st1 = (a.A1 != nullptr && a.K1 > 0) ? (a.K1 + SG_K - 1) / SG_K : 0;
+    const int nsplit = gridDim.y, split = blockIdx.y;
+    const int s_lo = (int)((int64_t)(st0 + st1) * split / nsplit), s_hi = (int)((int64_t)(st0 + st1) * (split + 1) / nsplit);
     for (int seg = 0; seg < 2; ++seg) {
         const float* A = seg == 0 ? a.A0 : a.A1;
         const float* B = seg == 0 ? a.B0 : B1;
         const int K = seg == 0 ? a.K0 : a.K1;
         const int64_t lda = seg == 0 ? a.lda0 : a.lda1;
-        if (A == nullptr || K == 0) continue;
-        if (seg == 0 && a.offsets && a.dense_last && e == a.E - 1) continue;  // the dense path: z x W2 alone
+        const int seg_st = seg == 0 ? st0 : st1, seg_base = seg == 0 ? 0 : st0;
+        const int lo = max(s_lo - seg_base, 0), hi = min(s_hi - seg_base, seg_st);
+        if (lo >= hi) continue;
+        const int k_begin = lo * SG_K, k_end = min(hi * SG_K, K);
         int arow[LD];  // this thread's A rows (gathered for fc1), -1 outside the tile
 #pragma unroll
         for (int i = 0; i < LD; ++i) {
@@ -89,15 +101,15 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
                 rb[i] = (n < a.N && k < K) ? B[(int64_t)n * K + k] : 0.f;
             }
         };
-        gload(0);
-        for (int k0 = 0; k0 < K; k0 += SG_K) {
+        gload(k_begin);
+        for (int k0 = k_begin; k0 < k_end; k0 += SG_K) {
 #pragma unroll
             for (int i = 0; i < LD; ++i) {
                 As[kk][r0 + RS * i] = ra[i];
                 Bs[kk][r0 + RS * i] = rb[i];
             }
             __syncthreads();
-            if (k0 + SG_K < K) gload(k0 + SG_K);
+            if (k0 + SG_K < k_end) gload(k0 + SG_K);
 #pragma unroll 8
             for (int k = 0; k < SG_K; ++k) {
                 float av[R], bv[R];
@@ -112,6 +124,31 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
             }
             __syncthreads();
         }
+    }
+    if (nsplit > 1) {
+        // this split's partial tile to the workspace; the tile's last block adds all of them in
+        // split order (a fixed order: deterministic) and runs the epilogue, then clears the counter
+        float* part = a.ws + (int64_t)blockIdx.x * nsplit * (TM * TM);
+#pragma unroll
+        for (int i = 0; i < R; ++i)
+#pragma unroll
+            for (int j = 0; j < R; ++j) part[(int64_t)split * (TM * TM) + (ty * R + i) * TM + tx * R + j] = acc[i][j];
+        __threadfence();
+        __syncthreads();
+        __shared__ int s_last;
+        if (tid == 0) s_last = atomicAdd(a.cnt + blockIdx.x, 1) == nsplit - 1;
+        __syncthreads();
+        if (!s_last) return;
+        __threadfence();
+#pragma unroll
+        for (int i = 0; i < R; ++i)
+#pragma unroll
+            for (int j = 0; j < R; ++j) {
+                float v = 0.f;
+                for (int p = 0; p < nsplit; ++p) v += __ldcg(part + (int64_t)p * (TM * TM) + (ty * R + i) * TM + tx * R + j);
+                acc[i][j] = v;
+            }
+        if (tid == 0) a.cnt[blockIdx.x] = 0;
     }
 #pragma unroll
     for (int i = 0; i < R; ++i) {
@@ -157,10 +194,25 @@ cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
     int n64 = 0, n32 = 0;
     const int64_t b64 = simt_blocks<64>(a, &n64), b32 = simt_blocks<32>(a, &n32);
     if (b64 <= 0) return cudaSuccess;
-    if (b64 < 2 * (int64_t)num_sms)  // too few 64-wide tiles to fill the GPU: 32-wide ones
-        simt_gemm_kernel<32><<<(unsigned)b32, 256, 0, s>>>(a, n32);
+    const bool t32 = b64 < 2 * (int64_t)num_sms;  // too few 64-wide tiles to fill the GPU: 32-wide ones
+    const int64_t blocks = t32 ? b32 : b64;
+    const int tm = t32 ? 32 : 64;
+    // split K while the tiles alone would give fewer than four blocks per SM, each part at least two
+    // SG_K steps, within the workspace
+    const int steps = (a.K0 + SG_K - 1) / SG_K + (a.A1 ? (a.K1 + SG_K - 1) / SG_K : 0);
+    int64_t nsplit = 1;
+    if (a.ws && a.cnt && blocks <= a.cnt_len) {
+        nsplit = (4 * (int64_t)num_sms) / blocks;
+        if (nsplit > SIMT_MAX_SPLIT) nsplit = SIMT_MAX_SPLIT;
+        if (nsplit > steps / 2) nsplit = steps / 2;
+        while (nsplit > 1 && nsplit * blocks * tm * tm > a.ws_floats) --nsplit;
+        if (nsplit < 1) nsplit = 1;
+    }
+    const dim3 grid((unsigned)blocks, (unsigned)nsplit);
+    if (t32)
+        simt_gemm_kernel<32><<<grid, 256, 0, s>>>(a, n32);
     else
-        simt_gemm_kernel<64><<<(unsigned)b64, 256, 0, s>>>(a, n64);
+        simt_gemm_kernel<64><<<grid, 256, 0, s>>>(a, n64);
     return cudaGetLastError();
 }
 
