@@ -150,6 +150,27 @@ def test_deterministic_and_token_split(workload):
     assert T == 12608
 
 
+def test_fp32_split_k_deterministic(workload):
+    """The fp32 layer's SIMT GEMMs split K when their tiles alone would leave the GPU idle (DeiT-T:
+    the basis factor six ways, the grouped GEMM three ways); the tile's last block adds the partial
+    sums in split order. Repeated forwards on one handle (whose per-tile counters clear themselves)
+    are bitwise equal, and a second handle gives the same bits; the T = 1 and T = 300 launches in
+    between split differently and must not disturb the counters."""
+    L = workload(synth.DEIT_TINY_FP32)
+    D = synth.to_torch(L)
+    with handle_for(L) as h:
+        a = run_ffn(h, D).clone()
+        run_ffn(h, D, T=1)
+        run_ffn(h, D, T=300)
+        b = run_ffn(h, D).clone()
+        assert cm.clearmoe_layer_status(h.h) == 0
+    with handle_for(L) as h2:
+        c = run_ffn(h2, D).clone()
+    torch.cuda.synchronize()
+    assert torch.equal(a, b) and torch.equal(a, c)
+    assert torch.isfinite(a).all()
+
+
 def test_bounded_wait_reports_timeout(workload):
     """The routing kernel's producer withholds its first stage copy on purpose
     (clearmoe_debug_set_wait), so the MMA thread's bounded mbarrier wait for it runs out after
