@@ -19,6 +19,11 @@
  *     return; they never synchronise, except clearmoe_layer_status and clearmoe_layer_destroy.
  *   - One handle may be used by one stream at a time: its workspace holds the hidden states and
  *     routing of the last forward.
+ *   - Kernels are launched with programmatic dependent launch: the first kernel of a call may start,
+ *     and read the weights (every tensor argument except x), while the kernel enqueued just before it
+ *     on the same stream is finishing; x is read only after that kernel has completed. So weights
+ *     must not be written by the kernel immediately before the call (any later-enqueued work in
+ *     between, or a synchronisation, is enough).
  *   - Arguments are validated on the host first; on a validation error (EINVAL, EUNSUPPORTED)
  *     nothing is enqueued and the outputs are untouched. CLEARMOE_ECUDA can also come from a
  *     launch after earlier kernels of the same call were enqueued; the outputs are then
