@@ -30,6 +30,11 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SimtGemmArgs a, co
     const int tid = threadIdx.x;
     const int nt = blockIdx.x % n_tiles_n;
     const int mt = blockIdx.x / n_tiles_n;
+    // Launched with programmatic dependent launch: the next kernel may be scheduled once every block
+    // of this one has started, and this one reads nothing (offsets, operands, the split-K workspace
+    // and counters) before the previous kernel has completed.
+    pdl_launch_dependents();
+    pdl_wait();
     int64_t m_lo, m_hi;
     int e = 0;
     if (a.offsets) {
@@ -208,12 +213,17 @@ cudaError_t launch_simt_gemm(const SimtGemmArgs& a, cudaStream_t s) {
         while (nsplit > 1 && nsplit * blocks * tm * tm > a.ws_floats) --nsplit;
         if (nsplit < 1) nsplit = 1;
     }
-    const dim3 grid((unsigned)blocks, (unsigned)nsplit);
-    if (t32)
-        simt_gemm_kernel<32><<<grid, 256, 0, s>>>(a, n32);
-    else
-        simt_gemm_kernel<64><<<grid, 256, 0, s>>>(a, n64);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks, (unsigned)nsplit);
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (t32) return cudaLaunchKernelEx(&cfg, simt_gemm_kernel<32>, a, n32);
+    return cudaLaunchKernelEx(&cfg, simt_gemm_kernel<64>, a, n64);
 }
 
 // ------------------------------------------------------------------ LayerNorm (no affine)
