@@ -43,6 +43,7 @@ struct clearmoe_layer {
 namespace {
 
 using cm::encode_tmap_bf16;
+using cm::encode_tmap_f32;
 
 inline bool misaligned(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
 
@@ -53,6 +54,21 @@ int cuda_fail(cudaError_t e) {
 }
 
 // The fp32 layers' SIMT GEMMs, with the handle's split-K workspace.
+// The fp32 tensor-core GEMMs' tiling: N tile and K split for an [M x N] x K product (row tiles:
+// ceil(M / 128) + extra), with the handle's split workspace and counters (fp32 layers own them).
+cm::TcTf32Plan tf32_plan(const clearmoe_layer* L, cm::TcGemmArgs& g, int N, int K, int64_t M, int extra_tiles) {
+    g.tf32 = 1;
+    g.c_f32 = 1;
+    g.ws = L->simt_ws;
+    g.ws_floats = L->simt_ws ? cm::simt_ws_floats(L->num_sms) : 0;
+    g.cnt = L->simt_cnt;
+    g.cnt_len = L->simt_cnt ? cm::simt_cnt_len(L->num_sms) : 0;
+    const cm::TcTf32Plan p = cm::tc_plan_tf32(N, K, (M + 127) / 128 + extra_tiles, L->num_sms, g.ws_floats, g.cnt_len);
+    g.bn_tf32 = p.bn;
+    g.ksplit = p.ksplit;
+    return p;
+}
+
 int launch_simt(clearmoe_layer* L, cm::SimtGemmArgs& g, cudaStream_t s) {
     g.ws = L->simt_ws;
     g.ws_floats = L->simt_ws ? cm::simt_ws_floats(L->num_sms) : 0;
@@ -484,6 +500,94 @@ static int ffn_router_in_fc1(clearmoe_layer* L, const void* x, int64_t T, const 
     return rc;
 }
 
+// fp32 layers on the tensor cores (the 1-SM kernel's TF32 variant: three TF32 products per K step,
+// section on fp32 accuracy in tc_gemm.cu), after the routing and the finalize kernel:
+//   fc1: z[inv[t]] = GELU(W1 x_t + b1), x read in token order, each row stored at its slot;
+//   basis (factorised): t = diag(S_r) Vh_r z over the routed slots;
+//   grouped: out[perm[slot]] = [t | z] [U_r | W_e^res]^T + b2 per group (materialised: [z | z] x
+//   [W_sh | W_e^res]; folded: z x W_e^comb alone; class tokens: z x W2 alone).
+// Needs d, H (and r when factorised) multiples of 16; the caller falls back to the SIMT kernels
+// otherwise.
+static bool f32_tc_ok(int d, int H, int r, bool factored) {
+    return d % 16 == 0 && H % 16 == 0 && (!factored || r % 16 == 0);
+}
+
+static int ffn_f32_tc(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1, const void* U_r,
+                      const float* S_r, const void* Vh_r, const void* W_sh, const void* const* residual_e, int E,
+                      int r, int64_t n_cls, int G, const void* b2, const void* W2, void* out, cudaStream_t s) {
+    const bool factored = U_r != nullptr;
+    const bool materialized = !factored && W_sh != nullptr;
+    const int d = L->desc.d, H = L->desc.hidden;
+    int rc;
+    cm::TcGemmArgs g;
+    std::memset(&g, 0, sizeof(g));
+    g.status = L->status;
+    g.wait_limit_ns = L->wait_limit_ns;
+    const int bn1 = tf32_plan(L, g, H, d, T, 0).bn;
+    if (encode_tmap_f32(&g.tmA0, x, T, d, 128) || encode_tmap_f32(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
+    g.mode = cm::TC_DENSE;
+    g.epi = cm::TC_EPI_BIAS_GELU;
+    g.M = T;
+    g.N = H;
+    g.K0 = d;
+    g.bias = b1;
+    g.rows = L->inv;  // token t's row goes to its slot
+    g.C = L->z;
+    g.ldc = H;
+    if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
+    mark(L, 2, s);
+    if (factored && T - n_cls > 0) {
+        cm::TcGemmArgs g2;
+        std::memset(&g2, 0, sizeof(g2));
+        g2.status = L->status;
+        g2.wait_limit_ns = L->wait_limit_ns;
+        const int64_t M2 = T - n_cls;  // the routed slots (class tokens' follow them)
+        const int bn2 = tf32_plan(L, g2, r, H, M2, 0).bn;
+        if (encode_tmap_f32(&g2.tmA0, L->z, M2, H, 128) || encode_tmap_f32(&g2.tmB0, Vh_r, r, H, bn2))
+            return CLEARMOE_ECUDA;
+        g2.mode = cm::TC_DENSE;
+        g2.epi = cm::TC_EPI_SCALE;
+        g2.M = M2;
+        g2.N = r;
+        g2.K0 = H;
+        g2.scale = S_r;
+        g2.C = L->t;
+        g2.ldc = r;
+        if ((rc = cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s)))) return rc;
+    }
+    mark(L, 3, s);
+    cm::TcGemmArgs g3;
+    std::memset(&g3, 0, sizeof(g3));
+    g3.status = L->status;
+    g3.wait_limit_ns = L->wait_limit_ns;
+    const int bn3 = tf32_plan(L, g3, d, (factored ? r : materialized ? H : 0) + H, T, G).bn;
+    if ((factored && (encode_tmap_f32(&g3.tmA0, L->t, T, r, 128) || encode_tmap_f32(&g3.tmB0, U_r, d, r, bn3))) ||
+        (materialized && (encode_tmap_f32(&g3.tmA0, L->z, T, H, 128) || encode_tmap_f32(&g3.tmB0, W_sh, d, H, bn3))) ||
+        encode_tmap_f32(&g3.tmA1, L->z, T, H, 128))
+        return CLEARMOE_ECUDA;
+    for (int e = 0; e < E; ++e)
+        if (encode_tmap_f32(&g3.tmB1[e], residual_e[e], d, H, bn3)) return CLEARMOE_ECUDA;
+    if (n_cls > 0) {  // the dense path's group: W2
+        if (encode_tmap_f32(&g3.tmB1[E], W2, d, H, bn3)) return CLEARMOE_ECUDA;
+        g3.dense_last = 1;
+    }
+    g3.mode = cm::TC_GROUPED;
+    g3.epi = cm::TC_EPI_SCATTER;
+    g3.M = T;
+    g3.N = d;
+    g3.K0 = factored ? r : materialized ? H : 0;  // folded: the K chain is z x W_e^comb alone
+    g3.K1 = H;
+    g3.offsets = L->offsets;
+    g3.E = G;
+    g3.rows = L->perm;
+    g3.out_bias = b2;
+    g3.C = out;
+    g3.ldc = d;
+    rc = cuda_fail(cm::launch_tc_gemm(g3, L->num_sms, s));
+    mark(L, 4, s);
+    return rc;
+}
+
 static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1,
                     const void* U_r, const float* S_r, const void* Vh_r, const void* W_sh,
                     const void* const* residual_e, const clearmoe_router* router, int E, int r,
@@ -516,6 +620,9 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     if (!fused && (rc = do_finalize(L, s))) return rc;
     mark(L, 1, s);
 
+    if (!bf16 && !ln && f32_tc_ok(d, H, r, factored))
+        return ffn_f32_tc(L, x, T, W1, b1, U_r, S_r, Vh_r, W_sh, residual_e, E, r, n_cls, G, b2,
+                          opt ? opt->W2 : nullptr, out, s);
     if (!bf16) {
         cm::SimtGemmArgs g;
         std::memset(&g, 0, sizeof(g));

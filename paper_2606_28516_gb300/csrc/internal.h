@@ -218,6 +218,21 @@ struct TcGemmArgs {
     // 2-SM dense mode at 256-wide tiles: 12 epilogue warps (three per TMEM lane quarter) and a 160 KB
     // operand ring instead of 8 warps and 192 KB, for short K where the epilogue bounds a tile
     int epi12;
+    // 1-SM kernel, dense and grouped modes: fp32 operands (tensor maps from encode_tmap_f32) on the
+    // TF32 tensor cores with three products per K step (hi hi + hi lo + lo hi, each fp32 operand split
+    // into a TF32 part and its remainder in shared memory); bias, out_bias and C are fp32 (c_f32
+    // set), GELU is gelu_erf; no LayerNorm fold
+    int tf32;
+    // fp32 (TF32) variant: each tile's K blocks split into ksplit ranges (> 1 when tiles alone leave
+    // SMs idle), one unit each; a unit stores its fp32 partial tile in ws ([tiles x ksplit x 128 x BN]),
+    // and the tile's last unit (cnt[tile] counts arrivals and is reset by it) adds the partials in
+    // split order and runs the epilogue: deterministic for a given shape
+    int ksplit;
+    int bn_tf32;  // the N tile the B maps were encoded for (tc_plan_tf32)
+    float* ws;
+    int64_t ws_floats;
+    int* cnt;
+    int cnt_len;
 };
 // fc1 takes the 12-epilogue-warp kernel up to this K (d): there a 256 x 256 tile's MMAs are short
 // beside its bias + GELU epilogue
@@ -239,6 +254,15 @@ __device__ __forceinline__ float tc_row_scale(const TcGemmArgs& a, int64_t m) {
 }
 #endif
 int tc_pick_bn(int mode, int N);
+// N tile and K split of the 1-SM kernel's fp32 (TF32) variant for an [m_tiles x 128] x N x K
+// product: of the widths 128, 64, 32, 16 dividing N, the one (with the K split that fills the SMs,
+// at most 8 ways, at least 4 K blocks each, within ws_floats and cnt_len) whose busiest SM moves
+// the fewest bytes; bn = 0 if none divides N
+struct TcTf32Plan {
+    int bn;
+    int ksplit;
+};
+TcTf32Plan tc_plan_tf32(int N, int K, int64_t m_tiles, int num_sms, int64_t ws_floats, int cnt_len);
 // 2-SM (cta_group::2) variant for the dense and grouped modes: 256 x BN tiles per CTA pair, BN =
 // tc2_pick_bn(mode, N) (256, 192 or 128; 0 = shape not supported; each CTA's B box is BN / 2 rows).
 // Its bias + GELU and column-scale epilogues stage the vector in shared memory (N <= TC2_BIAS_CAP).
@@ -263,5 +287,8 @@ int encode_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t c
 // contiguous bytes of each of its rows.
 int encode_tmap_bf16_chunks(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows,
                             int box_chunks);
+// Encode a 2-D fp32 row-major [rows x cols] tensor map (cols % 4 == 0), box {32, box_rows}
+// (128-byte rows), 128-byte swizzle.
+int encode_tmap_f32(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows);
 
 }  // namespace cm
