@@ -45,8 +45,10 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # the GB300's nominal figures (HBM3e ~7.9 TB/s; dense bf16 2.25 PFLOP/s), reported beside the
 # measured peaks for context
 NOMINAL_PEAKS = {"hbm_gbs": 7900.0, "bf16_tflops": 2250.0}
-# fp32 CUDA-core peak of the fp32 layer: 152 SMs x 128 fp32 lanes x 2 FLOP (FMA) x 2.07 GHz
-FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+# The fp32 layer's GEMMs run on the TF32 tensor cores, three TF32 products per fp32 product: their
+# peak in fp32 FLOP/s is the measured bf16 peak x the nominal TF32 / bf16 ratio (1.1 / 2.25 PFLOP/s
+# dense) / 3
+TF32X3_OF_BF16 = 1.1 / 2.25 / 3
 STAGES = ("route", "fc1_gelu", "basis", "grouped")
 KERNEL_OF_STAGE = {"route": "cm::route_tc_kernel",
                    "fc1_gelu": "cm::tc_gemm2_kernel<256, 0, 0> (2-SM dense, rows stored at their routing slots)",
@@ -424,7 +426,8 @@ def stage_summary(s, stage_ms, pk, floor_us=None):
                                tensor_frac_sustained=tf / pk["bf16_tflops_sustained"],
                                tensor_frac_nominal=tf / NOMINAL_PEAKS["bf16_tflops"])
             else:
-                out[st]["alu_frac"] = tf / FP32_ALU_TFLOPS
+                out[st].update(tensor_frac=tf / (pk["bf16_tflops"] * TF32X3_OF_BF16),
+                               tensor_frac_sustained=tf / (pk["bf16_tflops_sustained"] * TF32X3_OF_BF16))
     return out
 
 
@@ -456,11 +459,13 @@ def layer_block(s, D, h, cm, args, world, dist, flush, stream, pk):
     if s.dtype == "bf16":
         res["layer_roofline_frac"] = layer_roofline_s(s, pk, "bf16_tflops") / (mean_ms / 1e3)
         res["layer_roofline_frac_sustained"] = layer_roofline_s(s, pk) / (mean_ms / 1e3)
-    else:  # exact fp32 on the CUDA cores (no tensor path meets 1e-4)
+    else:  # fp32 on the TF32 tensor cores, three products per fp32 product
         tf = layer_flops(s) / (mean_ms * 1e-3) / 1e12
-        res["roofline"] = {"bound": "alu", "achieved": tf, "peak": FP32_ALU_TFLOPS, "unit": "TFLOP/s",
-                           "frac": tf / FP32_ALU_TFLOPS,
-                           "peak_source": "152 SMs x 128 fp32 lanes x 2 FLOP x 2.07 GHz (nominal)"}
+        peak = pk["bf16_tflops"] * TF32X3_OF_BF16
+        res["roofline"] = {"bound": "tensor", "achieved": tf, "peak": peak, "unit": "TFLOP/s",
+                           "frac": tf / peak,
+                           "peak_source": "measured burst bf16 x nominal TF32 / bf16 (1.1 / 2.25) / 3 (three "
+                                          "TF32 products per fp32 product)"}
     return res, out
 
 
@@ -910,18 +915,26 @@ def main():
         roof = {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s"}
     else:  # the stage pass is sub-second: the burst peak; the sustained one beside it
         ach = work[dom]["flops"] / dur_s / 1e12
-        roof = {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
-                "frac_sustained": ach / pk["bf16_tflops_sustained"]}
+        scale = 1.0 if s.dtype == "bf16" else TF32X3_OF_BF16  # fp32: three TF32 products each
+        roof = {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops"] * scale, "unit": "TFLOP/s",
+                "frac_sustained": ach / (pk["bf16_tflops_sustained"] * scale)}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    tr = TRAFFIC.get(dom)
+    # the traffic table and kernel names are the bf16 layer's (the DeiT-B capture)
+    tr = TRAFFIC.get(dom) if s.dtype == "bf16" else None
     roof["traffic"] = tr["bytes"] if tr and tr["src"] == source_hash(dom) else None
     if tr and roof["traffic"] is None:
         roof["traffic_note"] = ("the kernel's sources changed after its ncu capture "
                                 f"(hash {source_hash(dom)} vs {tr['src']}): not re-captured yet")
-    roof["kernel"] = KERNEL_OF_STAGE[dom]
-    roof["peak_source"] = (f"{pk_src} ({'burst bf16: the stage pass is sub-second' if roof['bound'] == 'tensor' else 'HBM copy'})")
+    if s.dtype == "bf16":
+        roof["kernel"] = KERNEL_OF_STAGE[dom]
+        roof["peak_source"] = (f"{pk_src} ({'burst bf16: the stage pass is sub-second' if roof['bound'] == 'tensor' else 'HBM copy'})")
+    else:
+        roof["kernel"] = ("cm::route_f32_kernel" if dom == "route" else
+                          "cm::tc_gemm_kernel<BN, mode, true> (fp32 operands, three TF32 products)")
+        roof["peak_source"] = (f"{pk_src} (HBM copy)" if dom == "route" else
+                               f"{pk_src} burst bf16 x nominal TF32 / bf16 (1.1 / 2.25) / 3")
     for st in STAGES:  # per-kernel DRAM traffic where the committed capture still applies
-        t = TRAFFIC.get(st)
+        t = TRAFFIC.get(st) if s.dtype == "bf16" else None
         per_stage[st]["traffic"] = t["bytes"] if t and t["src"] == source_hash(st) else None
 
     cpu = None
