@@ -1082,6 +1082,42 @@ static int dense_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W
     if (ln && (rc = ln_prep(L, x, T, W1, nullptr, 0, s))) return rc;  // x is y: LN(y) folded into fc1
     const float2* lns = ln ? L->ln_stats : nullptr;
     const float* lnc = ln ? L->ln_sums : nullptr;
+    if (L->desc.dtype == CLEARMOE_F32 && !ln && f32_tc_ok(d, H, 0, false)) {  // TF32 tensor cores
+        cm::TcGemmArgs g;
+        std::memset(&g, 0, sizeof(g));
+        g.status = L->status;
+        g.wait_limit_ns = L->wait_limit_ns;
+        const int bn1 = tf32_plan(L, g, H, d, T, 0).bn;
+        if (encode_tmap_f32(&g.tmA0, x, T, d, 128) || encode_tmap_f32(&g.tmB0, W1, H, d, bn1)) return CLEARMOE_ECUDA;
+        g.mode = cm::TC_DENSE;
+        g.epi = cm::TC_EPI_BIAS_GELU;
+        g.M = T;
+        g.N = H;
+        g.K0 = d;
+        g.bias = b1;
+        g.C = L->z;
+        g.ldc = H;
+        if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
+        mark(L, 1, s);
+        cm::TcGemmArgs g2;
+        std::memset(&g2, 0, sizeof(g2));
+        g2.status = L->status;
+        g2.wait_limit_ns = L->wait_limit_ns;
+        const int bn2 = tf32_plan(L, g2, d, H, T, 0).bn;
+        if (encode_tmap_f32(&g2.tmA0, L->z, T, H, 128) || encode_tmap_f32(&g2.tmB0, W2, d, H, bn2))
+            return CLEARMOE_ECUDA;
+        g2.mode = cm::TC_DENSE;
+        g2.epi = cm::TC_EPI_STORE;
+        g2.out_bias = b2;
+        g2.M = T;
+        g2.N = d;
+        g2.K0 = H;
+        g2.C = out;
+        g2.ldc = d;
+        rc = cuda_fail(cm::launch_tc_gemm(g2, L->num_sms, s));
+        mark(L, 2, s);
+        return rc;
+    }
     if (L->desc.dtype == CLEARMOE_F32) {
         cm::SimtGemmArgs g;
         std::memset(&g, 0, sizeof(g));

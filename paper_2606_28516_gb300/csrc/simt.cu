@@ -2,8 +2,8 @@
 //
 // The fp32 forward's GEMMs run on the tensor cores (three TF32 products per step, tc_gemm.cu) where
 // the shapes allow; this CUDA-core kernel keeps exact fp32 products for the rest: the folded
-// LayerNorm, the scaled-residual form, the MLP router's hidden layer, the fp32 dense FFN, and widths
-// that are not multiples of 16. One tiled kernel covers every product of the layer:
+// LayerNorm, the scaled-residual form, the MLP router's hidden layer, and widths that are not
+// multiples of 16. One tiled kernel covers every product of the layer:
 //   C[m, n] = epi( sum_k A0[rowA(m), k] B0[n, k]  +  sum_k A1[m, k] B1_e[n, k] )
 // with an optional row gather of A0 (fc1 on tokens in expert order), an optional second K
 // segment with a per-expert B (the grouped residual GEMM, Algorithm 3 step 5; with dense_last the
