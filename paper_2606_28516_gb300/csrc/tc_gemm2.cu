@@ -41,10 +41,9 @@ struct T2 {
     static constexpr int NCH = BN / CW;                   // 32-column chunks per tile
     // chunks of the tile of epilogue warp group g (the warps g * 4 .. g * 4 + 3): [g NCH / G, (g + 1) NCH / G)
     static constexpr int GROUPS = NUM_EPI / 4;
-    static constexpr int SW = 16;                         // columns per staged store pass
-    // Staging: 32-byte rows (16 bf16); the two 16-byte chunks of row r swap places when bit 2 of r
-    // is set, which makes both the row-wise writes and the 2-lanes-per-row reads conflict-free.
-    static constexpr int STG_ROW = SW * 2;
+    // Staging: 1 KB per epilogue warp (32 x STG_ROW bytes), which each half warp in turn fills
+    // with its 16 rows of one 32-column chunk as 64-byte rows (layout at the epilogue).
+    static constexpr int STG_ROW = 32;
     static constexpr int STG_BYTES = NUM_EPI * 32 * STG_ROW;
     static constexpr int BIAS_CAP = TC2_BIAS_CAP;         // fp32 bias / scale staged in shared memory
     static constexpr int TAB_CAP = TC2_TAB_CAP;           // routing prefix table (fused fc1)
