@@ -58,10 +58,10 @@ KERNEL_OF_STAGE = {"route": "cm::route_tc_kernel",
 # capture (profiles/clearmoe_kernels_deit_base_T50432_full.md), with the hash of the kernel's sources
 # it was taken on (source_hash); a different hash means the kernel changed and the figure is void.
 TRAFFIC = {
-    "route": {"bytes": 78.700544e6, "src": "5ab9f9c634d9172d"},
-    "fc1_gelu": {"bytes": 337.686272e6, "src": "64b7e4cd54dfe09c"},
-    "basis": {"bytes": 315.97312e6, "src": "64b7e4cd54dfe09c"},
-    "grouped": {"bytes": 427.090944e6, "src": "64b7e4cd54dfe09c"},
+    "route": {"bytes": 78.52416e6, "src": "3deea90ad96906dc"},
+    "fc1_gelu": {"bytes": 338.377472e6, "src": "eb41af172793f61c"},
+    "basis": {"bytes": 316.010752e6, "src": "eb41af172793f61c"},
+    "grouped": {"bytes": 426.028544e6, "src": "eb41af172793f61c"},
 }
 
 
