@@ -281,7 +281,9 @@ int clearmoe_get_routing(clearmoe_layer* layer, int32_t* idx, int32_t* counts, i
                          int32_t* perm, void* stream);
 
 /* Synchronises the device, returns the handle's device status word (CLEARMOE_OK or the first
- * device-side error since the last call, e.g. CLEARMOE_ETIMEOUT) and clears it. */
+ * device-side error since the last call, e.g. CLEARMOE_ETIMEOUT) and clears it; after an error it
+ * also clears the handle's split-K arrival counters, which a GEMM that gave up may have left
+ * part-counted, so that the next calls run on a consistent handle. */
 int clearmoe_layer_status(clearmoe_layer* layer);
 
 /* Fault injection for tests of the bounded waits: every device-side wait of the routing kernel

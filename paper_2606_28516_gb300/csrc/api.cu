@@ -1235,8 +1235,12 @@ int clearmoe_layer_status(clearmoe_layer* L) {
     int32_t st = 0;
     if (cudaMemcpy(&st, L->status, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return CLEARMOE_ECUDA;
     if (st != 0) {
-        // (a routing launch that gave up has already retired its tag: nothing else to reset)
+        // A GEMM whose waits gave up may leave K-split arrival counters part-counted: clear them so
+        // that the next calls start from zero (a routing launch that gave up has already retired its
+        // tag: nothing else to reset).
         if (cudaMemset(L->status, 0, 4) != cudaSuccess) return CLEARMOE_ECUDA;
+        if (L->simt_cnt && cudaMemset(L->simt_cnt, 0, sizeof(int) * cm::simt_cnt_len(L->num_sms)) != cudaSuccess)
+            return CLEARMOE_ECUDA;
         if (cudaDeviceSynchronize() != cudaSuccess) return CLEARMOE_ECUDA;
     }
     return st;
