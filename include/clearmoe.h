@@ -56,7 +56,12 @@ typedef enum { CLEARMOE_F32 = 0, CLEARMOE_BF16 = 1 } clearmoe_dtype;
  * bounded by max_tokens, max_E and max_r. dtype selects the arithmetic:
  *   CLEARMOE_BF16: bf16 storage, fp32 accumulation on the tcgen05 tensor cores; z, the shared-
  *                  basis coefficients t = diag(S_r) Vh_r z and out are stored in bf16.
- *   CLEARMOE_F32:  fp32 storage and fp32 FMA on the CUDA cores (exact-fp32 path).
+ *   CLEARMOE_F32:  fp32 storage; the routing logits in fp32 FMA on the CUDA cores. The GEMMs of
+ *                  the forward and of the dense FFN run on the TF32 tensor cores with each fp32
+ *                  operand split into a TF32 part and its remainder and three products per term
+ *                  (relative error near 2^-21 per product) when d, hidden and r are multiples
+ *                  of 16 and the LayerNorm is not folded; otherwise, and in the other fp32 calls,
+ *                  in exact fp32 FMA on the CUDA cores.
  * Tiling limits (else CLEARMOE_EUNSUPPORTED): bf16 needs d % 64 == 0, d <= 1024, hidden % 64 == 0
  * and r % 16 == 0 per call; fp32 needs d % 4 == 0, d <= 512, hidden % 4 == 0 and r % 4 == 0.
  * max_E <= 16, max_r <= 256, max_tokens <= 2^30. */
