@@ -514,7 +514,8 @@ static bool f32_tc_ok(int d, int H, int r, bool factored) {
 
 static int ffn_f32_tc(clearmoe_layer* L, const void* x, int64_t T, const void* W1, const void* b1, const void* U_r,
                       const float* S_r, const void* Vh_r, const void* W_sh, const void* const* residual_e, int E,
-                      int r, int64_t n_cls, int G, const void* b2, const void* W2, void* out, cudaStream_t s) {
+                      int r, int64_t n_cls, int64_t cls_stride, int G, const void* b2, const void* W2, bool fused,
+                      void* out, cudaStream_t s) {
     const bool factored = U_r != nullptr;
     const bool materialized = !factored && W_sh != nullptr;
     const int d = L->desc.d, H = L->desc.hidden;
@@ -531,7 +532,19 @@ static int ffn_f32_tc(clearmoe_layer* L, const void* x, int64_t T, const void* W
     g.N = H;
     g.K0 = d;
     g.bias = b1;
-    g.rows = L->inv;  // token t's row goes to its slot
+    if (fused) {  // slots from the routing's per-range counts and ranks; writes perm, counts, offsets
+        g.rt_info = L->tinfo;
+        g.rt_counts = L->cta_counts;
+        g.rt_ctas = L->rt_grid;
+        g.rt_chunk = L->rt_chunk;
+        g.rt_E = E;
+        g.rt_perm = L->perm;
+        g.rt_out_counts = L->counts;
+        g.rt_out_offsets = L->offsets;
+        g.rt_cls_stride = cls_stride;
+    } else {
+        g.rows = L->inv;  // token t's row goes to its slot (the finalize kernel's inverse permutation)
+    }
     g.C = L->z;
     g.ldc = H;
     if ((rc = cuda_fail(cm::launch_tc_gemm(g, L->num_sms, s)))) return rc;
@@ -614,15 +627,17 @@ static int ffn_impl(clearmoe_layer* L, const void* x, int64_t T, const void* W1,
     mark(L, 0, s);
     if (ln && (rc = ln_prep(L, x, T, W1, mlp ? mlp->W_in : router->W, mlp ? mlp->hidden : E, s))) return rc;
     if ((rc = do_route(L, x, T, router, mlp, E, cls_stride, s, ln))) return rc;
-    // bf16 with the 2-SM fc1: the fc1 epilogue assigns the slots itself (no finalize launch)
+    // bf16 with the 2-SM fc1, or fp32 on the tensor cores: the fc1 epilogue assigns the slots
+    // itself (no finalize launch)
     const int p1 = bf16 && H <= cm::TC2_BIAS_CAP ? cm::tc2_pick_bn(cm::TC_DENSE, H) : 0;
-    const bool fused = p1 && L->rt_grid <= 256 && L->rt_grid * E <= cm::TC2_TAB_CAP;
+    const bool f32_tc = !bf16 && !ln && f32_tc_ok(d, H, r, factored);
+    const bool fused = (p1 || f32_tc) && L->rt_grid <= 256 && L->rt_grid * E <= cm::TC2_TAB_CAP;
     if (!fused && (rc = do_finalize(L, s))) return rc;
     mark(L, 1, s);
 
-    if (!bf16 && !ln && f32_tc_ok(d, H, r, factored))
-        return ffn_f32_tc(L, x, T, W1, b1, U_r, S_r, Vh_r, W_sh, residual_e, E, r, n_cls, G, b2,
-                          opt ? opt->W2 : nullptr, out, s);
+    if (f32_tc)
+        return ffn_f32_tc(L, x, T, W1, b1, U_r, S_r, Vh_r, W_sh, residual_e, E, r, n_cls, cls_stride, G, b2,
+                          opt ? opt->W2 : nullptr, fused, out, s);
     if (!bf16) {
         cm::SimtGemmArgs g;
         std::memset(&g, 0, sizeof(g));

@@ -69,7 +69,10 @@ struct TcCfg {
                                      : (2 * BN <= 256) ? 256 : 512;
     // + (fp32) the split stages' barriers and the two of the K-split handshake
     static constexpr int NBARS = 2 * STAGES + 5 + (TF32 ? STAGES + 2 : 0);
-    static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + NBARS * 8 + 16 + 4 * 20;
+    // fp32 fc1 with the slots formed in its epilogue: the routing's prefix table [range][expert]
+    // and the expert offsets
+    static constexpr int TAB_BYTES = TF32 ? (TC2_TAB_CAP + CM_MAX_E) * 4 : 0;
+    static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STG_BYTES + TAB_BYTES + NBARS * 8 + 16 + 4 * 20;
 };
 
 struct TileInfo {
@@ -130,7 +133,9 @@ __global__ void __launch_bounds__((MODE == TC_GATHER || TF32) ? TC_THREADS_GATHE
     const uint32_t raw_addr = smem_u32(smem_raw);
     unsigned char* sm = smem_raw + ((1024 - (raw_addr & 1023)) & 1023);
     unsigned char* stg = sm + C::STAGES * C::STAGE_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(stg + C::STG_BYTES);
+    int* s_tab = reinterpret_cast<int*>(stg + C::STG_BYTES);  // fp32 fused slots: [range][expert]
+    int* s_off = s_tab + TC2_TAB_CAP;                            // [expert] offsets
+    uint64_t* bars = reinterpret_cast<uint64_t*>(stg + C::STG_BYTES + C::TAB_BYTES);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::NBARS);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* s_prefix = reinterpret_cast<int*>(tmem_slot + 4);  // [CM_MAX_E + 1]
@@ -186,6 +191,79 @@ __global__ void __launch_bounds__((MODE == TC_GATHER || TF32) ? TC_THREADS_GATHE
     // everything above overlaps the predecessor kernel; from here on its results are read
     pdl_wait();
     if (a.pdl_trigger_late) pdl_launch_dependents();
+    if (TF32 && MODE == TC_DENSE && a.rt_info && warp < TC_NUM_EPI) {
+        // fp32 fc1 storing each token's row at its routing slot (as the 2-SM fc1 does): the
+        // routing's prefix table, by the epilogue warps while the producer and MMA warps start.
+        // Thread c holds range c's counts; per expert an exclusive scan over ranges (warp scans, warp
+        // totals in s_off's tail, named barrier 1 among the epilogue warps).
+        int* s_wt = s_tab + TC2_TAB_CAP - TC_NUM_EPI * CM_MAX_E;  // scratch below the table's end
+        const int c = threadIdx.x;
+        const int E = a.rt_E;
+        int cnt[CM_MAX_E], incl[CM_MAX_E];
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e) cnt[e] = (c < a.rt_ctas && e < E) ? __ldcg(a.rt_counts + (size_t)c * CM_MAX_E + e) : 0;
+        int wt[CM_MAX_E];
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e) {
+            incl[e] = cnt[e];
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, incl[e], off);
+                if (lane >= off) incl[e] += v;
+            }
+            wt[e] = __shfl_sync(0xffffffffu, incl[e], 31);
+        }
+        // the warp totals go to the table's last entries, read back before the table is written
+        asm volatile("bar.sync 1, %0;" ::"n"(TC_NUM_EPI * 32) : "memory");
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e)
+            if (lane == 0 && e < E) s_wt[warp * CM_MAX_E + e] = wt[e];
+        asm volatile("bar.sync 1, %0;" ::"n"(TC_NUM_EPI * 32) : "memory");
+        int before[CM_MAX_E], tot[CM_MAX_E];
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e) {
+            before[e] = incl[e] - cnt[e];
+            tot[e] = 0;
+            if (e < E)
+                for (int w = 0; w < TC_NUM_EPI; ++w) {
+                    const int v = s_wt[w * CM_MAX_E + e];
+                    if (w < warp) before[e] += v;
+                    tot[e] += v;
+                }
+        }
+        asm volatile("bar.sync 1, %0;" ::"n"(TC_NUM_EPI * 32) : "memory");  // scratch read before the table is written
+#pragma unroll
+        for (int e = 0; e < CM_MAX_E; ++e)
+            if (e < E && c < a.rt_ctas) s_tab[c * E + e] = before[e];
+        if (warp == 0) {  // lane e: expert offsets by a scan over experts
+            int te = 0;
+#pragma unroll
+            for (int e = 0; e < CM_MAX_E; ++e)
+                if (e == lane) te = tot[e];
+            int sc = lane < E ? te : 0;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, sc, off);
+                if (lane >= off) sc += v;
+            }
+            if (lane < E) {
+                s_off[lane] = sc - te;
+                if (blockIdx.x == 0) {
+                    a.rt_out_counts[lane] = te;
+                    a.rt_out_offsets[lane] = sc - te;
+                    if (lane == E - 1) {
+                        a.rt_out_offsets[E] = sc;
+                        const int64_t n_cls = n_class_tokens(a.M, a.rt_cls_stride);
+                        if (n_cls > 0) {  // the class tokens' group (the dense path)
+                            a.rt_out_counts[E] = (int32_t)n_cls;
+                            a.rt_out_offsets[E + 1] = sc + (int32_t)n_cls;
+                        }
+                    }
+                }
+            }
+        }
+        asm volatile("bar.sync 1, %0;" ::"n"(TC_NUM_EPI * 32) : "memory");
+    }
     if (MODE == TC_GROUPED) {
         if (threadIdx.x == 0) {
             int acc = 0;
@@ -408,6 +486,19 @@ __global__ void __launch_bounds__((MODE == TC_GATHER || TF32) ? TC_THREADS_GATHE
             // rows scattered by the grouped epilogue, or by a dense GEMM given a row map (t at its slot)
             if (r < t.rows)
                 orow = (a.epi == TC_EPI_SCATTER || (a.mode == TC_DENSE && a.rows)) ? (int64_t)a.rows[t.m0 + r] : t.m0 + r;
+            if (TF32 && MODE == TC_DENSE && a.rt_info && r < t.rows) {
+                // fp32 fc1: token m's slot from its routing word (expert | rank in its range << 8)
+                const int64_t m = t.m0 + r;
+                const uint32_t w = (uint32_t)a.rt_info[m];
+                const int e = (int)(w & 0xffu);
+                orow = -1;
+                if (a.rt_cls_stride > 0 && m % a.rt_cls_stride == 0)  // class token: the dense path's slots
+                    orow = a.M - n_class_tokens(a.M, a.rt_cls_stride) + m / a.rt_cls_stride;
+                else if (e < a.rt_E)
+                    orow = (int64_t)s_off[e] + s_tab[(int)(m / a.rt_chunk) * a.rt_E + e] + (int)(w >> 8);
+                if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;  // only a routing that gave up
+                if (orow >= 0 && t.n0 == 0 && c_lo == 0 && unit % ksp == 0) a.rt_perm[orow] = (int32_t)m;
+            }
             const float rsc = (a.group_scale && r < t.rows) ? tc_row_scale(a, t.m0 + r) : 1.f;
             if ((uint64_t)orow >= (uint64_t)a.M) orow = -1;
             // the LayerNorm folded into A: (mean, rstd) of the token whose row this lane holds
