@@ -1,6 +1,7 @@
 """bench.py's roofline arithmetic on the CPU: the algorithmic bytes and FLOPs per kernel launch and
 the layer roofline, written out by hand for the DeiT-B layer (T = 50,432, d = 768, H = 3,072,
-E = 8, r = 128, bf16), and the whole-job rate."""
+E = 8, r = 128, bf16), the whole-job rate, and the fp32 layer's tensor peak (three TF32 products
+per fp32 product)."""
 import importlib.util
 import os
 
@@ -48,3 +49,17 @@ def test_layer_roofline_deit_base(bench):
 def test_whole_job_rate(bench):
     assert bench.whole_job_rate(50432, 1, 10, 4.07) == pytest.approx(50432 * 10 / 4.07e-3)
     assert bench.whole_job_rate(50432, 8, 1, 1.0) == pytest.approx(8 * 50432 / 1e-3)  # weak scaling
+
+
+def test_fp32_layer_peak_is_tf32_over_three(bench):
+    """The fp32 layer's GEMMs run as three TF32 products per fp32 product: their peak in fp32
+    FLOP/s is the measured bf16 peak x 1.1 / 2.25 (nominal dense TF32 / bf16) / 3."""
+    assert bench.TF32X3_OF_BF16 == pytest.approx(1.1 / 2.25 / 3)
+    pk = {"bf16_tflops": 1916.0, "bf16_tflops_sustained": 1732.6, "hbm_gbs": 6682.5}
+    s = synth.DEIT_TINY_FP32
+    stages = {"route": [0.010], "fc1_gelu": [0.010], "basis": [0.010], "grouped": [0.010]}
+    out = bench.stage_summary(s, stages, pk)
+    tf = 2 * 788 * 192 * 768 / 10e-6 / 1e12  # fc1 in 10 us
+    assert out["fc1_gelu"]["TFLOP_s"] == pytest.approx(tf)
+    assert out["fc1_gelu"]["tensor_frac"] == pytest.approx(tf / (1916.0 * 1.1 / 2.25 / 3))
+    assert "alu_frac" not in out["fc1_gelu"]
