@@ -501,8 +501,10 @@ static int ffn_router_in_fc1(clearmoe_layer* L, const void* x, int64_t T, const 
 }
 
 // fp32 layers on the tensor cores (the 1-SM kernel's TF32 variant: three TF32 products per K step,
-// section on fp32 accuracy in tc_gemm.cu), after the routing and the finalize kernel:
-//   fc1: z[inv[t]] = GELU(W1 x_t + b1), x read in token order, each row stored at its slot;
+// their accuracy stated at the head of tc_gemm.cu), after the routing:
+//   fc1: z[slot(t)] = GELU(W1 x_t + b1), x read in token order, each row stored at its slot (formed
+//   in the epilogue from the routing's per-range counts and ranks when `fused`, else inv[t] from
+//   the finalize kernel);
 //   basis (factorised): t = diag(S_r) Vh_r z over the routed slots;
 //   grouped: out[perm[slot]] = [t | z] [U_r | W_e^res]^T + b2 per group (materialised: [z | z] x
 //   [W_sh | W_e^res]; folded: z x W_e^comb alone; class tokens: z x W2 alone).
